@@ -1,0 +1,587 @@
+#!/usr/bin/env python3
+"""Benchmark of the experience-path hot path on one GB300 (or N replicas).
+
+Default workload: prioritized replay over 1,000,000 uint8 84x84 frames
+(~7.06 GB in HBM), batch 512, frame stack 4, PER priorities from Exp(1) TD
+errors.  One step = one round of the hot path: stratified sampling through
+the sum-tree, fused frame-stack delivery of obs and next_obs as fp32 with
+collate and importance weights, and the priority update from fresh TD
+errors.  Other workloads (--workload) are for measurement by hand.
+
+Prints ONE JSON line (rank 0).  `value` = delivered GB/s (algorithmic bytes
+of the rounds / device time), `e2e` = the same through the C ABI with host
+buffers (TD errors copied in, the learner batch copied out every step).
+
+--impl reference times the CPU oracle (plain C, all host cores) on the same
+workload and metric; each step is one round of the same per-round work.
+"""
+import argparse
+import ctypes
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+HBM_FALLBACK_GBS = 6800.0
+ALPHA, EPS, BETA = 0.6, 1e-6, 0.4
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        d = json.load(open(p))
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return HBM_FALLBACK_GBS, "fallback"
+
+
+# ----------------------------------------------------------------------------
+# clocks during the timed region: NVML poller (1 ms) + nvidia-smi (100 ms)
+# ----------------------------------------------------------------------------
+REASONS = {0x1: "gpu_idle", 0x2: "applications_clocks_setting",
+           0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown",
+           0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown",
+           0x100: "display_clock_setting"}
+
+
+class Clocks:
+    def __init__(self, cuda_index):
+        self.samples = []
+        self.max_mhz = None
+        self._stop = threading.Event()
+        self._nvml = None
+        self._smi = None
+        self._smi_file = None
+        try:
+            import torch
+            props = torch.cuda.get_device_properties(cuda_index)
+            bus = "%08x:%02x:%02x.0" % (getattr(props, "pci_domain_id", 0),
+                                        props.pci_bus_id, props.pci_device_id)
+            nv = ctypes.CDLL("libnvidia-ml.so.1")
+            if nv.nvmlInit_v2() != 0:
+                raise OSError("nvmlInit")
+            h = ctypes.c_void_p()
+            if nv.nvmlDeviceGetHandleByPciBusId_v2(bus.encode(), ctypes.byref(h)) != 0:
+                raise OSError("nvml handle")
+            mx = ctypes.c_uint()
+            if nv.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(mx)) == 0:
+                self.max_mhz = float(mx.value)
+            self._nvml = (nv, h)
+            self._bus = bus
+        except Exception:
+            self._nvml = None
+
+    def _poll(self):
+        nv, h = self._nvml
+        mhz = ctypes.c_uint()
+        rs = ctypes.c_ulonglong()
+        get_r = getattr(nv, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+            nv.nvmlDeviceGetCurrentClocksThrottleReasons
+        while not self._stop.is_set():
+            if nv.nvmlDeviceGetClockInfo(h, 1, ctypes.byref(mhz)) == 0:
+                r = rs.value if get_r(h, ctypes.byref(rs)) == 0 else 0
+                self.samples.append((float(mhz.value), int(r)))
+            time.sleep(0.001)
+
+    def start(self):
+        if self._nvml:
+            self._t = threading.Thread(target=self._poll, daemon=True)
+            self._t.start()
+        try:
+            self._smi_file = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+            q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+                 "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+                 "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+            self._smi = subprocess.Popen(
+                ["nvidia-smi", "--query-gpu=" + q, "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=self._smi_file, stderr=subprocess.DEVNULL)
+        except Exception:
+            self._smi = None
+
+    def stop(self):
+        self._stop.set()
+        if self._nvml:
+            self._t.join(timeout=1)
+        smi = []
+        if self._smi:
+            self._smi.terminate()
+            try:
+                self._smi.wait(timeout=2)
+            except Exception:
+                self._smi.kill()
+            try:
+                self._smi_file.flush()
+                for line in open(self._smi_file.name):
+                    f = [x.strip() for x in line.split(",")]
+                    if len(f) >= 9:
+                        smi.append(f)
+                os.unlink(self._smi_file.name)
+            except Exception:
+                pass
+        out = {"sm_mhz": None, "sm_max_mhz": self.max_mhz, "reasons": [],
+               "samples": len(self.samples), "smi_samples": len(smi)}
+        if self.samples:
+            out["sm_mhz"] = statistics.median(s[0] for s in self.samples)
+            bits = 0
+            for _, r in self.samples:
+                bits |= r
+            out["reasons"] = sorted(n for b, n in REASONS.items()
+                                    if bits & b and n != "gpu_idle")
+        elif smi:
+            try:
+                out["sm_mhz"] = statistics.median(float(f[1]) for f in smi)
+                out["sm_max_mhz"] = float(smi[0][2])
+                names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown",
+                         "sw_power_cap"]
+                out["reasons"] = sorted({names[i] for f in smi for i in range(4)
+                                         if f[5 + i].lower() == "active"})
+            except Exception:
+                pass
+        return out
+
+
+# ----------------------------------------------------------------------------
+# helpers
+# ----------------------------------------------------------------------------
+def kernel_traffic(kernel, workload):
+    """Per-launch DRAM bytes from the committed ncu summary, or None when the
+    kernel source changed since the counters were taken."""
+    p = os.path.join(ROOT, "profiles", "ncu_traffic.json")
+    try:
+        d = json.load(open(p))[kernel]
+    except Exception:
+        return None
+    src = os.path.join(ROOT, "paper_2609_24456_gb300", "csrc", d["source"])
+    try:
+        h = hashlib.sha256(open(src, "rb").read()).hexdigest()
+    except OSError:
+        return None
+    if h != d.get("source_sha256") or d.get("workload") != workload:
+        return None
+    return d.get("dram_bytes_per_launch")
+
+
+def dev(a, device):
+    import numpy as np
+    import torch
+    a = np.ascontiguousarray(a)
+    if a.dtype == np.uint32:
+        a = a.view(np.int32)
+    return torch.from_numpy(a).to(device)
+
+
+def oracle_threads():
+    import oracle
+    L = oracle.lib()
+    try:
+        fn = L.orc_num_threads
+        fn.restype = ctypes.c_int
+        return int(fn())
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+# ----------------------------------------------------------------------------
+# Workload: prioritized replay, 1,000,000 frames of 84x84, batch 512
+# ----------------------------------------------------------------------------
+class PerReplay:
+    name = "per-replay-1M-84x84-B512"
+    kernel = "k_deliver_stack"
+    kernel_src = "k_deliver.cu"
+
+    def __init__(self, capacity=1_000_000, batch=512, K=4, seed=1235,
+                 out_sets=4):
+        self.cap, self.B, self.K, self.seed = capacity, batch, K, seed
+        self.F = 84 * 84
+        self.R = out_sets
+        D = 1
+        while 32 ** D < capacity:
+            D += 1
+        self.D = D
+        F, B = self.F, batch
+        # algorithmic bytes: unique frame reads (K+1 per sample) + fp32 obs
+        # and next_obs writes + collate/IS scalars (idx 8, q 4 read; isw 4,
+        # action 4, reward 4, done 1 written; action 4, reward 4, done 5 read)
+        self.deliver_bytes = B * ((K + 1) * F + 2 * K * F * 4 + 38)
+        # sampling: one 32-child load per level + the leaf row, writes idx, q
+        self.sample_bytes = B * (32 * 8 * (D - 1) + 32 * 4 + 12)
+        # update: idx, td, leaf read+write, D ancestors read+write (8 B)
+        self.update_bytes = B * (8 + 4 + 8 + 16 * D)
+        self.round_bytes = self.deliver_bytes + self.sample_bytes + self.update_bytes
+
+    def config(self):
+        return {"workload": self.name, "capacity": self.cap, "batch": self.B,
+                "frame": "uint8 84x84", "frame_stack": self.K,
+                "outputs": "obs+next_obs fp32 [B,4,84,84], action, reward, done, isw",
+                "priorities": "PER alpha 0.6 (u32, 2^20 fixed point), beta 0.4",
+                "l2": "ring %.2f GB > L2; outputs rotate over %d buffers (%.0f MB)"
+                      % (self.cap * self.F / 1e9, self.R,
+                         self.R * self.B * 2 * self.K * self.F * 4 / 1e6)}
+
+    # -- GPU arm --------------------------------------------------------------
+    def setup(self, device):
+        import numpy as np
+        import torch
+        from paper_2609_24456_gb300 import edp
+        from paper_2609_24456_gb300 import fixtures as fx
+        self.edp = edp
+        cfg = edp.make_config(self.cap, (1, 84, 84), edp.EDP_XFORM_STACK_F32,
+                              frame_stack=self.K, next_obs=True, prioritized=True,
+                              device=device.index or 0)
+        self.ring = edp.Ring(cfg)
+        ctx = self.ring.ctx
+        _, action, reward, done = fx.dqn_transitions(self.seed, self.cap,
+                                                     with_frames=False)
+        td = fx.td_errors(self.seed, self.cap)
+        chunk = 65536
+        staging = torch.empty((chunk, self.F), dtype=torch.uint8, device=device)
+        qbuf = torch.empty(chunk, dtype=torch.int32, device=device)
+        self.setup_launches = 0
+        for lo in range(0, self.cap, chunk):
+            hi = min(self.cap, lo + chunk)
+            n = hi - lo
+            fx.content_fill_torch(self.seed, lo, staging[:n])
+            edp.edp_priorities_from_td(ctx, dev(td[lo:hi], device), n, ALPHA, EPS, qbuf)
+            edp.edp_ingest(ctx, staging[:n], n, action=dev(action[lo:hi], device),
+                           reward=dev(reward[lo:hi], device),
+                           done=dev(done[lo:hi], device), q=qbuf)
+        del staging
+        edp.edp_sync(ctx)
+        B, K, F = self.B, self.K, self.F
+        self.outs = []
+        for _ in range(self.R):
+            o = dict(idx=torch.empty(B, dtype=torch.int64, device=device),
+                     q=torch.empty(B, dtype=torch.int32, device=device),
+                     obs=torch.empty((B, K, F), device=device),
+                     nxt=torch.empty((B, K, F), device=device),
+                     act=torch.empty(B, dtype=torch.int32, device=device),
+                     rew=torch.empty(B, device=device),
+                     done=torch.empty(B, dtype=torch.uint8, device=device),
+                     isw=torch.empty(B, device=device))
+            o["batch"] = edp.make_batch(o["obs"], o["nxt"], o["act"], o["rew"],
+                                        o["done"], q=o["q"], isw=o["isw"], beta=BETA)
+            self.outs.append(o)
+        self.td_rounds = 64
+        self.td = torch.stack([dev(fx.td_errors(self.seed, B, r), device)
+                               for r in range(self.td_rounds)])
+        self.launches_per_round = 3
+
+    def round(self, r, ev=None):
+        edp, ctx = self.edp, self.ring.ctx
+        o = self.outs[r % self.R]
+        edp.edp_sample(ctx, edp.EDP_SAMPLE_PRIORITIZED, self.B, self.seed, r,
+                       o["idx"], o["q"])
+        edp.edp_deliver(ctx, o["idx"], self.B, o["batch"])
+        if ev:
+            ev[2].record()
+        edp.edp_update_priorities_td(ctx, o["idx"], self.td[r % self.td_rounds],
+                                     self.B, ALPHA, EPS)
+
+    def time_deliver(self, n, mk, stream, graph=True):
+        """Average duration (us) of the delivery kernel launched n times back
+        to back over the batches of the last rounds."""
+        import torch
+        edp, ctx = self.edp, self.ring.ctx
+
+        def body():
+            for r in range(n):
+                o = self.outs[r % self.R]
+                edp.edp_deliver(ctx, o["idx"], self.B, o["batch"])
+        body()
+        torch.cuda.synchronize()
+        if graph:
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, capture_error_mode="thread_local"):
+                body()
+            g.replay()
+            torch.cuda.synchronize()
+        e0, e1 = mk(), mk()
+        e0.record(stream)
+        g.replay() if graph else body()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) * 1e3 / n
+
+    def time_latency(self, n, mk, stream):
+        """Sample -> batch latency (us) of n rounds, events around each."""
+        import torch
+        evs = [(mk(), mk()) for _ in range(n)]
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, capture_error_mode="thread_local"):
+            for r in range(n):
+                evs[r][0].record()
+                self.round(100000 + r, (None, None, evs[r][1]))
+        g.replay()
+        torch.cuda.synchronize()
+        return [a.elapsed_time(b) * 1e3 for a, b in evs]
+
+    def e2e_setup(self, device):
+        import torch
+        B, K, F = self.B, self.K, self.F
+        pin = lambda *s, dt=torch.float32: torch.empty(s, dtype=dt, pin_memory=True)
+        self.h_td = pin(self.td_rounds, B)
+        self.h_td.copy_(self.td.cpu())
+        self.h_out = dict(obs=pin(B, K, F), nxt=pin(B, K, F),
+                          act=pin(B, dt=torch.int32), rew=pin(B),
+                          done=pin(B, dt=torch.uint8), isw=pin(B),
+                          idx=pin(B, dt=torch.int64))
+        self.d_td = torch.empty(B, device=device)
+        self.h2d = B * 4
+        self.d2h = sum(t.numel() * t.element_size() for t in self.h_out.values())
+
+    def e2e_round(self, r):
+        """User path with host buffers: TD errors in, learner batch out."""
+        edp, ctx = self.edp, self.ring.ctx
+        o = self.outs[r % self.R]
+        self.d_td.copy_(self.h_td[r % self.td_rounds], non_blocking=True)
+        edp.edp_sample(ctx, edp.EDP_SAMPLE_PRIORITIZED, self.B, self.seed, r,
+                       o["idx"], o["q"])
+        edp.edp_deliver(ctx, o["idx"], self.B, o["batch"])
+        edp.edp_update_priorities_td(ctx, o["idx"], self.d_td, self.B, ALPHA, EPS)
+        h = self.h_out
+        h["obs"].copy_(o["obs"], non_blocking=True)
+        h["nxt"].copy_(o["nxt"], non_blocking=True)
+        h["act"].copy_(o["act"], non_blocking=True)
+        h["rew"].copy_(o["rew"], non_blocking=True)
+        h["done"].copy_(o["done"], non_blocking=True)
+        h["isw"].copy_(o["isw"], non_blocking=True)
+        h["idx"].copy_(o["idx"], non_blocking=True)
+
+    # -- CPU oracle arm -------------------------------------------------------
+    def cpu_setup(self, host_frames=262_144):
+        import numpy as np
+        import oracle as orc
+        from paper_2609_24456_gb300 import fixtures as fx
+        self.orc = orc
+        self.hcap = min(host_frames, self.cap)
+        rng = np.random.default_rng(self.seed)
+        self.h_frames = rng.integers(0, 256, size=(self.hcap, self.F), dtype=np.uint8)
+        _, a, rw, d = fx.dqn_transitions(self.seed, self.hcap, with_frames=False)
+        self.h_act, self.h_rew, self.h_done = a, rw, d
+        self.st = orc.PerState(self.cap, True)
+        q = orc.priorities_from_td(fx.td_errors(self.seed, self.cap), ALPHA, EPS)
+        orc.ingest_leaves(self.st, 0, q)
+        self.h_tds = [fx.td_errors(self.seed, self.B, r) for r in range(8)]
+        self.cpu_sample = ("per-round work of this workload (B=%d stratified PER over "
+                           "%d leaves, K=%d fp32 stacks + next_obs, IS weights, "
+                           "priority update) reading a %d-frame host ring (%.2f GB)"
+                           % (self.B, self.cap, self.K, self.hcap,
+                              self.hcap * self.F / 1e9))
+
+    def cpu_round(self, r):
+        orc = self.orc
+        idx, q = orc.sample_prioritized_bisect(self.st.leaves, self.B, self.seed, r)
+        orc.is_weights(q, BETA)
+        slots = idx % self.hcap
+        orc.deliver_dqn(self.h_frames, self.h_done, self.h_act, self.h_rew,
+                        self.hcap, self.hcap, self.K, slots)
+        qn = orc.priorities_from_td(self.h_tds[r % 8], ALPHA, EPS)
+        orc.update_leaves(self.st, self.cap, idx, qn)
+
+
+WORKLOADS = {"per1m": PerReplay}
+
+
+# ----------------------------------------------------------------------------
+def time_cpu(wl, budget_s, min_rounds=3):
+    wl.cpu_round(0)
+    n, t0 = 0, time.perf_counter()
+    while n < min_rounds or time.perf_counter() - t0 < budget_s:
+        wl.cpu_round(n + 1)
+        n += 1
+    dt = time.perf_counter() - t0
+    return n, dt
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    wl = WORKLOADS[args.workload]()
+    wl.cpu_setup()
+    for r in range(args.warmup):
+        wl.cpu_round(r)
+    t0 = time.perf_counter()
+    for r in range(args.steps):
+        wl.cpu_round(args.warmup + r)
+    dt = time.perf_counter() - t0
+    gbs = wl.round_bytes * args.steps / dt / 1e9
+    cores = oracle_threads()
+    line = {"metric": "experience-delivery GB/s", "value": gbs, "unit": "GB/s",
+            "impl": "reference", "n_gpus": args.gpus, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": dt * 1e3 / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "u8->f32", "data": "synthetic", "config": wl.config(),
+            "cpu_baseline": {"value": gbs, "unit": "GB/s", "cores": cores,
+                             "kind": "oracle", "sample": wl.cpu_sample},
+            "e2e": {"value": gbs, "unit": "GB/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+    return 0
+
+
+def run_edp(args):
+    import torch
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    device = torch.device("cuda", local)
+    from paper_2609_24456_gb300 import build
+    build.build()
+
+    wl = WORKLOADS[args.workload](**({"capacity": args.capacity} if args.capacity else {}))
+    wl.setup(device)
+    K, W = args.steps, args.warmup
+    mk = lambda: torch.cuda.Event(enable_timing=True, external=True)
+    stream = torch.cuda.current_stream()
+
+    # warm-up rounds (eager), then capture the timed rounds in one graph;
+    # no events inside it (event nodes split the graph and cost several us)
+    for r in range(W):
+        wl.round(K + r)
+    torch.cuda.synchronize()
+    use_graph = not args.no_graph
+    if use_graph:
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, capture_error_mode="thread_local"):
+            for r in range(K):
+                wl.round(r)
+        g.replay()  # upload + warm the graph (rounds are re-timed below)
+        torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks = Clocks(local)
+    clocks.start()
+    time.sleep(0.02)
+    t_start, t_end = mk(), mk()
+    t_start.record(stream)
+    if use_graph:
+        g.replay()
+    else:
+        for r in range(K):
+            wl.round(r)
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    ms = t_start.elapsed_time(t_end)
+    if dist:
+        t = torch.tensor([ms], device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    ms_step = ms / K
+    value = wl.round_bytes * K * world / (ms / 1e3) / 1e9
+    peak, peak_kind = peaks()
+
+    # dominant kernel: the fused delivery, timed back to back on the same
+    # stream (events bracket the launches; the batches are real samples)
+    Kd = min(K, args.kernel_steps)
+    deliver_us = wl.time_deliver(Kd, mk, stream, graph=use_graph)
+    # p50 sample -> batch latency: events before sampling and after delivery
+    Kl = min(K, args.latency_steps)
+    lat_us = sorted(wl.time_latency(Kl, mk, stream))
+    p50 = lat_us[len(lat_us) // 2]
+
+    # end-to-end through the C ABI with host buffers (eager calls)
+    e2e = None
+    if not args.no_e2e:
+        wl.e2e_setup(device)
+        Ke = min(K, args.e2e_steps)
+        for r in range(3):
+            wl.e2e_round(r)
+        torch.cuda.synchronize()
+        if dist:
+            dist.barrier()
+        e0, e1 = mk(), mk()
+        e0.record(stream)
+        for r in range(Ke):
+            wl.e2e_round(r)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ems = e0.elapsed_time(e1)
+        if dist:
+            t = torch.tensor([ems], device=device)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            ems = float(t.item())
+        e2e = {"value": wl.round_bytes * Ke * world / (ems / 1e3) / 1e9,
+               "unit": "GB/s", "h2d_bytes_per_step": wl.h2d,
+               "d2h_bytes_per_step": wl.d2h, "steps": Ke,
+               "ms_per_step": ems / Ke}
+
+    avg_deliver_s = deliver_us / 1e6
+    achieved = wl.deliver_bytes / avg_deliver_s / 1e9
+    roofline = {"bound": "hbm", "achieved": achieved, "peak": peak,
+                "unit": "GB/s", "frac": achieved / peak, "peak_kind": peak_kind,
+                "kernel": wl.kernel,
+                "traffic": kernel_traffic(wl.kernel, wl.name),
+                "algorithmic_bytes_per_launch": wl.deliver_bytes,
+                "avg_launch_us": avg_deliver_s * 1e6, "launches_timed": Kd}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        wl.cpu_setup()
+        n, dt = time_cpu(wl, args.cpu_seconds)
+        cpu = {"value": wl.round_bytes * n / dt / 1e9, "unit": "GB/s",
+               "cores": oracle_threads(), "kind": "oracle",
+               "sample": "%d rounds: %s" % (n, wl.cpu_sample)}
+
+    if rank == 0:
+        line = {"metric": "experience-delivery GB/s", "value": value,
+                "unit": "GB/s", "n_gpus": world, "steps": K, "warmup": W,
+                "ms_per_step": ms_step, "higher_is_better": True,
+                "scaling": "weak", "vs_baseline": None, "dtype": "u8->f32",
+                "data": "synthetic", "config": dict(wl.config(),
+                                                    parallelism="replicas%d" % world,
+                                                    graph=use_graph),
+                "pct_hbm_peak": 100.0 * value / peak,
+                "batches_per_s": K * world / (ms / 1e3),
+                "p50_sample_to_batch_us": p50,
+                "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
+                "gpu_launches": wl.launches_per_round * K,
+                "clocks": clk}
+        print(json.dumps(line))
+    if dist:
+        dist.barrier()
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", default="edp", choices=["edp", "reference"])
+    ap.add_argument("--workload", default="per1m", choices=sorted(WORKLOADS))
+    ap.add_argument("--capacity", type=int, default=0,
+                    help="override the ring capacity (profiling small cases)")
+    ap.add_argument("--no-graph", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--e2e-steps", type=int, default=200)
+    ap.add_argument("--kernel-steps", type=int, default=500)
+    ap.add_argument("--latency-steps", type=int, default=200)
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_edp(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

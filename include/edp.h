@@ -1,0 +1,293 @@
+/*
+ * edp.h -- C ABI of libedp, the GB300 (sm_103a) hot path of an Experience
+ * Data Plane for distributed reinforcement learning.
+ *
+ * The paper (Conduit) exposes the experience path through three control
+ * points -- ingestion, placement, delivery (Sec. 3, "Overview"; Sec. 2.2,
+ * "Experience Path Responsibilities") -- plus the replay-state priority
+ * callback (Appendix C, Invariant 2).  This header maps them to calls:
+ *
+ *   ingestion  -> edp_ingest            (ring scatter; two-tier demotion)
+ *                 edp_gae               (on-policy returns/advantages)
+ *   placement  -> edp_config.hbm_capacity / edp_storage.host_*  (two tiers)
+ *   delivery   -> edp_sample            (uniform, prioritized, shuffle)
+ *                 edp_deliver           (gather + transform + collate)
+ *   callback   -> edp_update_priorities / edp_update_priorities_td
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ * - Plain C types only.  A `edp_stream` is a cudaStream_t (NULL = the legacy
+ *   default stream).  Pointers documented "device" must be device memory of
+ *   the context's GPU; "device-accessible" also admits page-locked host
+ *   memory (cudaHostAlloc / cudaHostRegister, e.g. torch pin_memory), which
+ *   kernels then read or write over the host link.
+ * - Ownership: the caller allocates and frees every buffer it passes (ring
+ *   storage, inputs, outputs).  libedp owns only the context, the priority
+ *   tree and small scratch, allocated through edp_config.alloc (cudaMalloc
+ *   when NULL) and released by edp_destroy.  libedp never frees caller memory.
+ * - Asynchrony: every call validates its arguments on the host, enqueues its
+ *   kernels on `stream` and returns without synchronising.  Results are
+ *   valid once the stream has reached that point.  Host-side cursors
+ *   (head, total) advance at enqueue time, so calls on one context must be
+ *   issued in program order on one stream (or with the caller's own
+ *   cross-stream ordering).
+ * - Errors: argument and state errors are returned synchronously and leave
+ *   the context unchanged.  A CUDA launch error returns EDP_ERR_CUDA.
+ *   Data-dependent faults found on the device (an index out of range, an
+ *   all-zero priority distribution, a bounded wait that expired) never trap:
+ *   the kernel records a flag, writes zeros / -1 for the affected outputs and
+ *   returns; edp_sync reports the flag.  No C++ exception crosses the ABI.
+ *   edp_last_error() describes the last failure of a context.
+ * - Randomness is stateless: each sampling call derives its draws from
+ *   (seed, round, stream id) through Philox4x32-10 (Salmon et al., SC'11),
+ *   so the same arguments give the same indices.
+ */
+#ifndef EDP_H
+#define EDP_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define EDP_ABI_VERSION 1
+
+/* Symbols of the ABI are exported; everything else in libedp is hidden. */
+#if defined(__GNUC__)
+#define EDP_API __attribute__((visibility("default")))
+#else
+#define EDP_API
+#endif
+
+typedef struct edp_ctx edp_ctx;  /* opaque; created by edp_create */
+typedef void *edp_stream;        /* cudaStream_t */
+
+typedef enum {
+  EDP_OK = 0,
+  EDP_ERR_INVALID = 1, /* bad argument, or a device-detected bad index */
+  EDP_ERR_OOM = 2,     /* the allocator returned NULL */
+  EDP_ERR_CUDA = 3,    /* a CUDA runtime error (launch or asynchronous) */
+  EDP_ERR_TIMEOUT = 4, /* a bounded device-side wait expired */
+  EDP_ERR_EMPTY = 5,   /* nothing to sample (no valid transition, or total
+                          priority 0) */
+  EDP_ERR_STATE = 6    /* call not valid for this context's configuration */
+} edp_status;
+
+/* How edp_deliver turns a stored uint8 observation into the learner layout.
+ * All three divide by 255 as one correctly rounded binary32 division
+ * x = fl32(b / 255); bfloat16 outputs are then rounded to nearest even. */
+typedef enum {
+  /* DQN-style frame stack (frame stacking of Mnih et al., Nature 2015):
+   * obs[b][m] = frame of logical offset i-K+1+m, next_obs[b][m] = that of
+   * i-K+2+m; a frame is all zeros when it precedes the oldest stored
+   * transition or an episode end (done == 1) lies between it and the anchor
+   * (exclusive of the anchor).  Output float32 [B][K][obs_h][obs_w]. */
+  EDP_XFORM_STACK_F32 = 0,
+  /* Stored HWC (obs_h x obs_w x obs_c), delivered CHW bfloat16
+   * [B][obs_c][obs_h][obs_w] = RNE_bf16(x). */
+  EDP_XFORM_HWC_CHW_BF16 = 1,
+  /* Stored CHW, delivered bfloat16 [B][obs_c][obs_h][obs_w] =
+   * RNE_bf16(fl32(fl32(x - mean_c) / std_c)), each step rounded. */
+  EDP_XFORM_CHW_NORM_BF16 = 2
+} edp_transform;
+
+typedef enum {
+  /* index_k = slot of logical offset mulhi64(u64(k; seed, round, 0), n_valid)
+   * where n_valid = size - 1 when next_obs is delivered, else size. */
+  EDP_SAMPLE_UNIFORM = 0,
+  /* PER proportional sampling, stratified (Schaul et al., ICLR'16): with
+   * S = total priority, stratum k of B targets t_k = lo_k + mulhi64(u64(k;
+   * seed, round, 1), hi_k - lo_k), lo_k = floor(k S / B), hi_k =
+   * floor((k+1) S / B); the answer is the slot whose priority interval
+   * [prefix(i), prefix(i) + q_i) over physical slot order holds t_k. */
+  EDP_SAMPLE_PRIORITIZED = 1,
+  /* Shuffle of all `size` stored transitions (on-policy mini-batching):
+   * logical offsets sorted by (u64(j; seed, round, 2), j); idx[r] = slot of
+   * the r-th.  Mini-batch m of size M is idx[mM, (m+1)M). */
+  EDP_SAMPLE_PERMUTE = 2
+} edp_sample_mode;
+
+/* Allocator for libedp-owned device memory (256-byte aligned).  Returning
+ * NULL makes the calling function fail with EDP_ERR_OOM. */
+typedef void *(*edp_alloc_fn)(void *user, size_t bytes);
+typedef void (*edp_free_fn)(void *user, void *ptr);
+
+typedef struct {
+  uint64_t capacity;     /* logical ring capacity in transitions, 1..2^32-1 */
+  uint64_t hbm_capacity; /* transitions whose payload (obs, tokens) lives in
+                            HBM.  == capacity: single tier.  < capacity:
+                            two-tier ring -- the newest hbm_capacity
+                            transitions in HBM, the older ones in page-locked
+                            host memory; requires transform CHW_NORM_BF16 */
+  uint32_t obs_c, obs_h, obs_w; /* stored observation shape; obs_bytes =
+                            c*h*w must be a multiple of 16 */
+  uint32_t transform;    /* edp_transform */
+  uint32_t frame_stack;  /* K for STACK_F32 (1..16); must be 1 otherwise */
+  uint32_t next_obs;     /* STACK_F32 only: 1 = deliver next_obs as well; the
+                            newest transition is then not sampleable */
+  uint32_t tokens;       /* int32 tokens stored per transition (0 = none);
+                            a multiple of 4 */
+  uint32_t prioritized;  /* 1 = keep the priority sum-tree (PER) */
+  float norm_mean[4];    /* CHW_NORM_BF16 per-channel mean (of byte/255) */
+  float norm_std[4];     /* CHW_NORM_BF16 per-channel std, > 0 */
+  edp_alloc_fn alloc;    /* NULL = cudaMalloc */
+  edp_free_fn free;      /* NULL = cudaFree */
+  void *alloc_user;
+  int32_t device;        /* CUDA device ordinal of every device pointer */
+  uint32_t reserved[7];  /* must be 0 */
+} edp_config;
+
+/* Caller-owned ring storage.  Slot s of the logical ring holds the
+ * transition with logical id L where L mod capacity == s.  Its payload lives
+ * in HBM slot L mod hbm_capacity or, for the two-tier ring, in host slot
+ * L mod (capacity - hbm_capacity); metadata is HBM-resident for every slot. */
+typedef struct {
+  uint8_t *obs;         /* device [hbm_capacity][obs_bytes], 16-B aligned */
+  int32_t *tokens;      /* device [hbm_capacity][tokens]; NULL iff tokens==0 */
+  uint8_t *host_obs;    /* page-locked host [capacity-hbm_capacity][obs_bytes]
+                           (two-tier only, else NULL), 16-B aligned */
+  int32_t *host_tokens; /* page-locked host [capacity-hbm_capacity][tokens] */
+  int32_t *action;      /* device [capacity] or NULL */
+  float *reward;        /* device [capacity] or NULL */
+  uint8_t *done;        /* device [capacity]; required for STACK_F32 */
+} edp_storage;
+
+/* n transitions to insert, logical order.  Device-accessible pointers. */
+typedef struct {
+  const uint8_t *obs;    /* [n][obs_bytes], 16-B aligned; required */
+  const int32_t *tokens; /* [n][tokens]; required iff tokens > 0 */
+  const int32_t *action; /* [n] or NULL (stores 0) */
+  const float *reward;   /* [n] or NULL (stores 0) */
+  const uint8_t *done;   /* [n] or NULL (stores 0) */
+} edp_fields;
+
+/* Learner batch written by edp_deliver.  Device pointers; NULL skips an
+ * output.  B = the `batch` argument of edp_deliver. */
+typedef struct {
+  void *obs;      /* see edp_transform; required */
+  void *next_obs; /* STACK_F32 with next_obs == 1: float [B][K][h][w] */
+  int32_t *action;
+  float *reward;
+  uint8_t *done;  /* [B] each, of the sampled (anchor) transition */
+  int32_t *tokens;/* [B][tokens] */
+  /* Importance-sampling weights (PER): isw[b] = (q_min / q[b])^beta with
+   * q_min the minimum of q over the batch; fp64, rounded once to fp32.
+   * q = the priorities edp_sample(PRIORITIZED) returned for this batch. */
+  const uint32_t *q;
+  float *isw;
+  double beta;
+  /* Per-sample scalars gathered by the sample's logical offset k (0 = the
+   * oldest stored transition): dst[b] = src[k].  Used for the advantages and
+   * returns of an on-policy rollout.  NULL pairs are skipped. */
+  const float *gather_src[2];
+  float *gather_dst[2];
+} edp_batch;
+
+/* Inspection of a context (host values, device pointers). */
+typedef struct {
+  uint64_t capacity, hbm_capacity, total, size, head, oldest, n_valid;
+  uint32_t tree_depth;          /* D: leaves are level D, the root level 0 */
+  uint32_t tree_fanout;         /* 32 */
+  const uint32_t *tree_leaves;  /* device [32^D] */
+  const uint64_t *tree_level[8];/* device; level d has 32^d nodes, d < D */
+  const uint32_t *pending_q;    /* device [1]: deferred priority of newest */
+  const uint32_t *max_q;        /* device [1]: running maximum priority */
+} edp_info;
+
+/* Create a context on cfg->device over caller storage.  Fails with
+ * EDP_ERR_INVALID for inconsistent shapes or pointers, EDP_ERR_OOM when the
+ * allocator fails.  Synchronous (initialises the tree). */
+EDP_API edp_status edp_create(const edp_config *cfg, const edp_storage *st,
+                      edp_ctx **out);
+
+/* Free libedp-owned memory.  Waits for the device to finish with it. */
+EDP_API edp_status edp_destroy(edp_ctx *ctx);
+
+/* Ingestion (Sec. 2.2 "experience ingestion", off-policy insertion with
+ * FIFO eviction; Sec. 5 placement).  Inserts n (0..capacity) transitions at
+ * logical ids total .. total+n-1.  Two-tier ring: first moves the payload of
+ * the oldest HBM-resident transitions that must leave HBM into the host tier
+ * (evicting the oldest host entries), then writes the new payload to HBM.
+ * PER: q (device [n] or NULL) gives each new transition's priority (NULL =
+ * the running maximum, initially 2^20 = 1.0).  With next_obs, the newest
+ * transition's priority is deferred until its successor arrives. */
+EDP_API edp_status edp_ingest(edp_ctx *ctx, const edp_fields *src, uint64_t n,
+                      const uint32_t *q, edp_stream stream);
+
+/* Sampling (Sec. 2.2 delivery "select").  Writes idx (device int64 [batch])
+ * and, for PRIORITIZED, q (device uint32 [batch], may be NULL) = the sampled
+ * leaves.  Errors: EDP_ERR_EMPTY when no transition is sampleable;
+ * EDP_ERR_STATE for PRIORITIZED without a tree; EDP_ERR_INVALID when
+ * batch == 0 or, for PERMUTE, batch != size. */
+EDP_API edp_status edp_sample(edp_ctx *ctx, edp_sample_mode mode, uint32_t batch,
+                      uint64_t seed, uint64_t round, int64_t *idx,
+                      uint32_t *q, edp_stream stream);
+
+/* Delivery (Sec. 2.2 "materializes the selected transitions and performs
+ * batch/layout transformations"): fused gather + transform + collate (+ IS
+ * weights) of the `batch` slots in idx (device int64).  A slot outside the
+ * sampleable range is reported by edp_sync and its outputs are zeroed. */
+EDP_API edp_status edp_deliver(edp_ctx *ctx, const int64_t *idx, uint32_t batch,
+                       const edp_batch *out, edp_stream stream);
+
+/* Priority callback (Appendix C, Invariant 2; PER).  Sets the priority of
+ * each (idx[p], q[p]); for a repeated slot the last pair wins.  Pairs whose
+ * slot holds no transition are skipped; the newest transition's priority is
+ * deferred (next_obs).  Ancestor sums change by exact integer deltas. */
+EDP_API edp_status edp_update_priorities(edp_ctx *ctx, const int64_t *idx,
+                                 const uint32_t *q, uint32_t n,
+                                 edp_stream stream);
+
+/* Same, from TD errors: q = clamp(rn((|td| + eps)^alpha * 2^20), 1,
+ * 2^32-1) computed in fp64 on the device.  pow is not correctly rounded, so
+ * q may differ by 1 from a host evaluation. */
+EDP_API edp_status edp_update_priorities_td(edp_ctx *ctx, const int64_t *idx,
+                                    const float *td, uint32_t n, double alpha,
+                                    double eps, edp_stream stream);
+
+/* The TD-error rule alone: q[i] from td[i] (device arrays [n]). */
+EDP_API edp_status edp_priorities_from_td(edp_ctx *ctx, const float *td, uint32_t n,
+                                  double alpha, double eps, uint32_t *q,
+                                  edp_stream stream);
+
+/* Generalized advantage estimation (Schulman et al., ICLR'16) -- the
+ * "computing returns/advantages" and "normalization" of on-policy ingestion
+ * (Sec. 2.2).  Device arrays, time-major: r, d [T][E]; v [T+1][E].
+ *   delta_t = r_t + gamma V_{t+1} (1 - d_t) - V_t
+ *   A_t = delta_t + gamma lambda (1 - d_t) A_{t+1},  A_T = 0
+ *   ret_t = A_t + V_t
+ *   adv_norm = (A - mean(A)) / (std(A) + 1e-8), std with n-1, over T*E
+ * Computed in fp64, stored fp32 [T][E].  adv/ret/adv_norm may be NULL
+ * individually.  T*E >= 2. */
+EDP_API edp_status edp_gae(edp_ctx *ctx, const float *r, const float *v,
+                   const uint8_t *d, uint32_t T, uint32_t E, double gamma,
+                   double lambda, float *adv, float *ret, float *adv_norm,
+                   edp_stream stream);
+
+/* Wait for `stream`, then report (and clear) asynchronous CUDA errors and
+ * device-side flags recorded since the previous edp_sync. */
+EDP_API edp_status edp_sync(edp_ctx *ctx, edp_stream stream);
+
+/* Describe the context's last failure ("" if none).  Valid until the next
+ * call on the context. */
+EDP_API const char *edp_last_error(const edp_ctx *ctx);
+
+/* Fill *out with the context's cursors and tree layout. */
+EDP_API edp_status edp_get_info(const edp_ctx *ctx, edp_info *out);
+
+/* Host-link probe: streams `bytes` (a multiple of 16) of page-locked host
+ * memory through the GPU with 16-byte loads, xor-folding them into
+ * *d_fold (device uint64).  Used to measure achievable host-link read
+ * bandwidth for the two-tier ring. */
+EDP_API edp_status edp_probe_host_read(const void *host_src, uint64_t bytes,
+                               uint64_t *d_fold, edp_stream stream);
+
+/* ABI version compiled into the library (EDP_ABI_VERSION). */
+EDP_API int edp_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* EDP_H */

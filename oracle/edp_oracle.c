@@ -25,8 +25,20 @@
 #include <stdlib.h>
 #include <string.h>
 #include <math.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
 
 #define ORC_API __attribute__((visibility("default")))
+
+/* Threads the OpenMP loops over batch rows use (1 without OpenMP). */
+ORC_API int orc_num_threads(void) {
+#ifdef _OPENMP
+  return omp_get_max_threads();
+#else
+  return 1;
+#endif
+}
 
 /* ------------------------------------------------------------------------ */
 /* Philox4x32-10, Salmon, Moraes, Dror, Shaw, "Parallel Random Numbers: As   */

@@ -1,0 +1,640 @@
+// edp_api.cu -- the C ABI of libedp: argument validation, host-side cursors
+// of the logical ring, and kernel dispatch.  Every step of the data path
+// runs in the kernels of the other translation units.
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <new>
+
+#include "edp_internal.cuh"
+
+using namespace edp;
+
+namespace {
+
+void *default_alloc(void *, size_t bytes) {
+  void *p = nullptr;
+  if (cudaMalloc(&p, bytes) != cudaSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  return p;
+}
+
+void default_free(void *, void *p) { cudaFree(p); }
+
+edp_status fail(edp_ctx *c, edp_status s, const char *fmt, ...) {
+  if (c) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    c->err = buf;
+  }
+  return s;
+}
+
+edp_status cuda_fail(edp_ctx *c, cudaError_t e, const char *where) {
+  return fail(c, EDP_ERR_CUDA, "%s: %s", where, cudaGetErrorString(e));
+}
+
+// Resolve a caller pointer to a device-usable address.  Device memory of the
+// context's GPU passes through; page-locked host memory is translated to its
+// mapped device address; pageable or foreign memory is rejected.
+bool device_view(const edp_ctx *c, const void *p, const void **out,
+                 bool allow_host) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  if (a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged) {
+    if (a.device != c->cfg.device) return false;
+    *out = p;
+    return true;
+  }
+  if (a.type == cudaMemoryTypeHost && allow_host && a.devicePointer) {
+    *out = a.devicePointer;
+    return true;
+  }
+  return false;
+}
+
+edp_status create_fail(edp_ctx *c, const char *fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof buf, fmt, ap);
+  va_end(ap);
+  fprintf(stderr, "edp_create: %s\n", buf);
+  delete c;
+  return EDP_ERR_INVALID;
+}
+
+bool aligned16(const void *p) { return ((uintptr_t)p & 15u) == 0; }
+
+uint64_t ring_size(const edp_ctx *c) { return c->total < c->cap ? c->total : c->cap; }
+
+uint64_t n_valid(const edp_ctx *c) {
+  const uint64_t s = ring_size(c);
+  return s >= (uint64_t)c->defer ? s - c->defer : 0;
+}
+
+void free_all(edp_ctx *c) {
+  edp_free_fn fr = c->cfg.free ? c->cfg.free : default_free;
+  if (c->tree_mem) fr(c->cfg.alloc_user, c->tree_mem);
+  if (c->ctrl) fr(c->cfg.alloc_user, c->ctrl);
+  if (c->scratch) fr(c->cfg.alloc_user, c->scratch);
+  if (c->qbuf) fr(c->cfg.alloc_user, c->qbuf);
+  c->qbuf = nullptr;
+  c->tree_mem = nullptr;
+  c->ctrl = nullptr;
+  c->scratch = nullptr;
+}
+
+// Host self-check of the transform constants against IEEE division (the
+// device evaluates exactly these operations).
+bool unit_constants(float *r1, float *r2) {
+  *r1 = 1.0f / 255.0f;
+  *r2 = (float)(1.0 / 255.0 - (double)*r1);
+  for (int b = 0; b < 256; ++b) {
+    const float x = (float)b;
+    const float ref = x / 255.0f;
+    const float got = fmaf(x, *r1, x * *r2);
+    if (got != ref) return false;
+  }
+  return true;
+}
+
+bool norm_constants(edp_ctx *c) {
+  bool fast = true;
+  for (uint32_t ch = 0; ch < c->cfg.obs_c; ++ch) {
+    const float m = c->cfg.norm_mean[ch], s = c->cfg.norm_std[ch];
+    const float s1 = (float)(1.0 / (double)s);
+    const float s2 = (float)(1.0 / (double)s - (double)s1);
+    c->nmean[ch] = m;
+    c->nstd[ch] = s;
+    c->ns1[ch] = s1;
+    c->ns2[ch] = s2;
+    for (int b = 0; b < 256; ++b) {
+      const float x = (float)b / 255.0f;
+      const float t = x - m;
+      if (fmaf(t, s1, t * s2) != t / s) fast = false;
+    }
+  }
+  return fast;
+}
+
+}  // namespace
+
+void *edp::ctx_scratch(edp_ctx *ctx, size_t bytes) {
+  if (bytes <= ctx->scratch_bytes) return ctx->scratch;
+  edp_alloc_fn al = ctx->cfg.alloc ? ctx->cfg.alloc : default_alloc;
+  edp_free_fn fr = ctx->cfg.free ? ctx->cfg.free : default_free;
+  if (ctx->scratch) {
+    cudaDeviceSynchronize();  // the old block may still be in use
+    fr(ctx->cfg.alloc_user, ctx->scratch);
+    ctx->scratch = nullptr;
+    ctx->scratch_bytes = 0;
+  }
+  bytes = (bytes + 255) & ~(size_t)255;
+  void *p = al(ctx->cfg.alloc_user, bytes);
+  if (!p) return nullptr;
+  ctx->scratch = p;
+  ctx->scratch_bytes = bytes;
+  return p;
+}
+
+uint32_t *edp::ctx_qbuf(edp_ctx *ctx, size_t n) {
+  if (n <= ctx->qbuf_n) return ctx->qbuf;
+  edp_alloc_fn al = ctx->cfg.alloc ? ctx->cfg.alloc : default_alloc;
+  edp_free_fn fr = ctx->cfg.free ? ctx->cfg.free : default_free;
+  if (ctx->qbuf) {
+    cudaDeviceSynchronize();
+    fr(ctx->cfg.alloc_user, ctx->qbuf);
+    ctx->qbuf = nullptr;
+    ctx->qbuf_n = 0;
+  }
+  n = n < 4096 ? 4096 : n;
+  void *p = al(ctx->cfg.alloc_user, n * 4);
+  if (!p) return nullptr;
+  ctx->qbuf = (uint32_t *)p;
+  ctx->qbuf_n = n;
+  return ctx->qbuf;
+}
+
+extern "C" {
+
+int edp_abi_version(void) { return EDP_ABI_VERSION; }
+
+const char *edp_last_error(const edp_ctx *ctx) {
+  return ctx ? ctx->err.c_str() : "null context";
+}
+
+edp_status edp_create(const edp_config *cfg, const edp_storage *st,
+                      edp_ctx **out) {
+  if (!cfg || !st || !out) return EDP_ERR_INVALID;
+  *out = nullptr;
+  edp_ctx *c = new (std::nothrow) edp_ctx();
+  if (!c) return EDP_ERR_OOM;
+  c->cfg = *cfg;
+  c->st = *st;
+#define bad(...) create_fail(c, __VA_ARGS__)
+  for (int i = 0; i < 7; ++i)
+    if (cfg->reserved[i]) return bad("reserved fields must be 0");
+  if (cfg->capacity == 0 || cfg->capacity > 0xFFFFFFFFull)
+    return bad("capacity must be in [1, 2^32-1]");
+  if (cfg->hbm_capacity == 0 || cfg->hbm_capacity > cfg->capacity)
+    return bad("hbm_capacity must be in [1, capacity]");
+  if (!cfg->obs_c || !cfg->obs_h || !cfg->obs_w) return bad("empty obs shape");
+  const uint64_t ob = (uint64_t)cfg->obs_c * cfg->obs_h * cfg->obs_w;
+  if (ob % 16) return bad("obs bytes (%llu) must be a multiple of 16",
+                          (unsigned long long)ob);
+  if (ob > 0x7FFFFFFFull) return bad("obs too large");
+  if (cfg->tokens % 4) return bad("tokens must be a multiple of 4");
+  if (cfg->transform > EDP_XFORM_CHW_NORM_BF16) return bad("bad transform");
+  const uint64_t hw = (uint64_t)cfg->obs_h * cfg->obs_w;
+  if (cfg->transform == EDP_XFORM_STACK_F32) {
+    if (cfg->obs_c != 1) return bad("STACK_F32 stores single-channel frames");
+    if (cfg->frame_stack < 1 || cfg->frame_stack > 16)
+      return bad("frame_stack must be in [1, 16]");
+    if (!st->done) return bad("STACK_F32 needs the done field");
+  } else {
+    if (cfg->frame_stack != 1) return bad("frame_stack must be 1");
+    if (cfg->next_obs) return bad("next_obs only with STACK_F32");
+    if (cfg->obs_c > 4) return bad("obs_c must be <= 4");
+    if (hw % 16) return bad("obs_h*obs_w must be a multiple of 16");
+  }
+  if (cfg->transform == EDP_XFORM_CHW_NORM_BF16)
+    for (uint32_t ch = 0; ch < cfg->obs_c; ++ch)
+      if (!(cfg->norm_std[ch] > 0.f) || !std::isfinite(cfg->norm_mean[ch]))
+        return bad("norm_std must be > 0 and norm_mean finite");
+  const bool tiered = cfg->hbm_capacity < cfg->capacity;
+  if (tiered && cfg->transform != EDP_XFORM_CHW_NORM_BF16)
+    return bad("the two-tier ring serves CHW_NORM_BF16 payloads");
+
+  int ndev = 0;
+  if (cudaGetDeviceCount(&ndev) != cudaSuccess || cfg->device < 0 ||
+      cfg->device >= ndev) {
+    cudaGetLastError();
+    return bad("no CUDA device %d", cfg->device);
+  }
+  if (cudaSetDevice(cfg->device) != cudaSuccess) {
+    cudaGetLastError();
+    return bad("cudaSetDevice failed");
+  }
+  c->cap = cfg->capacity;
+  c->cap_h = cfg->hbm_capacity;
+  c->cap_c = cfg->capacity - cfg->hbm_capacity;
+  c->obs_bytes = ob;
+  c->tok_bytes = (uint64_t)cfg->tokens * 4;
+  c->defer = cfg->next_obs ? 1 : 0;
+
+  // storage pointers
+  const void *p;
+  if (!st->obs || !device_view(c, st->obs, &p, false) || !aligned16(st->obs))
+    return bad("storage.obs must be 16-B aligned device memory");
+  if ((cfg->tokens > 0) != (st->tokens != nullptr))
+    return bad("storage.tokens must be given iff tokens > 0");
+  if (st->tokens && (!device_view(c, st->tokens, &p, false) ||
+                     !aligned16(st->tokens)))
+    return bad("storage.tokens must be 16-B aligned device memory");
+  if (tiered) {
+    if (!st->host_obs || !device_view(c, st->host_obs, &p, true) ||
+        !aligned16(p))
+      return bad("storage.host_obs must be page-locked host memory");
+    c->st.host_obs = (uint8_t *)p;
+    if ((cfg->tokens > 0) != (st->host_tokens != nullptr))
+      return bad("storage.host_tokens must be given iff tokens > 0");
+    if (st->host_tokens) {
+      if (!device_view(c, st->host_tokens, &p, true) || !aligned16(p))
+        return bad("storage.host_tokens must be page-locked host memory");
+      c->st.host_tokens = (int32_t *)p;
+    }
+  } else if (st->host_obs || st->host_tokens) {
+    return bad("host tier given but hbm_capacity == capacity");
+  }
+  if (st->action && !device_view(c, st->action, &p, false))
+    return bad("storage.action must be device memory");
+  if (st->reward && !device_view(c, st->reward, &p, false))
+    return bad("storage.reward must be device memory");
+  if (st->done && !device_view(c, st->done, &p, false))
+    return bad("storage.done must be device memory");
+
+  if (!unit_constants(&c->r1, &c->r2)) return bad("byte/255 self-check failed");
+  if (cfg->transform == EDP_XFORM_CHW_NORM_BF16) c->norm_fast = norm_constants(c);
+
+  int dev_sms = 0;
+  cudaDeviceGetAttribute(&dev_sms, cudaDevAttrMultiProcessorCount, cfg->device);
+  c->coop_sms = dev_sms;
+
+  edp_alloc_fn al = cfg->alloc ? cfg->alloc : default_alloc;
+  c->ctrl = (Ctrl *)al(cfg->alloc_user, sizeof(Ctrl));
+  if (!c->ctrl) {
+    free_all(c);
+    delete c;
+    return EDP_ERR_OOM;
+  }
+  Ctrl init{};
+  init.max_q = 1u << 20;
+  cudaError_t e = cudaMemcpy(c->ctrl, &init, sizeof init, cudaMemcpyHostToDevice);
+  if (cfg->prioritized && e == cudaSuccess) {
+    uint32_t D = 1;
+    uint64_t n = kFanout;
+    while (n < c->cap) {
+      n *= kFanout;
+      ++D;
+    }
+    c->depth = D;
+    c->nleaves = n;
+    uint64_t internal = 0, m = 1;
+    for (uint32_t d = 0; d < D; ++d) {
+      internal += m;
+      m *= kFanout;
+    }
+    const size_t bytes = internal * 8 + n * 4;
+    c->tree_mem = al(cfg->alloc_user, bytes);
+    if (!c->tree_mem) {
+      free_all(c);
+      delete c;
+      return EDP_ERR_OOM;
+    }
+    uint64_t off = 0;
+    m = 1;
+    for (uint32_t d = 0; d < D; ++d) {
+      c->level[d] = (uint64_t *)c->tree_mem + off;
+      off += m;
+      m *= kFanout;
+    }
+    c->leaves = (uint32_t *)((uint64_t *)c->tree_mem + internal);
+    e = cudaMemset(c->tree_mem, 0, bytes);
+  }
+  if (e == cudaSuccess) e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    free_all(c);
+    delete c;
+    return EDP_ERR_CUDA;
+  }
+  *out = c;
+  return EDP_OK;
+}
+#undef bad
+
+edp_status edp_destroy(edp_ctx *ctx) {
+  if (!ctx) return EDP_ERR_INVALID;
+  cudaSetDevice(ctx->cfg.device);
+  cudaDeviceSynchronize();
+  free_all(ctx);
+  delete ctx;
+  return EDP_OK;
+}
+
+edp_status edp_get_info(const edp_ctx *ctx, edp_info *o) {
+  if (!ctx || !o) return EDP_ERR_INVALID;
+  memset(o, 0, sizeof *o);
+  o->capacity = ctx->cap;
+  o->hbm_capacity = ctx->cap_h;
+  o->total = ctx->total;
+  o->size = ring_size(ctx);
+  o->head = ctx->total % ctx->cap;
+  o->oldest = (ctx->total - o->size) % ctx->cap;
+  o->n_valid = n_valid(ctx);
+  o->tree_depth = ctx->depth;
+  o->tree_fanout = kFanout;
+  o->tree_leaves = ctx->leaves;
+  for (uint32_t d = 0; d < ctx->depth && d < 8; ++d) o->tree_level[d] = ctx->level[d];
+  o->pending_q = &ctx->ctrl->pending_q;
+  o->max_q = &ctx->ctrl->max_q;
+  return EDP_OK;
+}
+
+edp_status edp_ingest(edp_ctx *ctx, const edp_fields *src, uint64_t n,
+                      const uint32_t *q, edp_stream stream) {
+  if (!ctx) return EDP_ERR_INVALID;
+  if (!src) return fail(ctx, EDP_ERR_INVALID, "edp_ingest: src is NULL");
+  if (n > ctx->cap)
+    return fail(ctx, EDP_ERR_INVALID, "edp_ingest: n=%llu exceeds capacity",
+                (unsigned long long)n);
+  if (n == 0) return EDP_OK;
+  cudaSetDevice(ctx->cfg.device);
+  cudaStream_t s = (cudaStream_t)stream;
+  edp_fields f{};
+  const void *p;
+  if (!src->obs || !device_view(ctx, src->obs, &p, true) || !aligned16(p))
+    return fail(ctx, EDP_ERR_INVALID,
+                "edp_ingest: src.obs must be 16-B aligned device or page-locked memory");
+  f.obs = (const uint8_t *)p;
+  if ((ctx->tok_bytes > 0) != (src->tokens != nullptr))
+    return fail(ctx, EDP_ERR_INVALID, "edp_ingest: src.tokens given iff tokens > 0");
+  if (src->tokens) {
+    if (!device_view(ctx, src->tokens, &p, true) || !aligned16(p))
+      return fail(ctx, EDP_ERR_INVALID, "edp_ingest: bad src.tokens");
+    f.tokens = (const int32_t *)p;
+  }
+#define EDP_VIEW(field, T)                                                     \
+  if (src->field) {                                                            \
+    if (!device_view(ctx, src->field, &p, true))                               \
+      return fail(ctx, EDP_ERR_INVALID, "edp_ingest: bad src." #field);        \
+    f.field = (T)p;                                                            \
+  }
+  EDP_VIEW(action, const int32_t *)
+  EDP_VIEW(reward, const float *)
+  EDP_VIEW(done, const uint8_t *)
+#undef EDP_VIEW
+  if (q && !device_view(ctx, q, &p, false))
+    return fail(ctx, EDP_ERR_INVALID, "edp_ingest: q must be device memory");
+  if (q && !ctx->depth)
+    return fail(ctx, EDP_ERR_STATE, "edp_ingest: q given to a context without priorities");
+
+  cudaError_t e = cudaSuccess;
+  // Placement of ids [T, T+n).  Afterwards HBM holds [Tn - keep_h, Tn) and
+  // the host tier [Tn - keep, Tn - keep_h).  Resident ids that leave HBM
+  // but stay retained are demoted first (same stream, so before their HBM
+  // slots are overwritten); new ids older than the HBM window go straight
+  // to the host tier; the rest are written to HBM.
+  const uint64_t T = ctx->total, Tn = T + n;
+  const uint64_t keep_h = Tn < ctx->cap_h ? Tn : ctx->cap_h;
+  const uint64_t keep = Tn < ctx->cap ? Tn : ctx->cap;
+  uint64_t new_hbm_lo = T;
+  if (ctx->cap_c) {
+    const uint64_t in_hbm = T < ctx->cap_h ? T : ctx->cap_h;
+    uint64_t lo = T - in_hbm;
+    if (lo < Tn - keep) lo = Tn - keep;  // evicted outright
+    const uint64_t hi = (Tn - keep_h) < T ? (Tn - keep_h) : T;
+    if (hi > lo) e = launch_demote(ctx, lo, hi - lo, s);
+    // new ids [max(T, Tn - keep), Tn - keep_h) -> host tier directly
+    const uint64_t dlo = T > Tn - keep ? T : Tn - keep;
+    const uint64_t dhi = Tn - keep_h;
+    if (e == cudaSuccess && dhi > dlo)
+      e = launch_copy_rows_to_host(ctx, f.obs, f.tokens, dlo - T, dlo, dhi - dlo, s);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_ingest(host tier)");
+    if (new_hbm_lo < Tn - keep_h) new_hbm_lo = Tn - keep_h;
+  }
+  const uint64_t skip = new_hbm_lo - T, nh = Tn - new_hbm_lo;
+  e = launch_copy_rows(ctx->st.obs, ctx->cap_h, new_hbm_lo % ctx->cap_h,
+                       f.obs + skip * ctx->obs_bytes, nh, ctx->obs_bytes, s);
+  if (e == cudaSuccess && ctx->tok_bytes)
+    e = launch_copy_rows((uint8_t *)ctx->st.tokens, ctx->cap_h,
+                         new_hbm_lo % ctx->cap_h,
+                         (const uint8_t *)f.tokens + skip * ctx->tok_bytes, nh,
+                         ctx->tok_bytes, s);
+  if (e == cudaSuccess) e = launch_ingest_meta(ctx, &f, n, q, s);
+  if (e == cudaSuccess && ctx->depth) {
+    uint64_t first = ctx->total % ctx->cap, count = n;
+    if (ctx->defer && ctx->total >= 1) {
+      first = (ctx->total - 1) % ctx->cap;
+      count = n + 1;
+    }
+    if (count > ctx->cap) count = ctx->cap;
+    e = launch_tree_refresh(ctx, first, count, s);
+  }
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_ingest");
+  ctx->total += n;
+  return EDP_OK;
+}
+
+edp_status edp_sample(edp_ctx *ctx, edp_sample_mode mode, uint32_t batch,
+                      uint64_t seed, uint64_t round, int64_t *idx, uint32_t *q,
+                      edp_stream stream) {
+  if (!ctx) return EDP_ERR_INVALID;
+  if (!idx) return fail(ctx, EDP_ERR_INVALID, "edp_sample: idx is NULL");
+  if (batch == 0) return fail(ctx, EDP_ERR_INVALID, "edp_sample: batch == 0");
+  const void *p;
+  if (!device_view(ctx, idx, &p, false) || (q && !device_view(ctx, q, &p, false)))
+    return fail(ctx, EDP_ERR_INVALID, "edp_sample: outputs must be device memory");
+  cudaSetDevice(ctx->cfg.device);
+  cudaStream_t s = (cudaStream_t)stream;
+  cudaError_t e;
+  switch (mode) {
+    case EDP_SAMPLE_UNIFORM:
+      if (n_valid(ctx) == 0)
+        return fail(ctx, EDP_ERR_EMPTY, "edp_sample: no sampleable transition");
+      e = launch_sample_uniform(ctx, batch, seed, round, idx, s);
+      break;
+    case EDP_SAMPLE_PRIORITIZED:
+      if (!ctx->depth)
+        return fail(ctx, EDP_ERR_STATE, "edp_sample: context has no priorities");
+      if (n_valid(ctx) == 0)
+        return fail(ctx, EDP_ERR_EMPTY, "edp_sample: no sampleable transition");
+      e = launch_sample_prioritized(ctx, batch, seed, round, idx, q, s);
+      break;
+    case EDP_SAMPLE_PERMUTE:
+      if (ring_size(ctx) == 0)
+        return fail(ctx, EDP_ERR_EMPTY, "edp_sample: ring is empty");
+      if (batch != ring_size(ctx))
+        return fail(ctx, EDP_ERR_INVALID,
+                    "edp_sample: PERMUTE needs batch == size (%llu)",
+                    (unsigned long long)ring_size(ctx));
+      e = launch_permute(ctx, batch, seed, round, idx, s);
+      break;
+    default:
+      return fail(ctx, EDP_ERR_INVALID, "edp_sample: unknown mode %d", (int)mode);
+  }
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_sample");
+  return EDP_OK;
+}
+
+edp_status edp_deliver(edp_ctx *ctx, const int64_t *idx, uint32_t batch,
+                       const edp_batch *out, edp_stream stream) {
+  if (!ctx) return EDP_ERR_INVALID;
+  if (!idx || !out || !out->obs)
+    return fail(ctx, EDP_ERR_INVALID, "edp_deliver: idx/out/out->obs is NULL");
+  if (batch == 0) return fail(ctx, EDP_ERR_INVALID, "edp_deliver: batch == 0");
+  if (ring_size(ctx) == 0) return fail(ctx, EDP_ERR_EMPTY, "edp_deliver: ring is empty");
+  if (out->next_obs && !ctx->defer)
+    return fail(ctx, EDP_ERR_STATE, "edp_deliver: next_obs needs next_obs=1");
+  if (out->tokens && !ctx->tok_bytes)
+    return fail(ctx, EDP_ERR_STATE, "edp_deliver: context stores no tokens");
+  if (out->action && !ctx->st.action)
+    return fail(ctx, EDP_ERR_STATE, "edp_deliver: context stores no action");
+  if (out->reward && !ctx->st.reward)
+    return fail(ctx, EDP_ERR_STATE, "edp_deliver: context stores no reward");
+  if (out->done && !ctx->st.done)
+    return fail(ctx, EDP_ERR_STATE, "edp_deliver: context stores no done");
+  if (out->isw && !out->q)
+    return fail(ctx, EDP_ERR_INVALID, "edp_deliver: isw needs q");
+  if (out->isw && !(out->beta >= 0.0))
+    return fail(ctx, EDP_ERR_INVALID, "edp_deliver: beta must be >= 0");
+  for (int i = 0; i < 2; ++i)
+    if ((out->gather_src[i] == nullptr) != (out->gather_dst[i] == nullptr))
+      return fail(ctx, EDP_ERR_INVALID, "edp_deliver: gather pair %d half-NULL", i);
+  const void *p;
+  const void *outs[] = {idx, out->obs, out->next_obs, out->action, out->reward,
+                        out->done, out->tokens, out->q, out->isw,
+                        out->gather_src[0], out->gather_dst[0],
+                        out->gather_src[1], out->gather_dst[1]};
+  for (const void *o : outs)
+    if (o && !device_view(ctx, o, &p, false))
+      return fail(ctx, EDP_ERR_INVALID, "edp_deliver: pointers must be device memory");
+  if (!aligned16(out->obs) || (out->next_obs && !aligned16(out->next_obs)) ||
+      (out->tokens && !aligned16(out->tokens)))
+    return fail(ctx, EDP_ERR_INVALID, "edp_deliver: obs/next_obs/tokens 16-B aligned");
+  cudaSetDevice(ctx->cfg.device);
+  cudaError_t e = launch_deliver(ctx, idx, batch, out, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_deliver");
+  return EDP_OK;
+}
+
+static edp_status update_common(edp_ctx *ctx, const int64_t *idx,
+                                const uint32_t *q, const float *td, uint32_t n,
+                                double alpha, double eps, edp_stream stream) {
+  if (!ctx) return EDP_ERR_INVALID;
+  if (!ctx->depth)
+    return fail(ctx, EDP_ERR_STATE, "edp_update_priorities: context has no priorities");
+  if (n == 0) return EDP_OK;
+  if (!idx || (!q && !td))
+    return fail(ctx, EDP_ERR_INVALID, "edp_update_priorities: NULL input");
+  const void *p;
+  if (!device_view(ctx, idx, &p, false) ||
+      (q && !device_view(ctx, q, &p, false)) ||
+      (td && !device_view(ctx, td, &p, false)))
+    return fail(ctx, EDP_ERR_INVALID, "edp_update_priorities: inputs must be device memory");
+  cudaSetDevice(ctx->cfg.device);
+  cudaError_t e = launch_update(ctx, idx, q, td, alpha, eps, n, (cudaStream_t)stream);
+  if (e == cudaErrorMemoryAllocation)
+    return fail(ctx, EDP_ERR_OOM, "edp_update_priorities: scratch allocation failed");
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_update_priorities");
+  return EDP_OK;
+}
+
+edp_status edp_update_priorities(edp_ctx *ctx, const int64_t *idx,
+                                 const uint32_t *q, uint32_t n,
+                                 edp_stream stream) {
+  if (ctx && n && !q) return fail(ctx, EDP_ERR_INVALID, "edp_update_priorities: q NULL");
+  return update_common(ctx, idx, q, nullptr, n, 0.0, 0.0, stream);
+}
+
+edp_status edp_update_priorities_td(edp_ctx *ctx, const int64_t *idx,
+                                    const float *td, uint32_t n, double alpha,
+                                    double eps, edp_stream stream) {
+  if (ctx && n && !td) return fail(ctx, EDP_ERR_INVALID, "edp_update_priorities_td: td NULL");
+  if (ctx && !(alpha >= 0.0 && eps >= 0.0))
+    return fail(ctx, EDP_ERR_INVALID, "edp_update_priorities_td: alpha, eps >= 0");
+  return update_common(ctx, idx, nullptr, td, n, alpha, eps, stream);
+}
+
+edp_status edp_priorities_from_td(edp_ctx *ctx, const float *td, uint32_t n,
+                                  double alpha, double eps, uint32_t *q,
+                                  edp_stream stream) {
+  if (!ctx) return EDP_ERR_INVALID;
+  if (n == 0) return EDP_OK;
+  const void *p;
+  if (!td || !q || !device_view(ctx, td, &p, false) || !device_view(ctx, q, &p, false))
+    return fail(ctx, EDP_ERR_INVALID, "edp_priorities_from_td: device arrays required");
+  if (!(alpha >= 0.0 && eps >= 0.0))
+    return fail(ctx, EDP_ERR_INVALID, "edp_priorities_from_td: alpha, eps >= 0");
+  cudaSetDevice(ctx->cfg.device);
+  cudaError_t e = launch_prio_from_td(td, n, alpha, eps, q, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_priorities_from_td");
+  return EDP_OK;
+}
+
+edp_status edp_gae(edp_ctx *ctx, const float *r, const float *v,
+                   const uint8_t *d, uint32_t T, uint32_t E, double gamma,
+                   double lambda, float *adv, float *ret, float *adv_norm,
+                   edp_stream stream) {
+  if (!ctx) return EDP_ERR_INVALID;
+  if (!r || !v || !d) return fail(ctx, EDP_ERR_INVALID, "edp_gae: r/v/d NULL");
+  if (T == 0 || E == 0 || (uint64_t)T * E < 2 || (uint64_t)T * E > 0x7FFFFFFFull)
+    return fail(ctx, EDP_ERR_INVALID, "edp_gae: need 2 <= T*E < 2^31");
+  if (!std::isfinite(gamma) || !std::isfinite(lambda))
+    return fail(ctx, EDP_ERR_INVALID, "edp_gae: gamma/lambda not finite");
+  const void *p;
+  const void *ptrs[] = {r, v, d, adv, ret, adv_norm};
+  for (const void *o : ptrs)
+    if (o && !device_view(ctx, o, &p, false))
+      return fail(ctx, EDP_ERR_INVALID, "edp_gae: arrays must be device memory");
+  cudaSetDevice(ctx->cfg.device);
+  cudaError_t e = launch_gae(ctx, r, v, d, T, E, gamma, lambda, adv, ret, adv_norm,
+                             (cudaStream_t)stream);
+  if (e == cudaErrorMemoryAllocation)
+    return fail(ctx, EDP_ERR_OOM, "edp_gae: scratch allocation failed");
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_gae");
+  return EDP_OK;
+}
+
+edp_status edp_sync(edp_ctx *ctx, edp_stream stream) {
+  if (!ctx) return EDP_ERR_INVALID;
+  cudaSetDevice(ctx->cfg.device);
+  cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
+  if (e == cudaSuccess) e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_sync");
+  Ctrl h;
+  e = cudaMemcpy(&h, ctx->ctrl, sizeof h, cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_sync(read flags)");
+  if (h.err == 0) return EDP_OK;
+  const uint32_t zero[2] = {0, 0};
+  cudaMemcpy(&ctx->ctrl->err, zero, 4, cudaMemcpyHostToDevice);
+  cudaMemcpy(&ctx->ctrl->bad_index, zero, 8, cudaMemcpyHostToDevice);
+  const unsigned long long bi = h.bad_index ? h.bad_index - 1 : 0;
+  if (h.err & DEVERR_TIMEOUT)
+    return fail(ctx, EDP_ERR_TIMEOUT, "device: a bounded wait expired (flags 0x%x)", h.err);
+  if (h.err & DEVERR_EMPTY)
+    return fail(ctx, EDP_ERR_EMPTY, "device: total priority was 0 (flags 0x%x)", h.err);
+  if (h.err & DEVERR_TREE)
+    return fail(ctx, EDP_ERR_STATE, "device: inconsistent priority tree (flags 0x%x)", h.err);
+  return fail(ctx, EDP_ERR_INVALID,
+              "device: index out of range (first offender %llu, flags 0x%x)", bi, h.err);
+}
+
+edp_status edp_probe_host_read(const void *host_src, uint64_t bytes,
+                               uint64_t *d_fold, edp_stream stream) {
+  if (!host_src || !d_fold || bytes % 16) return EDP_ERR_INVALID;
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, host_src) != cudaSuccess) {
+    cudaGetLastError();
+    return EDP_ERR_INVALID;
+  }
+  const void *src = host_src;
+  if (a.type == cudaMemoryTypeHost) src = a.devicePointer;
+  else if (a.type != cudaMemoryTypeDevice) return EDP_ERR_INVALID;
+  if (!src || !aligned16(src)) return EDP_ERR_INVALID;
+  return launch_probe_read(src, bytes, d_fold, (cudaStream_t)stream) == cudaSuccess
+             ? EDP_OK
+             : EDP_ERR_CUDA;
+}
+
+}  // extern "C"

@@ -1,0 +1,435 @@
+// edp_internal.cuh -- context layout, device helpers and kernel launchers
+// shared by the translation units of libedp.  Not part of the ABI.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <string>
+
+#include "edp.h"
+
+namespace edp {
+
+// Device-side fault flags (edp_ctrl::err).  Kernels never trap: they record a
+// flag, zero the affected outputs and return; edp_sync reports the flags.
+enum : uint32_t {
+  DEVERR_INDEX = 1u,    // a slot index outside the sampleable range
+  DEVERR_EMPTY = 2u,    // total priority 0 at sampling time
+  DEVERR_TIMEOUT = 4u,  // a bounded wait (grid barrier, bulk copy) expired
+  DEVERR_TREE = 8u,     // a tree descent found no child holding its target
+};
+
+// Small device-resident control block (one per context).
+struct Ctrl {
+  uint32_t err;
+  uint32_t pending_q;  // deferred priority of the newest transition
+  uint32_t max_q;      // running maximum priority
+  uint32_t bar_count;  // grid barrier: arrivals
+  uint32_t bar_gen;    // grid barrier: generation
+  uint32_t upd_count;  // priority update: CTAs done with phase 1
+  uint32_t pad[2];
+  unsigned long long bad_index;  // first offending index (diagnostics)
+};
+
+constexpr int kFanout = 32;
+constexpr int kMaxDepth = 7;  // 32^7 > 2^32 leaves
+
+}  // namespace edp
+
+struct edp_ctx {
+  edp_config cfg;
+  edp_storage st;  // payload and metadata pointers, device-accessible
+  uint64_t cap = 0, cap_h = 0, cap_c = 0;
+  uint64_t obs_bytes = 0, tok_bytes = 0;
+  uint64_t total = 0;
+  int defer = 0;  // next_obs: newest transition not sampleable
+  // priority sum-tree: level d < depth holds 32^d uint64 sums; leaves uint32
+  uint32_t depth = 0;
+  uint64_t nleaves = 0;
+  uint32_t *leaves = nullptr;
+  uint64_t *level[edp::kMaxDepth] = {};
+  void *tree_mem = nullptr;
+  edp::Ctrl *ctrl = nullptr;
+  // lazily grown scratch (shuffle, GAE partials)
+  void *scratch = nullptr;
+  size_t scratch_bytes = 0;
+  // priorities computed from TD errors before they are applied
+  uint32_t *qbuf = nullptr;
+  size_t qbuf_n = 0;
+  // byte -> fl32(b/255) constants: x*R1 + x*R2 with one rounding
+  float r1 = 0.f, r2 = 0.f;
+  // per-channel normalisation: t = x - mean; y = t*S1 + t*S2 (one rounding)
+  float nmean[4] = {}, ns1[4] = {}, ns2[4] = {}, nstd[4] = {};
+  int norm_fast = 1;  // 0: the constants do not reproduce t/std -> divide
+  int coop_sms = 0;
+  std::string err;
+};
+
+namespace edp {
+
+// ---------------------------------------------------------------------------
+// Device helpers
+// ---------------------------------------------------------------------------
+
+// Philox4x32-10 (Salmon et al., SC'11).
+__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint32_t k0,
+                                               uint32_t k1) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    if (r) {
+      k0 += 0x9E3779B9u;
+      k1 += 0xBB67AE85u;
+    }
+    const uint32_t hi0 = __umulhi(0xD2511F53u, c.x);
+    const uint32_t lo0 = 0xD2511F53u * c.x;
+    const uint32_t hi1 = __umulhi(0xCD9E8D57u, c.z);
+    const uint32_t lo1 = 0xCD9E8D57u * c.z;
+    c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
+  }
+  return c;
+}
+
+// Draw j of (seed, round, stream): counter (j, round.lo, stream, round.hi),
+// key (seed.lo, seed.hi), value (word1 << 32) | word0.
+__device__ __forceinline__ uint64_t philox_u64(uint64_t seed, uint32_t j,
+                                               uint64_t round,
+                                               uint32_t stream) {
+  const uint4 o = philox4x32_10(
+      make_uint4(j, (uint32_t)round, stream, (uint32_t)(round >> 32)),
+      (uint32_t)seed, (uint32_t)(seed >> 32));
+  return ((uint64_t)o.y << 32) | (uint64_t)o.x;
+}
+
+__device__ __forceinline__ uint64_t mulhi64(uint64_t a, uint64_t n) {
+  return __umul64hi(a, n);
+}
+
+// fl32(b/255) for an integer-valued x = b in [0, 255]: r1 + r2 is 1/255 to
+// ~2^-48 relative, and b/255 never lies that close to a rounding boundary
+// of binary32, so one fused multiply-add rounds to the correctly rounded
+// quotient.  (The host checks all 256 inputs at context creation.)
+__device__ __forceinline__ float unit_f32(float x, float r1, float r2) {
+  return __fmaf_rn(x, r1, __fmul_rn(x, r2));
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t *>(&v);
+}
+
+// x^a for x in [2^-1000, 2^1000], fp64, written for GB300's narrow fp64
+// pipe (a dependent fp64 FMA costs ~64 cycles and a divide ~500, so a
+// general pow is ~6,000 cycles):
+//   x = 2^e m with m in [sqrt(1/2), sqrt(2));
+//   ln m = 2 atanh(s) = 2 (s + s^3/3 + s^5/5 + ...),  s = (m-1)/(m+1),
+//     |s| <= 0.1716; the reciprocal 1/(m+1) is an fp32 seed refined by
+//     two Newton steps (2^-23 -> 2^-92);
+//   t = a (e ln 2 + ln m);  e^t = 2^n e^r,  n = rint(t / ln 2),
+//     r = t - n ln 2 (ln 2 split in a high and a low part), |r| <= 0.35,
+//     e^r by its Taylor polynomial.
+// (Series: Abramowitz & Stegun 4.1.27 and 4.2.1.)  FULL: 11 + 17 terms,
+// relative error ~1e-15; otherwise 7 + 11 terms, ~1e-10, ample for a result
+// rounded to fp32.
+template <bool FULL>
+__device__ __forceinline__ double pow_pos(double x, double a) {
+  long long bits = __double_as_longlong(x);
+  int e = (int)((bits >> 52) & 0x7ff) - 1023;
+  double m = __longlong_as_double((bits & 0x000fffffffffffffll) | 0x3ff0000000000000ll);
+  if (m > 1.4142135623730951) {
+    m *= 0.5;
+    e += 1;
+  }
+  const double den = m + 1.0;
+  double y = (double)(1.0f / (float)den);
+  y = fma(y, fma(-den, y, 1.0), y);
+  y = fma(y, fma(-den, y, 1.0), y);
+  const double s = (m - 1.0) * y;
+  const double s2 = s * s;
+  double p;
+  if (FULL) {
+    p = 1.0 / 23;
+    p = fma(p, s2, 1.0 / 21);
+    p = fma(p, s2, 1.0 / 19);
+    p = fma(p, s2, 1.0 / 17);
+    p = fma(p, s2, 1.0 / 15);
+  } else {
+    p = 1.0 / 15;
+  }
+  p = fma(p, s2, 1.0 / 13);
+  p = fma(p, s2, 1.0 / 11);
+  p = fma(p, s2, 1.0 / 9);
+  p = fma(p, s2, 1.0 / 7);
+  p = fma(p, s2, 1.0 / 5);
+  p = fma(p, s2, 1.0 / 3);
+  p = fma(p, s2, 1.0);
+  const double ln2_hi = 6.93147180369123816490e-01;  // 2^-32 accurate
+  const double ln2_lo = 1.90821492927058770002e-10;
+  const double lnm = 2.0 * s * p;
+  const double t_hi = a * (double)e * ln2_hi;
+  const double t_lo = a * ((double)e * ln2_lo + lnm);
+  const double t = t_hi + t_lo;
+  const double n = rint(t * 1.44269504088896340736);
+  const double r = (t_hi - n * ln2_hi) + (t_lo - n * ln2_lo);
+  double q;
+  if (FULL) {
+    q = 1.0 / 355687428096000.0;  // 1/17!
+    q = fma(q, r, 1.0 / 20922789888000.0);
+    q = fma(q, r, 1.0 / 1307674368000.0);
+    q = fma(q, r, 1.0 / 87178291200.0);
+    q = fma(q, r, 1.0 / 6227020800.0);
+    q = fma(q, r, 1.0 / 479001600.0);
+    q = fma(q, r, 1.0 / 39916800.0);
+  } else {
+    q = 1.0 / 39916800.0;  // 1/11!
+  }
+  q = fma(q, r, 1.0 / 3628800.0);
+  q = fma(q, r, 1.0 / 362880.0);
+  q = fma(q, r, 1.0 / 40320.0);
+  q = fma(q, r, 1.0 / 5040.0);
+  q = fma(q, r, 1.0 / 720.0);
+  q = fma(q, r, 1.0 / 120.0);
+  q = fma(q, r, 1.0 / 24.0);
+  q = fma(q, r, 1.0 / 6.0);
+  q = fma(q, r, 0.5);
+  q = fma(q, r, 1.0);
+  q = fma(q, r, 1.0);
+  const long long ni = (long long)n;
+  return q * __longlong_as_double((ni + 1023) << 52);
+}
+
+// ---------------------------------------------------------------------------
+// Bulk asynchronous copies (TMA, cp.async.bulk) and mbarriers.  Addresses
+// and sizes are multiples of 16 bytes.  Every wait on an mbarrier is bounded:
+// after ~1 s of clock cycles it records DEVERR_TIMEOUT and gives up.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_u32(const void *p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+__device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)),
+               "r"(count)
+               : "memory");
+}
+__device__ __forceinline__ void fence_mbar_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+// make this thread's shared-memory writes visible to the bulk-copy engine
+__device__ __forceinline__ void fence_proxy_async() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+// arrive once and expect `bytes` of bulk-copy transactions (0: plain arrive)
+__device__ __forceinline__ void mbar_expect_tx(uint64_t *bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(
+                   smem_u32(bar)),
+               "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void tma_load(void *dst_smem, const void *src,
+                                         uint32_t bytes, uint64_t *bar,
+                                         uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1], %2, [%3], %4;" ::"r"(smem_u32(dst_smem)),
+      "l"(src), "r"(bytes), "r"(smem_u32(bar)), "l"(policy)
+      : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;"
+      " selp.u32 %0, 1, 0, p; }"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity,
+                                          Ctrl *ctrl) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const long long t0 = clock64();
+  while (!mbar_try_wait(bar, parity)) {
+    if (clock64() - t0 > 2000000000ll) {
+      atomicOr(&ctrl->err, DEVERR_TIMEOUT);
+      return false;
+    }
+  }
+  return true;
+}
+__device__ __forceinline__ void tma_store(void *dst, const void *src_smem,
+                                          uint32_t bytes, uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.global.shared::cta.bulk_group.L2::cache_hint [%0], [%1], %2, %3;" ::"l"(dst),
+      "r"(smem_u32(src_smem)), "r"(bytes), "l"(policy)
+      : "memory");
+}
+__device__ __forceinline__ void tma_commit() {
+  asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+// wait until at most N committed store groups still read shared memory
+template <int N>
+__device__ __forceinline__ void tma_wait_read() {
+  asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+__device__ __forceinline__ void tma_wait_all() {
+  asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+}
+
+// L2 residency hints: payload streams through (an evict_first policy) so
+// the small, reused priority tree stays resident (evict_last).
+__device__ __forceinline__ uint64_t policy_stream() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+__device__ __forceinline__ uint64_t policy_keep() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+__device__ __forceinline__ uint64_t ld_keep(const uint64_t *p, uint64_t pol) {
+  uint64_t v;
+  asm volatile("ld.global.L2::cache_hint.u64 %0, [%1], %2;"
+               : "=l"(v) : "l"(p), "l"(pol));
+  return v;
+}
+__device__ __forceinline__ uint32_t ld_keep(const uint32_t *p, uint64_t pol) {
+  uint32_t v;
+  asm volatile("ld.global.L2::cache_hint.u32 %0, [%1], %2;"
+               : "=r"(v) : "l"(p), "l"(pol));
+  return v;
+}
+__device__ __forceinline__ uint32_t ld_stream(const uint32_t *p, uint64_t pol) {
+  uint32_t v;
+  asm volatile("ld.global.nc.L1::no_allocate.L2::cache_hint.u32 %0, [%1], %2;"
+               : "=r"(v) : "l"(p), "l"(pol));
+  return v;
+}
+__device__ __forceinline__ uint2 ld_stream(const uint2 *p, uint64_t pol) {
+  uint2 v;
+  asm volatile("ld.global.nc.L1::no_allocate.L2::cache_hint.v2.u32 {%0, %1}, [%2], %3;"
+               : "=r"(v.x), "=r"(v.y) : "l"(p), "l"(pol));
+  return v;
+}
+__device__ __forceinline__ void st_stream(float4 *p, float4 v, uint64_t pol) {
+  asm volatile("st.global.L1::no_allocate.L2::cache_hint.v4.f32 [%0], {%1, %2, %3, %4}, %5;"
+               :: "l"(p), "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w), "l"(pol)
+               : "memory");
+}
+__device__ __forceinline__ void st_stream(uint4 *p, uint4 v, uint64_t pol) {
+  asm volatile("st.global.L1::no_allocate.L2::cache_hint.v4.u32 [%0], {%1, %2, %3, %4}, %5;"
+               :: "l"(p), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w), "l"(pol)
+               : "memory");
+}
+
+__device__ __forceinline__ void flag(Ctrl *c, uint32_t bits,
+                                     unsigned long long detail) {
+  if ((atomicOr(&c->err, bits) & bits) == 0)
+    atomicCAS(&c->bad_index, 0ull, detail + 1);
+}
+
+// Grid-wide barrier for cooperative launches (all CTAs co-resident by
+// construction).  The wait is bounded: after ~`budget` clock cycles the CTA
+// records DEVERR_TIMEOUT and proceeds, so a fault can never hang the GPU.
+__device__ __forceinline__ void grid_barrier(Ctrl *c, unsigned nblocks) {
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    volatile uint32_t *gen = &c->bar_gen;
+    const uint32_t g = *gen;
+    __threadfence();
+    const uint32_t arrived = atomicAdd(&c->bar_count, 1u) + 1u;
+    if (arrived == nblocks) {
+      c->bar_count = 0;
+      __threadfence();
+      atomicAdd(&c->bar_gen, 1u);
+    } else {
+      const long long t0 = clock64();
+      while (*gen == g) {
+        __nanosleep(64);
+        if (clock64() - t0 > 4000000000ll) {  // ~2 s at 2 GHz
+          atomicOr(&c->err, DEVERR_TIMEOUT);
+          break;
+        }
+      }
+    }
+    __threadfence();
+  }
+  __syncthreads();
+}
+
+// Programmatic dependent launch (sm_90+): a kernel launched with
+// launch_pdl may be scheduled while its predecessor in the stream is still
+// running; pdl_wait() blocks until the predecessor has completed and its
+// writes are visible, so every such kernel calls it before touching memory.
+// pdl_launch() lets the next kernel in the stream start launching.  Both are
+// no-ops for a kernel launched without the attribute.
+__device__ __forceinline__ void pdl_wait() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_launch() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block,
+                       cudaStream_t s, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+}
+
+// ---------------------------------------------------------------------------
+// Launchers (host).  Each returns cudaGetLastError() after its launches.
+// ---------------------------------------------------------------------------
+cudaError_t launch_copy_rows(uint8_t *dst, uint64_t dst_cap, uint64_t first,
+                             const uint8_t *src, uint64_t n, uint64_t row_bytes,
+                             cudaStream_t s);
+cudaError_t launch_ingest_meta(edp_ctx *ctx, const edp_fields *src, uint64_t n,
+                               const uint32_t *q, cudaStream_t s);
+cudaError_t launch_demote(edp_ctx *ctx, uint64_t first_id, uint64_t n,
+                          cudaStream_t s);
+// rows [src_row, src_row + n) of an ingest source -> host-tier slots of ids
+// first_id .. first_id + n - 1
+cudaError_t launch_copy_rows_to_host(edp_ctx *ctx, const uint8_t *obs,
+                                     const int32_t *tokens, uint64_t src_row,
+                                     uint64_t first_id, uint64_t n,
+                                     cudaStream_t s);
+cudaError_t launch_tree_refresh(edp_ctx *ctx, uint64_t first_leaf,
+                                uint64_t count, cudaStream_t s);
+cudaError_t launch_tree_build_all(edp_ctx *ctx, cudaStream_t s);
+cudaError_t launch_sample_uniform(edp_ctx *ctx, uint32_t B, uint64_t seed,
+                                  uint64_t round, int64_t *idx, cudaStream_t s);
+cudaError_t launch_sample_prioritized(edp_ctx *ctx, uint32_t B, uint64_t seed,
+                                      uint64_t round, int64_t *idx,
+                                      uint32_t *q, cudaStream_t s);
+cudaError_t launch_permute(edp_ctx *ctx, uint32_t n, uint64_t seed,
+                           uint64_t round, int64_t *idx, cudaStream_t s);
+cudaError_t launch_update(edp_ctx *ctx, const int64_t *idx, const uint32_t *q,
+                          const float *td, double alpha, double eps, uint32_t n,
+                          cudaStream_t s);
+cudaError_t launch_prio_from_td(const float *td, uint32_t n, double alpha,
+                                double eps, uint32_t *q, cudaStream_t s);
+cudaError_t launch_deliver(edp_ctx *ctx, const int64_t *idx, uint32_t B,
+                           const edp_batch *out, cudaStream_t s);
+cudaError_t launch_gae(edp_ctx *ctx, const float *r, const float *v,
+                       const uint8_t *d, uint32_t T, uint32_t E, double gamma,
+                       double lambda, float *adv, float *ret, float *adv_norm,
+                       cudaStream_t s);
+cudaError_t launch_probe_read(const void *src, uint64_t bytes, uint64_t *fold,
+                              cudaStream_t s);
+
+// scratch owned by the context, grown on demand (not stream-ordered: the
+// caller makes the first call of a given size outside graph capture)
+void *ctx_scratch(edp_ctx *ctx, size_t bytes);
+uint32_t *ctx_qbuf(edp_ctx *ctx, size_t n);
+
+}  // namespace edp

@@ -1,0 +1,195 @@
+// k_ring.cu -- ingestion kernels: ring scatter of payload rows, metadata and
+// priority leaves, two-tier demotion, and the host-link read probe.
+//
+// Ingestion inserts transitions into the persistent buffer and maintains the
+// indices and metadata used for sampling and eviction (Sec. 2.2, off-policy
+// ingestion).  Payload rows are moved with 16-byte vector loads and stores,
+// several loads in flight per thread; the ring index arithmetic is done once
+// per row, never per element.
+#include "edp_internal.cuh"
+
+namespace edp {
+namespace {
+
+constexpr int kCopyThreads = 256;
+constexpr int kCopyUnroll = 4;
+
+// Copy n rows of cpr 16-byte chunks: src row (src_first + j) mod src_cap ->
+// dst row (dst_first + j) mod dst_cap.  Grid: x tiles the chunks of a row,
+// y strides over rows.  src may be page-locked host memory (mapped).
+__global__ void __launch_bounds__(kCopyThreads)
+k_copy_rows(uint8_t *__restrict__ dst, uint64_t dst_cap, uint64_t dst_first,
+            const uint8_t *__restrict__ src, uint64_t src_cap,
+            uint64_t src_first, uint64_t n, uint32_t cpr) {
+  const uint64_t row_bytes = (uint64_t)cpr * 16u;
+  for (uint64_t j = blockIdx.y; j < n; j += gridDim.y) {
+    const uint64_t ds = (dst_first + j) % dst_cap;
+    const uint64_t ss = (src_first + j) % src_cap;
+    const uint4 *s = reinterpret_cast<const uint4 *>(src + ss * row_bytes);
+    uint4 *d = reinterpret_cast<uint4 *>(dst + ds * row_bytes);
+    const uint32_t step = gridDim.x * kCopyThreads * kCopyUnroll;
+    for (uint32_t w0 = blockIdx.x * kCopyThreads * kCopyUnroll + threadIdx.x;
+         w0 < cpr; w0 += step) {
+      uint4 v[kCopyUnroll];
+#pragma unroll
+      for (int u = 0; u < kCopyUnroll; ++u) {
+        const uint32_t w = w0 + u * kCopyThreads;
+        if (w < cpr) v[u] = s[w];
+      }
+#pragma unroll
+      for (int u = 0; u < kCopyUnroll; ++u) {
+        const uint32_t w = w0 + u * kCopyThreads;
+        if (w < cpr) d[w] = v[u];
+      }
+    }
+  }
+}
+
+cudaError_t copy_rows(uint8_t *dst, uint64_t dst_cap, uint64_t dst_first,
+                      const uint8_t *src, uint64_t src_cap, uint64_t src_first,
+                      uint64_t n, uint64_t row_bytes, cudaStream_t s) {
+  if (!n) return cudaSuccess;
+  const uint32_t cpr = (uint32_t)(row_bytes / 16);
+  uint32_t gx = (cpr + kCopyThreads * kCopyUnroll - 1) / (kCopyThreads * kCopyUnroll);
+  if (gx > 64) gx = 64;
+  const uint32_t gy = n < 65535 ? (uint32_t)n : 65535u;
+  k_copy_rows<<<dim3(gx, gy), kCopyThreads, 0, s>>>(dst, dst_cap, dst_first, src,
+                                                   src_cap, src_first, n, cpr);
+  return cudaGetLastError();
+}
+
+// Metadata of n new transitions at logical ids total.. and, for PER, their
+// leaves.  With `defer` the newest transition's leaf stays 0 and its
+// priority waits in ctrl->pending_q; the previous newest (id total-1) gets
+// its pending priority now -- unless this insertion overwrites its slot.
+__global__ void k_ingest_meta(int32_t *__restrict__ action,
+                              float *__restrict__ reward,
+                              uint8_t *__restrict__ done,
+                              const int32_t *__restrict__ s_action,
+                              const float *__restrict__ s_reward,
+                              const uint8_t *__restrict__ s_done,
+                              uint32_t *__restrict__ leaves,
+                              const uint32_t *__restrict__ q, Ctrl *ctrl,
+                              uint64_t cap, uint64_t total, uint64_t n,
+                              int defer) {
+  uint32_t qdefault = 0;
+  if (leaves && !q) qdefault = ctrl->max_q;
+  uint32_t qmax_local = 0;  // one atomic per warp, not per transition
+  for (uint64_t j = blockIdx.x * (uint64_t)blockDim.x + threadIdx.x; j < n;
+       j += (uint64_t)gridDim.x * blockDim.x) {
+    const uint64_t m = (total + j) % cap;
+    if (action) action[m] = s_action ? s_action[j] : 0;
+    if (reward) reward[m] = s_reward ? s_reward[j] : 0.f;
+    if (done) done[m] = s_done ? s_done[j] : (uint8_t)0;
+    if (leaves) {
+      const uint32_t qj = q ? q[j] : qdefault;
+      if (q) qmax_local = max(qmax_local, qj);
+      if (defer) {
+        leaves[m] = (j == n - 1) ? 0u : qj;
+        if (j == 0) {
+          // only this thread touches pending_q and the previous newest leaf
+          if (total >= 1 && n < cap) leaves[(total - 1) % cap] = ctrl->pending_q;
+          ctrl->pending_q = q ? q[n - 1] : qdefault;
+        }
+      } else {
+        leaves[m] = qj;
+      }
+    }
+  }
+  if (leaves && q) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1)
+      qmax_local = max(qmax_local, __shfl_xor_sync(0xffffffffu, qmax_local, o));
+    if ((threadIdx.x & 31) == 0 && qmax_local) atomicMax(&ctrl->max_q, qmax_local);
+  }
+}
+
+// Host-link probe: stream n16 16-byte words (page-locked host memory,
+// device-mapped) through the SMs, xor-folding them so no load is dead.
+__global__ void k_probe_read(const uint4 *__restrict__ src, uint64_t n16,
+                             unsigned long long *fold) {
+  uint4 acc = make_uint4(0, 0, 0, 0);
+  const uint64_t stride = (uint64_t)gridDim.x * blockDim.x;
+  uint64_t i = blockIdx.x * (uint64_t)blockDim.x + threadIdx.x;
+  for (; i + 3 * stride < n16; i += 4 * stride) {
+    const uint4 a = src[i], b = src[i + stride], c = src[i + 2 * stride],
+                d = src[i + 3 * stride];
+    acc.x ^= a.x ^ b.x ^ c.x ^ d.x;
+    acc.y ^= a.y ^ b.y ^ c.y ^ d.y;
+    acc.z ^= a.z ^ b.z ^ c.z ^ d.z;
+    acc.w ^= a.w ^ b.w ^ c.w ^ d.w;
+  }
+  for (; i < n16; i += stride) {
+    const uint4 a = src[i];
+    acc.x ^= a.x;
+    acc.y ^= a.y;
+    acc.z ^= a.z;
+    acc.w ^= a.w;
+  }
+  unsigned long long v = ((unsigned long long)(acc.x ^ acc.z) << 32) | (acc.y ^ acc.w);
+#pragma unroll
+  for (int o = 16; o; o >>= 1) v ^= __shfl_xor_sync(0xffffffffu, v, o);
+  if ((threadIdx.x & 31) == 0 && v) atomicXor(fold, v);
+}
+
+}  // namespace
+
+cudaError_t launch_copy_rows(uint8_t *dst, uint64_t dst_cap, uint64_t first,
+                             const uint8_t *src, uint64_t n, uint64_t row_bytes,
+                             cudaStream_t s) {
+  return copy_rows(dst, dst_cap, first, src, ~0ull, 0, n, row_bytes, s);
+}
+
+cudaError_t launch_ingest_meta(edp_ctx *c, const edp_fields *f, uint64_t n,
+                               const uint32_t *q, cudaStream_t s) {
+  if (!c->st.action && !c->st.reward && !c->st.done && !c->leaves)
+    return cudaSuccess;
+  const int threads = 256;
+  uint64_t blocks = (n + threads - 1) / threads;
+  if (blocks > 4096) blocks = 4096;
+  k_ingest_meta<<<(unsigned)blocks, threads, 0, s>>>(
+      c->st.action, c->st.reward, c->st.done, f->action, f->reward, f->done,
+      c->leaves, q, c->ctrl, c->cap, c->total, n, c->defer);
+  return cudaGetLastError();
+}
+
+// Two-tier demotion: payload of ids [first_id, first_id+n) moves from HBM
+// slot L mod cap_h to host slot L mod cap_c, before new payload overwrites
+// those HBM slots (same stream).
+cudaError_t launch_demote(edp_ctx *c, uint64_t first_id, uint64_t n,
+                          cudaStream_t s) {
+  cudaError_t e = copy_rows(c->st.host_obs, c->cap_c, first_id % c->cap_c,
+                            c->st.obs, c->cap_h, first_id % c->cap_h, n,
+                            c->obs_bytes, s);
+  if (e == cudaSuccess && c->tok_bytes)
+    e = copy_rows((uint8_t *)c->st.host_tokens, c->cap_c, first_id % c->cap_c,
+                  (const uint8_t *)c->st.tokens, c->cap_h, first_id % c->cap_h,
+                  n, c->tok_bytes, s);
+  return e;
+}
+
+cudaError_t launch_copy_rows_to_host(edp_ctx *c, const uint8_t *obs,
+                                     const int32_t *tokens, uint64_t src_row,
+                                     uint64_t first_id, uint64_t n,
+                                     cudaStream_t s) {
+  cudaError_t e = copy_rows(c->st.host_obs, c->cap_c, first_id % c->cap_c,
+                            obs + src_row * c->obs_bytes, ~0ull, 0, n,
+                            c->obs_bytes, s);
+  if (e == cudaSuccess && c->tok_bytes)
+    e = copy_rows((uint8_t *)c->st.host_tokens, c->cap_c, first_id % c->cap_c,
+                  (const uint8_t *)tokens + src_row * c->tok_bytes, ~0ull, 0, n,
+                  c->tok_bytes, s);
+  return e;
+}
+
+cudaError_t launch_probe_read(const void *src, uint64_t bytes, uint64_t *fold,
+                              cudaStream_t s) {
+  int sms = 0, dev = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  k_probe_read<<<sms * 4, 512, 0, s>>>((const uint4 *)src, bytes / 16,
+                                       (unsigned long long *)fold);
+  return cudaGetLastError();
+}
+
+}  // namespace edp

@@ -1,0 +1,413 @@
+// k_tree.cu -- the priority sum-tree of prioritized replay (Schaul et al.,
+// ICLR'16; the replay-state callback of Appendix C, Invariant 2):
+// refresh of ancestor sums, stratified inverse-CDF sampling by descent, and
+// the priority update with last-occurrence-wins duplicate handling.
+//
+// Layout: a 32-ary tree in fixed point.  Leaves are the uint32 priorities of
+// the ring slots (physical order, zero-padded to 32^D); level d < D holds
+// 32^d uint64 sums, node n of level d covering leaves [n*32^(D-d),
+// (n+1)*32^(D-d)).  Integer sums make every result independent of the order
+// in which threads add, so sums, targets and indices are bit-exact.
+//
+// One warp serves one tree node: a level is one coalesced 256-byte (or
+// 128-byte for leaves) load of the 32 children, a warp-shuffle inclusive
+// prefix sum and a ballot -- D dependent loads per descent instead of the
+// 5*D of a binary tree.
+#include "edp_internal.cuh"
+
+namespace edp {
+namespace {
+
+// Internal levels are stored back to back from the root: level d starts at
+// node (32^d - 1) / 31.
+struct TreeView {
+  uint64_t *nodes;
+  uint32_t *leaves;
+  uint32_t depth;
+  __device__ __forceinline__ uint64_t *lvl(uint32_t d) const {
+    return nodes + (((1ull << (5 * d)) - 1) / 31);
+  }
+};
+
+TreeView view(edp_ctx *c) {
+  TreeView t{};
+  t.nodes = c->level[0];
+  t.leaves = c->leaves;
+  t.depth = c->depth;
+  return t;
+}
+
+constexpr unsigned kFull = 0xffffffffu;
+
+__device__ __forceinline__ uint64_t warp_sum_u64(uint64_t v) {
+#pragma unroll
+  for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
+  return v;
+}
+
+// Recompute nodes [a0, a0+n0) and [a1, a1+n1) of level d from level d+1.
+__global__ void k_tree_level(uint64_t *__restrict__ out,
+                             const uint64_t *__restrict__ child64,
+                             const uint32_t *__restrict__ child32, uint64_t a0,
+                             uint64_t n0, uint64_t a1, uint64_t n1) {
+  const uint64_t w = (blockIdx.x * (uint64_t)blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (w >= n0 + n1) return;
+  const uint64_t node = w < n0 ? a0 + w : a1 + (w - n0);
+  const uint64_t c = node * kFanout + lane;
+  uint64_t v = child64 ? child64[c] : (uint64_t)child32[c];
+  v = warp_sum_u64(v);
+  if (lane == 0) out[node] = v;
+}
+
+// Stratified proportional sampling: one warp per stratum k.  The CTA first
+// copies the top of the tree (levels 1 and 2: 32 + 1024 sums, 8.2 KiB) into
+// shared memory, so a descent of a 1M-leaf tree makes two dependent global
+// loads (level 3, then the leaf row) instead of four.
+constexpr int kSmemLevels = 2;
+constexpr int kSmemNodes = 32 + 1024;
+
+__global__ void __launch_bounds__(256)
+k_sample_prio(TreeView t, uint32_t B, uint64_t seed, uint64_t round,
+              int64_t *__restrict__ idx, uint32_t *__restrict__ qout,
+              Ctrl *ctrl) {
+  __shared__ uint64_t top[kSmemNodes];
+  const int lane = threadIdx.x & 31;
+  const uint64_t keep = policy_keep();
+  pdl_wait();
+  pdl_launch();
+  const uint32_t cached = t.depth - 1 < (uint32_t)kSmemLevels ? t.depth - 1 : kSmemLevels;
+  const uint32_t ncached = cached == 0 ? 0 : (cached == 1 ? 32 : 32 + 1024);
+  for (uint32_t i = threadIdx.x; i < ncached; i += blockDim.x)
+    top[i] = t.nodes[1 + i];  // levels 1.. start right after the root
+  const uint64_t S = t.nodes[0];
+  __syncthreads();
+  const uint32_t warps = (gridDim.x * blockDim.x) >> 5;
+  for (uint32_t k = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; k < B;
+       k += warps) {
+    if (S == 0) {
+      if (lane == 0) {
+        idx[k] = -1;
+        if (qout) qout[k] = 0;
+        flag(ctrl, DEVERR_EMPTY, k);
+      }
+      continue;
+    }
+    // stratum [lo, hi) = [floor(kS/B), floor((k+1)S/B)); with S = aB + b,
+    // floor(kS/B) = ak + floor(bk/B), every term below 2^64.
+    const uint64_t a = S / B, b = S % B;
+    const uint64_t lo = a * k + (b * k) / B;
+    const uint64_t hi = a * (k + 1) + (b * (k + 1)) / B;
+    const uint64_t u = philox_u64(seed, k, round, 1);
+    uint64_t target = lo + mulhi64(u, hi - lo);
+    uint64_t node = 0;
+    bool ok = true;
+    for (uint32_t d = 1; d <= t.depth; ++d) {
+      const uint64_t c = node * kFanout + lane;
+      uint64_t v;
+      if (d <= cached)
+        v = top[(d == 1 ? 0 : 32) + c];
+      else
+        v = d < t.depth ? ld_keep(t.lvl(d) + c, keep) : (uint64_t)ld_keep(t.leaves + c, keep);
+      uint64_t incl = v;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint64_t y = __shfl_up_sync(kFull, incl, o);
+        if (lane >= o) incl += y;
+      }
+      unsigned m = __ballot_sync(kFull, target < incl);
+      if (m == 0) {  // sums disagree with children: report, stay in range
+        ok = false;
+        m = 1u << 31;
+      }
+      const int f = __ffs(m) - 1;
+      const uint64_t excl = __shfl_sync(kFull, incl - v, f);
+      target = target >= excl ? target - excl : 0;
+      node = node * kFanout + f;
+    }
+    if (lane == 0) {
+      if (!ok) flag(ctrl, DEVERR_TREE, k);
+      idx[k] = (int64_t)node;
+      if (qout) qout[k] = t.leaves[node];
+    }
+  }
+}
+
+// PER priority from a TD error: clamp(rn((|td| + eps)^alpha * 2^20), 1,
+// 2^32 - 1), fp64.
+__device__ __forceinline__ uint32_t prio_td(float td, double alpha, double eps) {
+  const double x = fabs((double)td) + eps;
+  double p = (x > 1e-300 && x < 1e300) ? pow_pos<true>(x, alpha) * 1048576.0
+                                       : pow(x, alpha) * 1048576.0;
+  double r = rint(p);
+  if (!(r >= 1.0)) r = 1.0;
+  if (r > 4294967295.0) r = 4294967295.0;
+  return (uint32_t)r;
+}
+
+__global__ void k_prio_from_td(const float *__restrict__ td, uint32_t n,
+                               double alpha, double eps,
+                               uint32_t *__restrict__ q) {
+  for (uint32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < n;
+       i += gridDim.x * blockDim.x)
+    q[i] = prio_td(td[i], alpha, eps);
+}
+
+constexpr int kUpdThreads = 512;
+constexpr int kUpdPer = 2;                          // pairs per thread per chunk
+constexpr int kUpdChunk = kUpdThreads * kUpdPer;
+constexpr int kUpdTable = 2 * kUpdChunk;            // open-addressing table
+constexpr uint32_t kEmpty = 0xffffffffu;
+
+__device__ __forceinline__ uint32_t tab_hash(uint32_t x, uint32_t mask) {
+  x ^= x >> 16;
+  x *= 0x45d9f3bu;
+  x ^= x >> 16;
+  return x & mask;
+}
+
+// Priority update.  Phase 1 (all CTAs): the priority of every pair -- the
+// given u32, or PER's rule from the TD error, whose fp64 pow is spread over
+// the CTAs -- goes to qbuf.  The last CTA to finish (ticket counter, no
+// waiting) then applies the pairs in batch order, in chunks of 2048 (two pairs per thread): a
+// shared-memory hash table keeps, per slot, the largest batch position
+// (atomicMax), so only the last occurrence of a slot writes its leaf.  The
+// exact signed delta of each written leaf is added to its ancestors
+// (two's complement wrap makes negative deltas exact); the two top levels,
+// which every pair shares, are summed on chip first.
+__global__ void __launch_bounds__(kUpdThreads, 1)
+k_update(TreeView t, const int64_t *__restrict__ idx,
+         const uint32_t *__restrict__ q, const float *__restrict__ td,
+         uint32_t *__restrict__ qbuf, double alpha, double eps, uint32_t n,
+         uint64_t cap, uint64_t oldest, uint64_t size, int defer, Ctrl *ctrl) {
+  __shared__ uint32_t hkey[kUpdTable];
+  __shared__ uint32_t hpos[kUpdTable];
+  __shared__ uint32_t ticket;
+  __shared__ uint32_t acc_lo[32], acc_hi[32];
+  __shared__ unsigned long long warp_root[kUpdThreads / 32];
+  const uint32_t *qv_src = q;
+  if (td) {
+    // phase 1 reads only the caller's TD errors, so it runs before the wait
+    // on the preceding kernel (overlapping it when SMs are free); one warp
+    // per CTA, one CTA per 32 pairs, so the fp64 work spreads over SMs
+    if (threadIdx.x < 32)
+      for (uint32_t p = blockIdx.x * 32 + threadIdx.x; p < n; p += gridDim.x * 32)
+        qbuf[p] = prio_td(td[p], alpha, eps);
+    __threadfence();
+    pdl_wait();
+    pdl_launch();
+    __syncthreads();
+    if (threadIdx.x == 0) ticket = atomicAdd(&ctrl->upd_count, 1u);
+    __syncthreads();
+    if (ticket != gridDim.x - 1) return;
+    __threadfence();
+    qv_src = qbuf;
+  } else {
+    pdl_wait();
+    pdl_launch();
+    if (blockIdx.x != 0) return;
+  }
+  const uint32_t tsize = n >= kUpdChunk ? kUpdTable
+                                        : max(64u, 2u << (31 - __clz(max(n, 1u))));
+  const uint32_t mask = tsize - 1;
+  uint32_t qmax_local = 0;  // running maximum: one atomic per CTA at the end
+  const int lane = threadIdx.x & 31;
+  unsigned long long root_sum = 0;
+  if (threadIdx.x < 32) {
+    acc_lo[threadIdx.x] = 0;
+    acc_hi[threadIdx.x] = 0;
+  }
+  for (uint32_t base = 0; base < n; base += kUpdChunk) {
+    const uint32_t cnt = min((uint32_t)kUpdChunk, n - base);
+    for (uint32_t i = threadIdx.x; i < tsize; i += kUpdThreads) {
+      hkey[i] = kEmpty;
+      hpos[i] = 0;
+    }
+    __syncthreads();
+    // every load of the chunk (index, priority, old leaf) is issued before
+    // the barrier; pairs are read in batch order p = r * threads + tid
+    int64_t s_[kUpdPer];
+    uint32_t qv_[kUpdPer], old_[kUpdPer];
+    uint64_t k_[kUpdPer];
+    bool holds_[kUpdPer];
+#pragma unroll
+    for (int r = 0; r < kUpdPer; ++r) {
+      const uint32_t p = r * kUpdThreads + threadIdx.x;
+      const bool active = p < cnt;
+      const int64_t sl = active ? idx[base + p] : -1;
+      const bool valid = active && sl >= 0 && (uint64_t)sl < cap;
+      if (active && !valid) flag(ctrl, DEVERR_INDEX, (unsigned long long)sl);
+      const uint64_t k = !valid ? 0
+                       : (uint64_t)sl >= oldest ? (uint64_t)sl - oldest
+                                                : (uint64_t)sl + cap - oldest;
+      const bool holds = valid && k < size;  // the slot holds a transition
+      s_[r] = sl;
+      k_[r] = k;
+      holds_[r] = holds;
+      qv_[r] = holds ? __ldcg(qv_src + base + p) : 0u;
+      old_[r] = holds ? t.leaves[sl] : 0u;
+      if (holds) {
+        const uint32_t key = (uint32_t)sl;
+        uint32_t h = tab_hash(key, mask);
+        for (uint32_t probe = 0; probe < tsize; ++probe) {
+          const uint32_t prev = atomicCAS(&hkey[h], kEmpty, key);
+          if (prev == kEmpty || prev == key) {
+            atomicMax(&hpos[h], p);
+            break;
+          }
+          h = (h + 1) & mask;
+        }
+      }
+    }
+    __syncthreads();
+#pragma unroll
+    for (int r = 0; r < kUpdPer; ++r) {
+      const uint32_t p = r * kUpdThreads + threadIdx.x;
+      const int64_t sl = s_[r];
+      const uint32_t qv = qv_[r];
+      qmax_local = max(qmax_local, qv);
+      bool win = false;
+      if (holds_[r]) {
+        uint32_t h = tab_hash((uint32_t)sl, mask);
+        for (uint32_t probe = 0; probe < tsize && hkey[h] != (uint32_t)sl; ++probe)
+          h = (h + 1) & mask;
+        win = hpos[h] == p;  // no later pair sets this slot
+      }
+      if (win && defer && k_[r] == size - 1) {
+        ctrl->pending_q = qv;
+        win = false;
+      }
+      unsigned long long delta = 0;
+      if (win) {
+        t.leaves[sl] = qv;
+        delta = (unsigned long long)((long long)qv - (long long)old_[r]);
+      }
+      // ancestors.  The root and level 1 (32 nodes) are shared by many
+      // pairs: the root delta is summed over the block (shuffles, then one
+      // atomic), level-1 deltas go to 32 shared accumulators kept as two
+      // 32-bit halves with explicit carries (exact mod 2^64).  Deeper nodes
+      // rarely collide and take one 64-bit atomic per pair.
+      root_sum += delta;
+      if (delta && t.depth >= 2) {
+        const uint32_t n1 = (uint32_t)((uint64_t)sl >> (5 * (t.depth - 1)));
+        const uint32_t lo = (uint32_t)delta, hi = (uint32_t)(delta >> 32);
+        const uint32_t old = atomicAdd(&acc_lo[n1], lo);
+        atomicAdd(&acc_hi[n1], hi + (old + lo < old ? 1u : 0u));
+      }
+      if (delta)
+        for (uint32_t d = 2; d < t.depth; ++d)
+          atomicAdd((unsigned long long *)&t.lvl(d)[(uint64_t)sl >> (5 * (t.depth - d))],
+                    delta);
+    }
+    // flush the chunk's root and level-1 sums
+#pragma unroll
+    for (int o = 16; o; o >>= 1) root_sum += __shfl_xor_sync(kFull, root_sum, o);
+    if (lane == 0) warp_root[threadIdx.x >> 5] = root_sum;
+    root_sum = 0;
+    __syncthreads();
+    if (threadIdx.x < 32 && t.depth >= 2) {
+      const unsigned long long v =
+          ((unsigned long long)acc_hi[threadIdx.x] << 32) | acc_lo[threadIdx.x];
+      if (v) atomicAdd((unsigned long long *)&t.lvl(1)[threadIdx.x], v);
+      acc_lo[threadIdx.x] = 0;
+      acc_hi[threadIdx.x] = 0;
+    }
+    if (threadIdx.x == 32) {
+      unsigned long long v = 0;
+      for (int w = 0; w < kUpdThreads / 32; ++w) v += warp_root[w];
+      if (v) atomicAdd((unsigned long long *)&t.nodes[0], v);
+    }
+    __syncthreads();
+  }
+#pragma unroll
+  for (int o = 16; o; o >>= 1)
+    qmax_local = max(qmax_local, __shfl_xor_sync(kFull, qmax_local, o));
+  if ((threadIdx.x & 31) == 0) ticket = 0;
+  __syncthreads();
+  if ((threadIdx.x & 31) == 0) atomicMax(&ticket, qmax_local);
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    if (ticket) atomicMax(&ctrl->max_q, ticket);
+    if (td) ctrl->upd_count = 0;  // ready for the next call
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_tree_refresh(edp_ctx *c, uint64_t first, uint64_t count,
+                                cudaStream_t s) {
+  if (!c->depth || !count) return cudaSuccess;
+  // leaf ranges [a0, b0) and [a1, b1) (the second only on ring wrap)
+  uint64_t a0 = first, b0 = first + count, a1 = 0, b1 = 0;
+  if (b0 > c->cap) {
+    b1 = b0 - c->cap;
+    b0 = c->cap;
+  }
+  for (int d = (int)c->depth - 1; d >= 0; --d) {
+    const unsigned shift = 5u * (c->depth - d);
+    uint64_t x0 = a0 >> shift, y0 = ((b0 - 1) >> shift) + 1;
+    uint64_t x1 = 0, y1 = 0;
+    if (b1 > a1) {
+      x1 = a1 >> shift;
+      y1 = ((b1 - 1) >> shift) + 1;
+      if (y1 >= x0) {  // ranges meet: one range covers both
+        x0 = x1 < x0 ? x1 : x0;
+        y0 = y1 > y0 ? y1 : y0;
+        x1 = y1 = 0;
+      }
+    }
+    const uint64_t nodes = (y0 - x0) + (y1 - x1);
+    const uint64_t threads = nodes * 32;
+    const unsigned blocks = (unsigned)((threads + 255) / 256);
+    const bool leaves_below = (uint32_t)(d + 1) == c->depth;
+    k_tree_level<<<blocks, 256, 0, s>>>(c->level[d],
+                                        leaves_below ? nullptr : c->level[d + 1],
+                                        leaves_below ? c->leaves : nullptr, x0,
+                                        y0 - x0, x1, y1 - x1);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+cudaError_t launch_tree_build_all(edp_ctx *c, cudaStream_t s) {
+  return launch_tree_refresh(c, 0, c->cap, s);
+}
+
+cudaError_t launch_sample_prioritized(edp_ctx *c, uint32_t B, uint64_t seed,
+                                      uint64_t round, int64_t *idx, uint32_t *q,
+                                      cudaStream_t s) {
+  const unsigned warps_per_block = 8;
+  uint64_t blocks = (B + warps_per_block - 1) / warps_per_block;
+  if (blocks > 8u * (unsigned)c->coop_sms) blocks = 8u * (unsigned)c->coop_sms;
+  return launch_pdl(k_sample_prio, dim3((unsigned)blocks), dim3(warps_per_block * 32),
+                    s, view(c), B, seed, round, idx, q, c->ctrl);
+}
+
+cudaError_t launch_update(edp_ctx *c, const int64_t *idx, const uint32_t *q,
+                          const float *td, double alpha, double eps, uint32_t n,
+                          cudaStream_t s) {
+  const uint64_t size = c->total < c->cap ? c->total : c->cap;
+  const uint64_t oldest = (c->total - size) % c->cap;
+  uint32_t *qbuf = nullptr;
+  unsigned grid = 1;
+  if (td) {
+    qbuf = ctx_qbuf(c, n);
+    if (!qbuf) return cudaErrorMemoryAllocation;
+    // 32 priorities (one warp) per CTA: the fp64 work spreads over SMs
+    grid = (n + 31) / 32;
+    if (grid > 2u * (unsigned)c->coop_sms) grid = 2u * (unsigned)c->coop_sms;
+  }
+  return launch_pdl(k_update, dim3(grid), dim3(kUpdThreads), s, view(c), idx, q,
+                    td, qbuf, alpha, eps, n, c->cap, oldest, size, c->defer,
+                    c->ctrl);
+}
+
+cudaError_t launch_prio_from_td(const float *td, uint32_t n, double alpha,
+                                double eps, uint32_t *q, cudaStream_t s) {
+  const unsigned blocks = (n + 255) / 256 < 1024 ? (n + 255) / 256 : 1024;
+  k_prio_from_td<<<blocks, 256, 0, s>>>(td, n, alpha, eps, q);
+  return cudaGetLastError();
+}
+
+}  // namespace edp

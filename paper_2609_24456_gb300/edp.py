@@ -1,0 +1,306 @@
+"""Thin Python binding of libedp (C ABI declared in include/edp.h).
+
+Argument marshalling only: every function forwards to the C entry point of the
+same name, converting torch tensors to raw pointers and torch streams to
+``cudaStream_t``.  PyTorch supplies device memory, page-locked host memory and
+streams; every step of the data path runs in libedp's CUDA kernels.  There is
+no fallback: if libedp.so cannot be loaded, every call raises.
+"""
+import ctypes as C
+import os
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libedp.so")
+
+EDP_OK, EDP_ERR_INVALID, EDP_ERR_OOM, EDP_ERR_CUDA, EDP_ERR_TIMEOUT, \
+    EDP_ERR_EMPTY, EDP_ERR_STATE = range(7)
+STATUS_NAMES = ["EDP_OK", "EDP_ERR_INVALID", "EDP_ERR_OOM", "EDP_ERR_CUDA",
+                "EDP_ERR_TIMEOUT", "EDP_ERR_EMPTY", "EDP_ERR_STATE"]
+EDP_XFORM_STACK_F32, EDP_XFORM_HWC_CHW_BF16, EDP_XFORM_CHW_NORM_BF16 = range(3)
+EDP_SAMPLE_UNIFORM, EDP_SAMPLE_PRIORITIZED, EDP_SAMPLE_PERMUTE = range(3)
+
+ALLOC_FN = C.CFUNCTYPE(C.c_void_p, C.c_void_p, C.c_size_t)
+FREE_FN = C.CFUNCTYPE(None, C.c_void_p, C.c_void_p)
+
+
+class edp_config(C.Structure):
+    _fields_ = [("capacity", C.c_uint64), ("hbm_capacity", C.c_uint64),
+                ("obs_c", C.c_uint32), ("obs_h", C.c_uint32),
+                ("obs_w", C.c_uint32), ("transform", C.c_uint32),
+                ("frame_stack", C.c_uint32), ("next_obs", C.c_uint32),
+                ("tokens", C.c_uint32), ("prioritized", C.c_uint32),
+                ("norm_mean", C.c_float * 4), ("norm_std", C.c_float * 4),
+                ("alloc", ALLOC_FN), ("free", FREE_FN),
+                ("alloc_user", C.c_void_p), ("device", C.c_int32),
+                ("reserved", C.c_uint32 * 7)]
+
+
+class edp_storage(C.Structure):
+    _fields_ = [("obs", C.c_void_p), ("tokens", C.c_void_p),
+                ("host_obs", C.c_void_p), ("host_tokens", C.c_void_p),
+                ("action", C.c_void_p), ("reward", C.c_void_p),
+                ("done", C.c_void_p)]
+
+
+class edp_fields(C.Structure):
+    _fields_ = [("obs", C.c_void_p), ("tokens", C.c_void_p),
+                ("action", C.c_void_p), ("reward", C.c_void_p),
+                ("done", C.c_void_p)]
+
+
+class edp_batch(C.Structure):
+    _fields_ = [("obs", C.c_void_p), ("next_obs", C.c_void_p),
+                ("action", C.c_void_p), ("reward", C.c_void_p),
+                ("done", C.c_void_p), ("tokens", C.c_void_p),
+                ("q", C.c_void_p), ("isw", C.c_void_p), ("beta", C.c_double),
+                ("gather_src", C.c_void_p * 2), ("gather_dst", C.c_void_p * 2)]
+
+
+class edp_info(C.Structure):
+    _fields_ = [("capacity", C.c_uint64), ("hbm_capacity", C.c_uint64),
+                ("total", C.c_uint64), ("size", C.c_uint64),
+                ("head", C.c_uint64), ("oldest", C.c_uint64),
+                ("n_valid", C.c_uint64), ("tree_depth", C.c_uint32),
+                ("tree_fanout", C.c_uint32), ("tree_leaves", C.c_void_p),
+                ("tree_level", C.c_void_p * 8), ("pending_q", C.c_void_p),
+                ("max_q", C.c_void_p)]
+
+
+# exported symbols and their signatures (restype, argtypes)
+_VP, _U32, _U64, _D = C.c_void_p, C.c_uint32, C.c_uint64, C.c_double
+SIGNATURES = {
+    "edp_create": (C.c_int, [C.POINTER(edp_config), C.POINTER(edp_storage),
+                             C.POINTER(C.c_void_p)]),
+    "edp_destroy": (C.c_int, [_VP]),
+    "edp_ingest": (C.c_int, [_VP, C.POINTER(edp_fields), _U64, _VP, _VP]),
+    "edp_sample": (C.c_int, [_VP, C.c_int, _U32, _U64, _U64, _VP, _VP, _VP]),
+    "edp_deliver": (C.c_int, [_VP, _VP, _U32, C.POINTER(edp_batch), _VP]),
+    "edp_update_priorities": (C.c_int, [_VP, _VP, _VP, _U32, _VP]),
+    "edp_update_priorities_td": (C.c_int, [_VP, _VP, _VP, _U32, _D, _D, _VP]),
+    "edp_priorities_from_td": (C.c_int, [_VP, _VP, _U32, _D, _D, _VP, _VP]),
+    "edp_gae": (C.c_int, [_VP, _VP, _VP, _VP, _U32, _U32, _D, _D, _VP, _VP,
+                          _VP, _VP]),
+    "edp_sync": (C.c_int, [_VP, _VP]),
+    "edp_last_error": (C.c_char_p, [_VP]),
+    "edp_get_info": (C.c_int, [_VP, C.POINTER(edp_info)]),
+    "edp_probe_host_read": (C.c_int, [_VP, _U64, _VP, _VP]),
+    "edp_abi_version": (C.c_int, []),
+}
+
+_lib = None
+
+
+def lib():
+    """Load libedp.so (raises if it is missing: there is no fallback)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(
+                "libedp.so not built (%s); run paper_2609_24456_gb300.build.build()"
+                % LIB_PATH)
+        L = C.CDLL(LIB_PATH)
+        for name, (res, args) in SIGNATURES.items():
+            fn = getattr(L, name)
+            fn.restype = res
+            fn.argtypes = args
+        _lib = L
+    return _lib
+
+
+class EdpError(RuntimeError):
+    def __init__(self, status, msg):
+        self.status = status
+        name = STATUS_NAMES[status] if 0 <= status < len(STATUS_NAMES) else str(status)
+        super().__init__("%s: %s" % (name, msg))
+
+
+def ptr(x):
+    """Raw address of a tensor / int / None."""
+    if x is None:
+        return None
+    if isinstance(x, int):
+        return x
+    return x.data_ptr()
+
+
+def stream_handle(stream):
+    if stream is None:
+        import torch
+        stream = torch.cuda.current_stream()
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def _check(ctx, status, what):
+    if status != EDP_OK:
+        msg = lib().edp_last_error(ctx) if ctx else b""
+        raise EdpError(status, "%s: %s" % (what, (msg or b"").decode()))
+    return status
+
+
+# --- the C entry points -------------------------------------------------------
+def edp_create(cfg: edp_config, st: edp_storage) -> int:
+    out = C.c_void_p()
+    s = lib().edp_create(C.byref(cfg), C.byref(st), C.byref(out))
+    if s != EDP_OK:
+        raise EdpError(s, "edp_create failed (details on stderr)")
+    return out.value
+
+
+def edp_destroy(ctx):
+    return _check(None, lib().edp_destroy(ctx), "edp_destroy")
+
+
+def edp_ingest(ctx, obs, n, tokens=None, action=None, reward=None, done=None,
+               q=None, stream=None):
+    f = edp_fields(ptr(obs), ptr(tokens), ptr(action), ptr(reward), ptr(done))
+    return _check(ctx, lib().edp_ingest(ctx, C.byref(f), n, ptr(q),
+                                        stream_handle(stream)), "edp_ingest")
+
+
+def edp_sample(ctx, mode, batch, seed, round_, idx, q=None, stream=None):
+    return _check(ctx, lib().edp_sample(ctx, mode, batch, seed, round_, ptr(idx),
+                                        ptr(q), stream_handle(stream)),
+                  "edp_sample")
+
+
+def make_batch(obs, next_obs=None, action=None, reward=None, done=None,
+               tokens=None, q=None, isw=None, beta=0.0, gather=()):
+    b = edp_batch()
+    b.obs, b.next_obs = ptr(obs), ptr(next_obs)
+    b.action, b.reward, b.done = ptr(action), ptr(reward), ptr(done)
+    b.tokens, b.q, b.isw, b.beta = ptr(tokens), ptr(q), ptr(isw), float(beta)
+    for i, (src, dst) in enumerate(gather):
+        b.gather_src[i] = ptr(src)
+        b.gather_dst[i] = ptr(dst)
+    return b
+
+
+def edp_deliver(ctx, idx, batch, out: edp_batch, stream=None):
+    return _check(ctx, lib().edp_deliver(ctx, ptr(idx), batch, C.byref(out),
+                                         stream_handle(stream)), "edp_deliver")
+
+
+def edp_update_priorities(ctx, idx, q, n, stream=None):
+    return _check(ctx, lib().edp_update_priorities(ctx, ptr(idx), ptr(q), n,
+                                                   stream_handle(stream)),
+                  "edp_update_priorities")
+
+
+def edp_update_priorities_td(ctx, idx, td, n, alpha, eps, stream=None):
+    return _check(ctx, lib().edp_update_priorities_td(
+        ctx, ptr(idx), ptr(td), n, alpha, eps, stream_handle(stream)),
+        "edp_update_priorities_td")
+
+
+def edp_priorities_from_td(ctx, td, n, alpha, eps, q, stream=None):
+    return _check(ctx, lib().edp_priorities_from_td(
+        ctx, ptr(td), n, alpha, eps, ptr(q), stream_handle(stream)),
+        "edp_priorities_from_td")
+
+
+def edp_gae(ctx, r, v, d, T, E, gamma, lam, adv=None, ret=None, adv_norm=None,
+            stream=None):
+    return _check(ctx, lib().edp_gae(ctx, ptr(r), ptr(v), ptr(d), T, E, gamma,
+                                     lam, ptr(adv), ptr(ret), ptr(adv_norm),
+                                     stream_handle(stream)), "edp_gae")
+
+
+def edp_sync(ctx, stream=None):
+    return _check(ctx, lib().edp_sync(ctx, stream_handle(stream)), "edp_sync")
+
+
+def edp_sync_status(ctx, stream=None):
+    """edp_sync returning (status, message) instead of raising."""
+    s = lib().edp_sync(ctx, stream_handle(stream))
+    return s, (lib().edp_last_error(ctx) or b"").decode()
+
+
+def edp_last_error(ctx):
+    return (lib().edp_last_error(ctx) or b"").decode()
+
+
+def edp_get_info(ctx) -> edp_info:
+    out = edp_info()
+    _check(ctx, lib().edp_get_info(ctx, C.byref(out)), "edp_get_info")
+    return out
+
+
+def edp_probe_host_read(host_src, nbytes, d_fold, stream=None):
+    s = lib().edp_probe_host_read(ptr(host_src), nbytes, ptr(d_fold),
+                                  stream_handle(stream))
+    if s != EDP_OK:
+        raise EdpError(s, "edp_probe_host_read")
+
+
+def edp_abi_version():
+    return lib().edp_abi_version()
+
+
+# --- storage plumbing (torch allocations) -------------------------------------
+def make_config(capacity, obs_shape, transform, hbm_capacity=None,
+                frame_stack=1, next_obs=False, tokens=0, prioritized=False,
+                norm_mean=(0.0,) * 4, norm_std=(1.0,) * 4, device=0):
+    """obs_shape = (c, h, w) of the stored observation."""
+    cfg = edp_config()
+    cfg.capacity = capacity
+    cfg.hbm_capacity = capacity if hbm_capacity is None else hbm_capacity
+    cfg.obs_c, cfg.obs_h, cfg.obs_w = obs_shape
+    cfg.transform = transform
+    cfg.frame_stack = frame_stack
+    cfg.next_obs = int(bool(next_obs))
+    cfg.tokens = tokens
+    cfg.prioritized = int(bool(prioritized))
+    for i in range(4):
+        cfg.norm_mean[i] = list(norm_mean)[i] if i < len(norm_mean) else 0.0
+        cfg.norm_std[i] = list(norm_std)[i] if i < len(norm_std) else 1.0
+    cfg.device = device
+    return cfg
+
+
+class Ring:
+    """Caller-side storage of a ring plus its context handle.
+
+    Tensors are allocated with torch (device memory for HBM fields,
+    pin_memory for the host tier) and handed to edp_create as raw pointers.
+    """
+
+    def __init__(self, cfg: edp_config, action=True, reward=True, done=True):
+        import torch
+        self.cfg = cfg
+        dev = torch.device("cuda", cfg.device)
+        ob = cfg.obs_c * cfg.obs_h * cfg.obs_w
+        cap, cap_h = cfg.capacity, cfg.hbm_capacity
+        self.obs = torch.empty((cap_h, ob), dtype=torch.uint8, device=dev)
+        self.tokens = (torch.empty((cap_h, cfg.tokens), dtype=torch.int32,
+                                   device=dev) if cfg.tokens else None)
+        self.host_obs = self.host_tokens = None
+        if cap_h < cap:
+            self.host_obs = torch.empty((cap - cap_h, ob), dtype=torch.uint8,
+                                        pin_memory=True)
+            if cfg.tokens:
+                self.host_tokens = torch.empty((cap - cap_h, cfg.tokens),
+                                               dtype=torch.int32,
+                                               pin_memory=True)
+        self.action = torch.zeros(cap, dtype=torch.int32, device=dev) if action else None
+        self.reward = torch.zeros(cap, dtype=torch.float32, device=dev) if reward else None
+        self.done = torch.zeros(cap, dtype=torch.uint8, device=dev) if done else None
+        st = edp_storage(ptr(self.obs), ptr(self.tokens), ptr(self.host_obs),
+                         ptr(self.host_tokens), ptr(self.action),
+                         ptr(self.reward), ptr(self.done))
+        self.ctx = edp_create(cfg, st)
+
+    def info(self):
+        return edp_get_info(self.ctx)
+
+    def close(self):
+        if self.ctx:
+            edp_destroy(self.ctx)
+            self.ctx = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
