@@ -247,6 +247,26 @@ EDP_API edp_status edp_update_priorities_td(edp_ctx *ctx, const int64_t *idx,
                                     const float *td, uint32_t n, double alpha,
                                     double eps, edp_stream stream);
 
+/* edp_update_priorities_td without any device allocation.  The paper has no
+ * counterpart: this entry point exists for callers that cannot allocate
+ * device memory when they update priorities -- code being captured into a
+ * CUDA graph, where cudaMalloc may not be called, and runtimes that hand out
+ * all device memory at start-up and forbid later allocation, or cannot
+ * afford the device-wide synchronisation an allocation may bring.
+ * edp_update_priorities_td allocates its scratch (one uint32 per pair) on
+ * first use; this variant keeps that scratch in a fixed per-device array of
+ * 16384 pairs (64 KiB), held by every GPU that loads libedp until the process
+ * exits.  n > 16384 returns EDP_ERR_INVALID.  The first call on a device
+ * looks up the array's device address (make it before any stream capture).
+ * All calls on a device share the array, so calls that overlap on the GPU --
+ * on any stream or context -- race; the array keeps the last call's
+ * contents, which a call never reads before writing.  Results equal those of
+ * edp_update_priorities_td for the same arguments. */
+EDP_API edp_status edp_update_priorities_td_static(edp_ctx *ctx, const int64_t *idx,
+                                                   const float *td, uint32_t n,
+                                                   double alpha, double eps,
+                                                   edp_stream stream);
+
 /* The TD-error rule alone: q[i] from td[i] (device arrays [n]). */
 EDP_API edp_status edp_priorities_from_td(edp_ctx *ctx, const float *td, uint32_t n,
                                   double alpha, double eps, uint32_t *q,

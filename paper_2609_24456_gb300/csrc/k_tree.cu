@@ -411,3 +411,107 @@ cudaError_t launch_prio_from_td(const float *td, uint32_t n, double alpha,
 }
 
 }  // namespace edp
+
+// ---------------------------------------------------------------------------
+// Allocation-free priority update.  Same kernel as edp_update_priorities_td,
+// but the per-pair priorities computed from the TD errors go to the fixed
+// array below instead of context-owned scratch that is allocated on first
+// use.  Callers that must not allocate device memory use it: code being
+// captured into a CUDA graph (cudaMalloc may not be called during stream
+// capture), and runtimes that hand out all device memory up front and forbid
+// allocation later, or that cannot afford the device-wide synchronisation a
+// cudaMalloc/cudaFree may bring.  The array is per device and lives until
+// the process exits; every call on that device shares it, so calls that
+// overlap on the GPU race.  Nothing in it needs to start at zero: a call
+// writes priorities [0, n) before it reads them.
+// ---------------------------------------------------------------------------
+#include <mutex>
+
+namespace edp {
+namespace {
+
+constexpr uint32_t kStaticMaxPairs = 16384;  // 64 KiB of priorities
+static __device__ __align__(256) uint32_t g_static_qbuf[kStaticMaxPairs];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_static_mu;
+uint32_t *g_static_ptr[kMaxDevices] = {};
+
+// Device address of g_static_qbuf on the current device (looked up once per
+// device; the host-side name is only a stand-in for the device symbol).
+cudaError_t static_qbuf(int dev, uint32_t **out) {
+  std::lock_guard<std::mutex> lock(g_static_mu);
+  if (!g_static_ptr[dev]) {
+    void *p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_static_qbuf);
+    if (e != cudaSuccess) return e;
+    g_static_ptr[dev] = (uint32_t *)p;
+  }
+  *out = g_static_ptr[dev];
+  return cudaSuccess;
+}
+
+bool is_device_ptr(const void *p, int dev) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return (a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged) &&
+         a.device == dev;
+}
+
+}  // namespace
+}  // namespace edp
+
+extern "C" edp_status edp_update_priorities_td_static(
+    edp_ctx *ctx, const int64_t *idx, const float *td, uint32_t n,
+    double alpha, double eps, edp_stream stream) {
+  using namespace edp;
+  if (!ctx) return EDP_ERR_INVALID;
+  if (!ctx->depth) {
+    ctx->err = "edp_update_priorities_td_static: context has no priorities";
+    return EDP_ERR_STATE;
+  }
+  if (n == 0) return EDP_OK;
+  if (n > kStaticMaxPairs) {
+    ctx->err = "edp_update_priorities_td_static: n exceeds the fixed maximum "
+               "of 16384 pairs (use edp_update_priorities_td)";
+    return EDP_ERR_INVALID;
+  }
+  if (!idx || !td || !is_device_ptr(idx, ctx->cfg.device) ||
+      !is_device_ptr(td, ctx->cfg.device)) {
+    ctx->err = "edp_update_priorities_td_static: idx and td must be device memory";
+    return EDP_ERR_INVALID;
+  }
+  if (!(alpha >= 0.0 && eps >= 0.0)) {
+    ctx->err = "edp_update_priorities_td_static: alpha, eps >= 0";
+    return EDP_ERR_INVALID;
+  }
+  if (ctx->cfg.device < 0 || ctx->cfg.device >= kMaxDevices) {
+    ctx->err = "edp_update_priorities_td_static: device ordinal out of range";
+    return EDP_ERR_INVALID;
+  }
+  cudaSetDevice(ctx->cfg.device);
+  uint32_t *qbuf = nullptr;
+  cudaError_t e = static_qbuf(ctx->cfg.device, &qbuf);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    ctx->err = std::string("edp_update_priorities_td_static: cudaGetSymbolAddress: ") +
+               cudaGetErrorString(e);
+    return EDP_ERR_CUDA;
+  }
+  const uint64_t size = ctx->total < ctx->cap ? ctx->total : ctx->cap;
+  const uint64_t oldest = (ctx->total - size) % ctx->cap;
+  unsigned grid = (n + 31) / 32;
+  if (grid > 2u * (unsigned)ctx->coop_sms) grid = 2u * (unsigned)ctx->coop_sms;
+  e = launch_pdl(k_update, dim3(grid), dim3(kUpdThreads), (cudaStream_t)stream,
+                 view(ctx), idx, (const uint32_t *)nullptr, td, qbuf, alpha, eps, n,
+                 ctx->cap, oldest, size, ctx->defer, ctx->ctrl);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    ctx->err = std::string("edp_update_priorities_td_static: ") + cudaGetErrorString(e);
+    return EDP_ERR_CUDA;
+  }
+  return EDP_OK;
+}

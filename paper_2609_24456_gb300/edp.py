@@ -77,6 +77,7 @@ SIGNATURES = {
     "edp_deliver": (C.c_int, [_VP, _VP, _U32, C.POINTER(edp_batch), _VP]),
     "edp_update_priorities": (C.c_int, [_VP, _VP, _VP, _U32, _VP]),
     "edp_update_priorities_td": (C.c_int, [_VP, _VP, _VP, _U32, _D, _D, _VP]),
+    "edp_update_priorities_td_static": (C.c_int, [_VP, _VP, _VP, _U32, _D, _D, _VP]),
     "edp_priorities_from_td": (C.c_int, [_VP, _VP, _U32, _D, _D, _VP, _VP]),
     "edp_gae": (C.c_int, [_VP, _VP, _VP, _VP, _U32, _U32, _D, _D, _VP, _VP,
                           _VP, _VP]),
@@ -192,6 +193,14 @@ def edp_update_priorities_td(ctx, idx, td, n, alpha, eps, stream=None):
     return _check(ctx, lib().edp_update_priorities_td(
         ctx, ptr(idx), ptr(td), n, alpha, eps, stream_handle(stream)),
         "edp_update_priorities_td")
+
+
+def edp_update_priorities_td_static(ctx, idx, td, n, alpha, eps, stream=None):
+    """Allocation-free edp_update_priorities_td (fixed per-device scratch of
+    16384 pairs; see include/edp.h)."""
+    return _check(ctx, lib().edp_update_priorities_td_static(
+        ctx, ptr(idx), ptr(td), n, alpha, eps, stream_handle(stream)),
+        "edp_update_priorities_td_static")
 
 
 def edp_priorities_from_td(ctx, td, n, alpha, eps, q, stream=None):
