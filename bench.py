@@ -17,6 +17,8 @@ workload and metric; each step is one round of the same per-round work.
 """
 import argparse
 import ctypes
+
+import numpy as np
 import hashlib
 import json
 import os
@@ -190,12 +192,76 @@ def oracle_threads():
 
 
 # ----------------------------------------------------------------------------
-# Workload: prioritized replay, 1,000,000 frames of 84x84, batch 512
+# Workloads.  A workload fixes the synthetic data, the step (one pass of its
+# hot path), the algorithmic bytes of a step and of its dominant kernel, the
+# end-to-end user path and the oracle's bounded CPU sample.
 # ----------------------------------------------------------------------------
-class PerReplay:
+class Workload:
+    name = kernel = ""
+    dtype = ""
+    launches_per_round = 0
+    h2d = d2h = 0
+
+    def config(self):
+        return {"workload": self.name}
+
+    def _graph_or_eager(self, body, graph):
+        import torch
+        body()
+        torch.cuda.synchronize()
+        if not graph:
+            return body
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, capture_error_mode="thread_local"):
+            body()
+        g.replay()
+        torch.cuda.synchronize()
+        return g.replay
+
+    def time_deliver(self, n, mk, stream, graph=True):
+        """Average duration (us) of the dominant kernel launched n times back
+        to back (events bracket the launches; inputs are real batches)."""
+        import torch
+        run = self._graph_or_eager(lambda: [self.deliver_once(r) for r in range(n)],
+                                   graph)
+        e0, e1 = mk(), mk()
+        e0.record(stream)
+        run()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) * 1e3 / n
+
+    def time_latency(self, n, mk, stream):
+        """Sample -> batch latency (us) of n steps, events around each."""
+        import torch
+        evs = [(mk(), mk()) for _ in range(n)]
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, capture_error_mode="thread_local"):
+            for r in range(n):
+                evs[r][0].record()
+                self.latency_step(100000 + r, evs[r][1])
+        g.replay()
+        torch.cuda.synchronize()
+        return [a.elapsed_time(b) * 1e3 for a, b in evs]
+
+
+def _stack_bytes(B, K, F, next_obs=True):
+    """Fused frame-stack delivery: unique frame reads (K+1 per sample with
+    next_obs), fp32 writes of obs (+ next_obs), collate and IS scalars (idx
+    8, q 4 read; isw 4, action 4, reward 4, done 1 written; action 4,
+    reward 4, done K+1 read)."""
+    frames = K + 1 if next_obs else K
+    return B * (frames * F + (2 if next_obs else 1) * K * F * 4 + 33 + frames)
+
+
+class PerReplay(Workload):
+    """Prioritized replay: 1,000,000 uint8 84x84 frames (~7.06 GB), batch
+    512, frame stack 4, obs + next_obs fp32, PER alpha 0.6 / beta 0.4 with
+    priorities from Exp(1) TD errors; step = sample, deliver, update."""
     name = "per-replay-1M-84x84-B512"
     kernel = "k_deliver_stack"
-    kernel_src = "k_deliver.cu"
+    dtype = "u8->f32"
+    launches_per_round = 3
 
     def __init__(self, capacity=1_000_000, batch=512, K=4, seed=1235,
                  out_sets=4):
@@ -206,14 +272,12 @@ class PerReplay:
         while 32 ** D < capacity:
             D += 1
         self.D = D
-        F, B = self.F, batch
-        # algorithmic bytes: unique frame reads (K+1 per sample) + fp32 obs
-        # and next_obs writes + collate/IS scalars (idx 8, q 4 read; isw 4,
-        # action 4, reward 4, done 1 written; action 4, reward 4, done 5 read)
-        self.deliver_bytes = B * ((K + 1) * F + 2 * K * F * 4 + 38)
-        # sampling: one 32-child load per level + the leaf row, writes idx, q
-        self.sample_bytes = B * (32 * 8 * (D - 1) + 32 * 4 + 12)
-        # update: idx, td, leaf read+write, D ancestors read+write (8 B)
+        B = batch
+        self.deliver_bytes = _stack_bytes(B, K, self.F)
+        # sampling: one 32-child row per global level + the leaf row, writes
+        # idx and q
+        self.sample_bytes = B * (32 * 8 * max(D - 3, 0) + 32 * 4 + 12)
+        # update: idx, td, leaf read + write, D ancestors read + write (8 B)
         self.update_bytes = B * (8 + 4 + 8 + 16 * D)
         self.round_bytes = self.deliver_bytes + self.sample_bytes + self.update_bytes
 
@@ -226,9 +290,7 @@ class PerReplay:
                       % (self.cap * self.F / 1e9, self.R,
                          self.R * self.B * 2 * self.K * self.F * 4 / 1e6)}
 
-    # -- GPU arm --------------------------------------------------------------
     def setup(self, device):
-        import numpy as np
         import torch
         from paper_2609_24456_gb300 import edp
         from paper_2609_24456_gb300 import fixtures as fx
@@ -244,7 +306,6 @@ class PerReplay:
         chunk = 65536
         staging = torch.empty((chunk, self.F), dtype=torch.uint8, device=device)
         qbuf = torch.empty(chunk, dtype=torch.int32, device=device)
-        self.setup_launches = 0
         for lo in range(0, self.cap, chunk):
             hi = min(self.cap, lo + chunk)
             n = hi - lo
@@ -272,56 +333,31 @@ class PerReplay:
         self.td_rounds = 64
         self.td = torch.stack([dev(fx.td_errors(self.seed, B, r), device)
                                for r in range(self.td_rounds)])
-        self.launches_per_round = 3
 
-    def round(self, r, ev=None):
-        edp, ctx = self.edp, self.ring.ctx
+    def _sample(self, r, o):
+        self.edp.edp_sample(self.ring.ctx, self.edp.EDP_SAMPLE_PRIORITIZED, self.B,
+                            self.seed, r, o["idx"], o["q"])
+
+    def round(self, r):
         o = self.outs[r % self.R]
-        edp.edp_sample(ctx, edp.EDP_SAMPLE_PRIORITIZED, self.B, self.seed, r,
-                       o["idx"], o["q"])
-        edp.edp_deliver(ctx, o["idx"], self.B, o["batch"])
-        if ev:
-            ev[2].record()
-        edp.edp_update_priorities_td(ctx, o["idx"], self.td[r % self.td_rounds],
-                                     self.B, ALPHA, EPS)
+        self._sample(r, o)
+        self.edp.edp_deliver(self.ring.ctx, o["idx"], self.B, o["batch"])
+        self.edp.edp_update_priorities_td(self.ring.ctx, o["idx"],
+                                          self.td[r % self.td_rounds], self.B,
+                                          ALPHA, EPS)
 
-    def time_deliver(self, n, mk, stream, graph=True):
-        """Average duration (us) of the delivery kernel launched n times back
-        to back over the batches of the last rounds."""
-        import torch
-        edp, ctx = self.edp, self.ring.ctx
+    def deliver_once(self, r):
+        o = self.outs[r % self.R]
+        self.edp.edp_deliver(self.ring.ctx, o["idx"], self.B, o["batch"])
 
-        def body():
-            for r in range(n):
-                o = self.outs[r % self.R]
-                edp.edp_deliver(ctx, o["idx"], self.B, o["batch"])
-        body()
-        torch.cuda.synchronize()
-        if graph:
-            g = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(g, capture_error_mode="thread_local"):
-                body()
-            g.replay()
-            torch.cuda.synchronize()
-        e0, e1 = mk(), mk()
-        e0.record(stream)
-        g.replay() if graph else body()
-        e1.record(stream)
-        torch.cuda.synchronize()
-        return e0.elapsed_time(e1) * 1e3 / n
-
-    def time_latency(self, n, mk, stream):
-        """Sample -> batch latency (us) of n rounds, events around each."""
-        import torch
-        evs = [(mk(), mk()) for _ in range(n)]
-        g = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g, capture_error_mode="thread_local"):
-            for r in range(n):
-                evs[r][0].record()
-                self.round(100000 + r, (None, None, evs[r][1]))
-        g.replay()
-        torch.cuda.synchronize()
-        return [a.elapsed_time(b) * 1e3 for a, b in evs]
+    def latency_step(self, r, ev_end):
+        o = self.outs[r % self.R]
+        self._sample(r, o)
+        self.edp.edp_deliver(self.ring.ctx, o["idx"], self.B, o["batch"])
+        ev_end.record()
+        self.edp.edp_update_priorities_td(self.ring.ctx, o["idx"],
+                                          self.td[r % self.td_rounds], self.B,
+                                          ALPHA, EPS)
 
     def e2e_setup(self, device):
         import torch
@@ -339,23 +375,18 @@ class PerReplay:
 
     def e2e_round(self, r):
         """User path with host buffers: TD errors in, learner batch out."""
-        edp, ctx = self.edp, self.ring.ctx
         o = self.outs[r % self.R]
         self.d_td.copy_(self.h_td[r % self.td_rounds], non_blocking=True)
-        edp.edp_sample(ctx, edp.EDP_SAMPLE_PRIORITIZED, self.B, self.seed, r,
-                       o["idx"], o["q"])
-        edp.edp_deliver(ctx, o["idx"], self.B, o["batch"])
-        edp.edp_update_priorities_td(ctx, o["idx"], self.d_td, self.B, ALPHA, EPS)
+        self._sample(r, o)
+        self.edp.edp_deliver(self.ring.ctx, o["idx"], self.B, o["batch"])
+        self.edp.edp_update_priorities_td(self.ring.ctx, o["idx"], self.d_td,
+                                          self.B, ALPHA, EPS)
         h = self.h_out
-        h["obs"].copy_(o["obs"], non_blocking=True)
-        h["nxt"].copy_(o["nxt"], non_blocking=True)
-        h["act"].copy_(o["act"], non_blocking=True)
-        h["rew"].copy_(o["rew"], non_blocking=True)
-        h["done"].copy_(o["done"], non_blocking=True)
-        h["isw"].copy_(o["isw"], non_blocking=True)
-        h["idx"].copy_(o["idx"], non_blocking=True)
+        for key, src in [("obs", "obs"), ("nxt", "nxt"), ("act", "act"),
+                         ("rew", "rew"), ("done", "done"), ("isw", "isw"),
+                         ("idx", "idx")]:
+            h[key].copy_(o[src], non_blocking=True)
 
-    # -- CPU oracle arm -------------------------------------------------------
     def cpu_setup(self, host_frames=262_144):
         import numpy as np
         import oracle as orc
@@ -387,7 +418,442 @@ class PerReplay:
         orc.update_leaves(self.st, self.cap, idx, qn)
 
 
-WORKLOADS = {"per1m": PerReplay}
+class DqnTiny(Workload):
+    """Uniform replay: 10,000 uint8 84x84 frames filled past capacity,
+    batch 32, frame stack 4, obs + next_obs fp32; step = sample, deliver.
+    Launch-bound: its headline is the sample -> batch latency."""
+    name = "dqn-uniform-10k-84x84-B32"
+    kernel = "k_deliver_stack"
+    dtype = "u8->f32"
+    launches_per_round = 2
+
+    def __init__(self, capacity=10_000, batch=32, K=4, seed=1234, out_sets=32):
+        self.cap, self.B, self.K, self.seed, self.R = capacity, batch, K, seed, out_sets
+        self.F = 84 * 84
+        self.deliver_bytes = _stack_bytes(batch, K, self.F)
+        self.round_bytes = self.deliver_bytes + batch * 8
+
+    def config(self):
+        return {"workload": self.name, "capacity": self.cap, "batch": self.B,
+                "frame": "uint8 84x84", "frame_stack": self.K,
+                "l2": "ring 70 MB and outputs (%d sets, %.0f MB) rotate through L2"
+                      % (self.R, self.R * self.B * 2 * self.K * self.F * 4 / 1e6)}
+
+    def setup(self, device):
+        import torch
+        from paper_2609_24456_gb300 import edp
+        from paper_2609_24456_gb300 import fixtures as fx
+        self.edp = edp
+        cfg = edp.make_config(self.cap, (1, 84, 84), edp.EDP_XFORM_STACK_F32,
+                              frame_stack=self.K, next_obs=True,
+                              device=device.index or 0)
+        self.ring = edp.Ring(cfg, reward=True)
+        n = self.cap + 2345
+        frames, action, reward, done = fx.dqn_transitions(self.seed, n)
+        for lo in range(0, n, 4096):
+            hi = min(n, lo + 4096)
+            edp.edp_ingest(self.ring.ctx, dev(frames[lo:hi], device), hi - lo,
+                           action=dev(action[lo:hi], device),
+                           reward=dev(reward[lo:hi], device),
+                           done=dev(done[lo:hi], device))
+        edp.edp_sync(self.ring.ctx)
+        self.host = (frames, action, reward, done, n)
+        B, K, F = self.B, self.K, self.F
+        self.outs = []
+        for _ in range(self.R):
+            o = dict(idx=torch.empty(B, dtype=torch.int64, device=device),
+                     obs=torch.empty((B, K, F), device=device),
+                     nxt=torch.empty((B, K, F), device=device),
+                     act=torch.empty(B, dtype=torch.int32, device=device),
+                     rew=torch.empty(B, device=device),
+                     done=torch.empty(B, dtype=torch.uint8, device=device))
+            o["batch"] = edp.make_batch(o["obs"], o["nxt"], o["act"], o["rew"], o["done"])
+            self.outs.append(o)
+
+    def round(self, r):
+        o = self.outs[r % self.R]
+        self.edp.edp_sample(self.ring.ctx, self.edp.EDP_SAMPLE_UNIFORM, self.B,
+                            self.seed, r, o["idx"])
+        self.edp.edp_deliver(self.ring.ctx, o["idx"], self.B, o["batch"])
+
+    def deliver_once(self, r):
+        o = self.outs[r % self.R]
+        self.edp.edp_deliver(self.ring.ctx, o["idx"], self.B, o["batch"])
+
+    def latency_step(self, r, ev_end):
+        self.round(r)
+        ev_end.record()
+
+    def e2e_setup(self, device):
+        import torch
+        B, K, F = self.B, self.K, self.F
+        pin = lambda *s, dt=torch.float32: torch.empty(s, dtype=dt, pin_memory=True)
+        self.h_out = dict(obs=pin(B, K, F), nxt=pin(B, K, F),
+                          act=pin(B, dt=torch.int32), rew=pin(B),
+                          done=pin(B, dt=torch.uint8), idx=pin(B, dt=torch.int64))
+        self.h2d = 0
+        self.d2h = sum(t.numel() * t.element_size() for t in self.h_out.values())
+
+    def e2e_round(self, r):
+        self.round(r)
+        o = self.outs[r % self.R]
+        for key in ["obs", "nxt", "act", "rew", "done", "idx"]:
+            self.h_out[key].copy_(o[key], non_blocking=True)
+
+    def cpu_setup(self):
+        import numpy as np
+        import oracle as orc
+        from paper_2609_24456_gb300 import fixtures as fx
+        self.orc = orc
+        if not hasattr(self, "host"):
+            n = self.cap + 2345
+            self.host = fx.dqn_transitions(self.seed, n) + (n,)
+        frames, action, reward, done, n = self.host
+        self.h_frames = np.zeros((self.cap, self.F), np.uint8)
+        self.h_act = np.zeros(self.cap, np.int32)
+        self.h_rew = np.zeros(self.cap, np.float32)
+        self.h_done = np.zeros(self.cap, np.uint8)
+        for arr, src in [(self.h_frames, frames), (self.h_act, action),
+                         (self.h_rew, reward), (self.h_done, done)]:
+            orc.ring_write(arr, self.cap, 0, np.ascontiguousarray(src))
+        self.total = n
+        self.cpu_sample = "rounds of this workload on the full 10,000-frame host ring"
+
+    def cpu_round(self, r):
+        idx = self.orc.sample_uniform(self.cap, self.total, self.cap - 1, self.B,
+                                      self.seed, r)
+        self.orc.deliver_dqn(self.h_frames, self.h_done, self.h_act, self.h_rew,
+                             self.cap, self.total, self.K, idx)
+
+
+class PpoIteration(Workload):
+    """On-policy iteration: 256 envs x 128 steps of uint8 64x64x3 obs; GAE
+    (gamma 0.99, lambda 0.95) with global advantage normalisation, Philox
+    shuffle of 32,768 samples into 8 mini-batches of 4,096, each delivered as
+    bf16 [4096,3,64,64] with gathered advantages and returns.  Step = one
+    iteration (GAE + shuffle + 8 deliveries); the rollout ingest is timed
+    separately."""
+    name = "ppo-iteration-256x128-64x64x3"
+    kernel = "k_deliver_hwc"
+    dtype = "u8->bf16,f64"
+    T, E, H, W, C, M = 128, 256, 64, 64, 3, 8
+
+    def __init__(self, seed=1236):
+        self.seed = seed
+        self.n = self.T * self.E
+        self.mb = self.n // self.M
+        F = self.H * self.W * self.C
+        self.F = F
+        # one mini-batch delivery: obs read + bf16 write + adv/ret gathers
+        self.deliver_bytes = self.mb * (F + 2 * F + 8 + 8 + 8)
+        gae = self.T * self.E * (4 + 1 + 4) + self.E * 4 + 3 * self.T * self.E * 4
+        perm = self.n * (8 + 8 + 8 + 4 + 8 + 4 + 8) + 3 * 4 * (self.n // 4)
+        self.round_bytes = gae + perm + self.M * self.deliver_bytes
+        self.launches_per_round = 2 + self.M
+
+    def config(self):
+        return {"workload": self.name, "envs": self.E, "steps": self.T,
+                "obs": "uint8 64x64x3 HWC -> bf16 CHW", "minibatches": self.M,
+                "gamma": 0.99, "lambda": 0.95,
+                "l2": "rollout 403 MB > L2; mini-batch outputs 805 MB per iteration"}
+
+    def setup(self, device):
+        import torch
+        from paper_2609_24456_gb300 import edp
+        from paper_2609_24456_gb300 import fixtures as fx
+        self.edp = edp
+        cfg = edp.make_config(self.n, (self.C, self.H, self.W),
+                              edp.EDP_XFORM_HWC_CHW_BF16, device=device.index or 0)
+        self.ring = edp.Ring(cfg, action=False, reward=False, done=False)
+        obs, r, v, d = fx.ppo_rollout(self.seed, self.T, self.E)
+        self.h_obs, self.h_r, self.h_v, self.h_d = obs, r, v, d
+        self.d_obs = dev(obs, device)
+        self.r, self.v, self.d = dev(r, device), dev(v, device), dev(d, device)
+        edp.edp_ingest(self.ring.ctx, self.d_obs, self.n)
+        T, E = self.T, self.E
+        self.adv = torch.empty((T, E), device=device)
+        self.ret = torch.empty((T, E), device=device)
+        self.nrm = torch.empty((T, E), device=device)
+        self.idx = torch.empty(self.n, dtype=torch.int64, device=device)
+        self.out = [torch.empty((self.mb, self.C, self.H, self.W), dtype=torch.bfloat16,
+                                device=device) for _ in range(2)]
+        self.a_out = torch.empty(self.mb, device=device)
+        self.r_out = torch.empty(self.mb, device=device)
+        # first calls allocate scratch outside any capture
+        self._gae()
+        edp.edp_sample(self.ring.ctx, edp.EDP_SAMPLE_PERMUTE, self.n, self.seed, 0, self.idx)
+        edp.edp_sync(self.ring.ctx)
+
+    def _gae(self):
+        self.edp.edp_gae(self.ring.ctx, self.r, self.v, self.d, self.T, self.E,
+                         0.99, 0.95, self.adv, self.ret, self.nrm)
+
+    def _mb(self, m, r):
+        sub = self.idx[m * self.mb:(m + 1) * self.mb]
+        b = self.edp.make_batch(self.out[(r * self.M + m) % 2],
+                                gather=[(self.nrm.view(-1), self.a_out),
+                                        (self.ret.view(-1), self.r_out)])
+        self.edp.edp_deliver(self.ring.ctx, sub, self.mb, b)
+
+    def round(self, r):
+        self._gae()
+        self.edp.edp_sample(self.ring.ctx, self.edp.EDP_SAMPLE_PERMUTE, self.n,
+                            self.seed, r, self.idx)
+        for m in range(self.M):
+            self._mb(m, r)
+
+    def deliver_once(self, r):
+        self._mb(r % self.M, r)
+
+    def latency_step(self, r, ev_end):
+        self._gae()
+        self.edp.edp_sample(self.ring.ctx, self.edp.EDP_SAMPLE_PERMUTE, self.n,
+                            self.seed, r, self.idx)
+        self._mb(0, r)
+        ev_end.record()
+
+    def e2e_setup(self, device):
+        import torch
+        pin = lambda t: torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
+        self.h_in = [pin(t) for t in (self.r, self.v, self.d)]
+        for h, t in zip(self.h_in, (self.r, self.v, self.d)):
+            h.copy_(t.cpu())
+        self.h_outs = [pin(self.out[0]) for _ in range(self.M)]
+        self.h_ao = [pin(self.a_out) for _ in range(self.M)]
+        self.h_ro = [pin(self.r_out) for _ in range(self.M)]
+        self.h2d = sum(t.numel() * t.element_size() for t in self.h_in)
+        self.d2h = self.M * (self.h_outs[0].numel() * 2 + 8 * self.mb)
+
+    def e2e_round(self, r):
+        for h, t in zip(self.h_in, (self.r, self.v, self.d)):
+            t.copy_(h, non_blocking=True)
+        self._gae()
+        self.edp.edp_sample(self.ring.ctx, self.edp.EDP_SAMPLE_PERMUTE, self.n,
+                            self.seed, r, self.idx)
+        for m in range(self.M):
+            self._mb(m, r)
+            self.h_outs[m].copy_(self.out[(r * self.M + m) % 2], non_blocking=True)
+            self.h_ao[m].copy_(self.a_out, non_blocking=True)
+            self.h_ro[m].copy_(self.r_out, non_blocking=True)
+
+    def cpu_setup(self):
+        import oracle as orc
+        from paper_2609_24456_gb300 import fixtures as fx
+        self.orc = orc
+        if not hasattr(self, "h_obs"):
+            self.h_obs, self.h_r, self.h_v, self.h_d = fx.ppo_rollout(
+                self.seed, self.T, self.E)
+        self.cpu_sample = "whole iterations of this workload (GAE direct sums, shuffle, 8 mini-batches)"
+
+    def cpu_round(self, r):
+        import numpy as np
+        orc = self.orc
+        adv, ret = orc.gae(self.h_r, self.h_v, self.h_d, 0.99, 0.95)
+        nrm, _, _ = orc.normalize(adv.ravel())
+        perm = orc.permutation(self.n, self.seed, r)
+        nrm32, ret32 = nrm.astype(np.float32), ret.ravel().astype(np.float32)
+        for m in range(self.M):
+            orc.deliver_ppo(self.h_obs, self.n, self.n, self.H, self.W, self.C,
+                            perm[m * self.mb:(m + 1) * self.mb], nrm32, ret32)
+
+
+MEAN3, STD3 = (0.485, 0.456, 0.406), (0.229, 0.224, 0.225)
+
+
+class MmReplay(Workload):
+    """Multimodal replay: 200,000 transitions of uint8 3x224x224 images
+    (~30.1 GB) + 512 int32 tokens + reward, uniform batch 1,024 delivered as
+    per-channel normalised bf16 with collated tokens and rewards; step =
+    sample, deliver.  With hbm_frac < 1 the oldest part of the ring lives in
+    page-locked host memory (two-tier placement) and each step also ingests
+    4,096 new transitions from page-locked staging, demoting the oldest HBM
+    entries."""
+    kernel = "k_deliver_norm"
+    dtype = "u8->bf16"
+    C, H, W, L = 3, 224, 224, 512
+
+    def __init__(self, capacity=200_000, batch=1024, seed=1237, hbm_frac=1.0,
+                 ingest=0):
+        self.cap, self.B, self.seed = capacity, batch, seed
+        self.cap_h = int(capacity * hbm_frac)
+        self.ingest = ingest
+        self.F = self.C * self.H * self.W
+        self.tiered = self.cap_h < self.cap
+        self.name = ("mm-tiered-%dk-%dk-host-B%d" % (self.cap // 1000,
+                                                    (self.cap - self.cap_h) // 1000, batch)
+                     if self.tiered else "mm-replay-%dk-3x224x224-B%d" % (capacity // 1000, batch))
+        per = self.F + 4 * self.L + 4  # bytes read per sample
+        self.deliver_bytes = batch * (per + 2 * self.F + 4 * self.L + 4 + 8)
+        rec = self.F + 4 * self.L + 4
+        self.ingest_bytes = ingest * (2 * rec + 4)  # staging read + HBM write
+        self.demote_bytes = ingest * 2 * (self.F + 4 * self.L)
+        self.round_bytes = self.deliver_bytes + batch * 8 + self.ingest_bytes + \
+            (self.demote_bytes if self.tiered else 0)
+        self.launches_per_round = 2 + (5 if ingest else 0)
+
+    def config(self):
+        c = {"workload": self.name, "capacity": self.cap, "batch": self.B,
+             "obs": "uint8 3x224x224 CHW -> bf16 normalised", "tokens": self.L,
+             "resident_hbm_GB": round(self.cap_h * (self.F + 4 * self.L) / 1e9, 1)}
+        if self.tiered:
+            c.update({"host_tier": self.cap - self.cap_h, "ingest_per_step": self.ingest,
+                      "host_GB": round((self.cap - self.cap_h) * (self.F + 4 * self.L) / 1e9, 1)})
+        return c
+
+    def setup(self, device):
+        import torch
+        from paper_2609_24456_gb300 import edp
+        from paper_2609_24456_gb300 import fixtures as fx
+        self.edp = edp
+        cfg = edp.make_config(self.cap, (self.C, self.H, self.W),
+                              edp.EDP_XFORM_CHW_NORM_BF16, hbm_capacity=self.cap_h,
+                              tokens=self.L, norm_mean=MEAN3, norm_std=STD3,
+                              device=device.index or 0)
+        self.ring = edp.Ring(cfg, action=False, done=False)
+        _, rew = fx.mm_metadata(self.seed, self.cap + max(self.ingest, 1) * 64, tokens=0)
+        self.rew_all = rew
+        chunk = 4096
+        obs = torch.empty((chunk, self.F), dtype=torch.uint8, device=device)
+        tok = torch.empty((chunk, self.L), dtype=torch.int32, device=device)
+        for lo in range(0, self.cap, chunk):
+            n = min(chunk, self.cap - lo)
+            fx.content_fill_torch(self.seed, lo, obs[:n])
+            fx.token_fill_torch(self.seed, lo, tok[:n])
+            edp.edp_ingest(self.ring.ctx, obs[:n], n, tokens=tok[:n],
+                           reward=dev(rew[lo:lo + n], device))
+        edp.edp_sync(self.ring.ctx)
+        self.total0 = self.cap
+        if self.ingest:
+            # page-locked staging of new transitions (actors on the host)
+            n = self.ingest
+            self.st_obs = torch.empty((n, self.F), dtype=torch.uint8, pin_memory=True)
+            self.st_tok = torch.empty((n, self.L), dtype=torch.int32, pin_memory=True)
+            fx.content_fill_torch(self.seed, self.cap, obs[:n])
+            fx.token_fill_torch(self.seed, self.cap, tok[:n])
+            self.st_obs.copy_(obs[:n])
+            self.st_tok.copy_(tok[:n])
+            self.st_rew = torch.from_numpy(rew[:n].copy()).pin_memory()
+        del obs, tok
+        B = self.B
+        self.outs = []
+        for _ in range(2):
+            o = dict(idx=torch.empty(B, dtype=torch.int64, device=device),
+                     obs=torch.empty((B, self.C, self.H, self.W), dtype=torch.bfloat16,
+                                     device=device),
+                     tok=torch.empty((B, self.L), dtype=torch.int32, device=device),
+                     rew=torch.empty(B, device=device))
+            o["batch"] = edp.make_batch(o["obs"], tokens=o["tok"], reward=o["rew"])
+            self.outs.append(o)
+
+    def round(self, r):
+        ctx = self.ring.ctx
+        if self.ingest:
+            self.edp.edp_ingest(ctx, self.st_obs, self.ingest, tokens=self.st_tok,
+                                reward=self.st_rew)
+        o = self.outs[r % 2]
+        self.edp.edp_sample(ctx, self.edp.EDP_SAMPLE_UNIFORM, self.B, self.seed, r, o["idx"])
+        self.edp.edp_deliver(ctx, o["idx"], self.B, o["batch"])
+
+    def deliver_once(self, r):
+        o = self.outs[r % 2]
+        self.edp.edp_deliver(self.ring.ctx, o["idx"], self.B, o["batch"])
+
+    def latency_step(self, r, ev_end):
+        o = self.outs[r % 2]
+        self.edp.edp_sample(self.ring.ctx, self.edp.EDP_SAMPLE_UNIFORM, self.B,
+                            self.seed, r, o["idx"])
+        self.edp.edp_deliver(self.ring.ctx, o["idx"], self.B, o["batch"])
+        ev_end.record()
+
+    def e2e_setup(self, device):
+        import torch
+        o = self.outs[0]
+        self.h_out = {k: torch.empty(o[k].shape, dtype=o[k].dtype, pin_memory=True)
+                      for k in ("obs", "tok", "rew", "idx")}
+        self.h2d = 0 if not self.ingest else self.ingest * (self.F + 4 * self.L + 4)
+        self.d2h = sum(t.numel() * t.element_size() for t in self.h_out.values())
+
+    def e2e_round(self, r):
+        self.round(r)
+        o = self.outs[r % 2]
+        for k in ("obs", "tok", "rew", "idx"):
+            self.h_out[k].copy_(o[k], non_blocking=True)
+
+    def extra(self, device, mk, stream, deliver_us):
+        """Two-tier only: host-link bandwidth measured in this run (zero-copy
+        read kernel and a pinned H2D copy) and the host-tier share of the
+        delivery's reads against it."""
+        if not self.tiered:
+            return {}
+        import torch
+        from paper_2609_24456_gb300 import edp
+        nbytes = 4 << 30
+        h = torch.empty(nbytes, dtype=torch.uint8, pin_memory=True)
+        h.fill_(3)
+        d = torch.empty(nbytes, dtype=torch.uint8, device=device)
+        fold = torch.zeros(1, dtype=torch.int64, device=device)
+        best_probe = best_copy = 0.0
+        for _ in range(3):
+            e0, e1 = mk(), mk()
+            e0.record(stream)
+            edp.edp_probe_host_read(h, nbytes, fold)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            best_probe = max(best_probe, nbytes / (e0.elapsed_time(e1) / 1e3) / 1e9)
+            e0.record(stream)
+            d.copy_(h, non_blocking=True)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            best_copy = max(best_copy, nbytes / (e0.elapsed_time(e1) / 1e3) / 1e9)
+        del h, d
+        link = max(best_probe, best_copy)
+        host_frac = (self.cap - self.cap_h) / self.cap
+        host_bytes = self.B * host_frac * (self.F + 4 * self.L)
+        achieved = host_bytes / (deliver_us / 1e6) / 1e9
+        return {"host_link": {"probe_read_GBs": best_probe, "h2d_copy_GBs": best_copy,
+                              "delivery_host_read_GBs": achieved,
+                              "frac_of_link": achieved / link,
+                              "host_bytes_per_delivery": host_bytes}}
+
+    def cpu_setup(self, host_rows=16384):
+        import numpy as np
+        import oracle as orc
+        from paper_2609_24456_gb300 import fixtures as fx
+        self.orc = orc
+        self.hrows = min(host_rows, self.cap)
+        rng = np.random.default_rng(self.seed)
+        self.h_obs = rng.integers(0, 256, size=(self.hrows, self.F), dtype=np.uint8)
+        self.h_tok, self.h_rew = fx.mm_metadata(self.seed, self.hrows, tokens=self.L)
+        if self.ingest:
+            self.h_stage = rng.integers(0, 256, size=(self.ingest, self.F), dtype=np.uint8)
+            self.h_demoted = np.empty_like(self.h_stage)
+        self.cpu_sample = ("per-step work of this workload (uniform B=%d, normalised bf16 "
+                           "images, tokens, rewards%s) reading a %d-transition host ring "
+                           "(%.1f GB)" % (self.B, ", ingest + demotion of %d" % self.ingest
+                                          if self.ingest else "", self.hrows,
+                                          self.hrows * self.F / 1e9))
+
+    def cpu_round(self, r):
+        orc = self.orc
+        if self.ingest:  # demote the oldest rows, then write the new ones
+            rows = (r * self.ingest + np.arange(self.ingest)) % self.hrows
+            self.h_demoted[:] = self.h_obs[rows]
+            self.h_obs[rows] = self.h_stage
+        idx = orc.sample_uniform(self.cap, self.cap, self.cap, self.B, self.seed, r)
+        orc.deliver_mm(self.h_obs, self.h_tok, self.h_rew, self.C, self.H * self.W,
+                       idx % self.hrows, MEAN3, STD3)
+
+
+WORKLOADS = {
+    "per1m": PerReplay,
+    "dqn10k": DqnTiny,
+    "ppo": PpoIteration,
+    "mm200k": MmReplay,
+    # two-tier: 800,000 transitions (the 1.6M of the full configuration scaled
+    # to the GPU box's host memory), newest half in HBM, 4,096 ingested per step
+    "tiered": lambda **kw: MmReplay(capacity=kw.get("capacity") or 800_000,
+                                    hbm_frac=0.5, ingest=4096),
+}
 
 
 # ----------------------------------------------------------------------------
@@ -419,7 +885,7 @@ def run_reference(args):
             "impl": "reference", "n_gpus": args.gpus, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": dt * 1e3 / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-            "dtype": "u8->f32", "data": "synthetic", "config": wl.config(),
+            "dtype": wl.dtype, "data": "synthetic", "config": wl.config(),
             "cpu_baseline": {"value": gbs, "unit": "GB/s", "cores": cores,
                              "kind": "oracle", "sample": wl.cpu_sample},
             "e2e": {"value": gbs, "unit": "GB/s", "h2d_bytes_per_step": 0,
@@ -443,6 +909,8 @@ def run_edp(args):
     build.build()
 
     wl = WORKLOADS[args.workload](**({"capacity": args.capacity} if args.capacity else {}))
+    if args.workload == "ppo" and args.capacity:
+        raise SystemExit("--capacity does not apply to the ppo workload")
     wl.setup(device)
     K, W = args.steps, args.warmup
     mk = lambda: torch.cuda.Event(enable_timing=True, external=True)
@@ -530,6 +998,7 @@ def run_edp(args):
                 "algorithmic_bytes_per_launch": wl.deliver_bytes,
                 "avg_launch_us": avg_deliver_s * 1e6, "launches_timed": Kd}
 
+    extra = wl.extra(device, mk, stream, deliver_us) if hasattr(wl, "extra") else {}
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         wl.cpu_setup()
@@ -542,7 +1011,7 @@ def run_edp(args):
         line = {"metric": "experience-delivery GB/s", "value": value,
                 "unit": "GB/s", "n_gpus": world, "steps": K, "warmup": W,
                 "ms_per_step": ms_step, "higher_is_better": True,
-                "scaling": "weak", "vs_baseline": None, "dtype": "u8->f32",
+                "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype,
                 "data": "synthetic", "config": dict(wl.config(),
                                                     parallelism="replicas%d" % world,
                                                     graph=use_graph),
@@ -552,6 +1021,7 @@ def run_edp(args):
                 "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
                 "gpu_launches": wl.launches_per_round * K,
                 "clocks": clk}
+        line.update(extra)
         print(json.dumps(line))
     if dist:
         dist.barrier()

@@ -88,7 +88,9 @@ void free_all(edp_ctx *c) {
   if (c->ctrl) fr(c->cfg.alloc_user, c->ctrl);
   if (c->scratch) fr(c->cfg.alloc_user, c->scratch);
   if (c->qbuf) fr(c->cfg.alloc_user, c->qbuf);
+  if (c->perm_scratch) fr(c->cfg.alloc_user, c->perm_scratch);
   c->qbuf = nullptr;
+  c->perm_scratch = nullptr;
   c->tree_mem = nullptr;
   c->ctrl = nullptr;
   c->scratch = nullptr;
@@ -144,6 +146,29 @@ void *edp::ctx_scratch(edp_ctx *ctx, size_t bytes) {
   if (!p) return nullptr;
   ctx->scratch = p;
   ctx->scratch_bytes = bytes;
+  return p;
+}
+
+void *edp::ctx_perm_scratch(edp_ctx *ctx, size_t bytes) {
+  if (bytes <= ctx->perm_bytes) return ctx->perm_scratch;
+  edp_alloc_fn al = ctx->cfg.alloc ? ctx->cfg.alloc : default_alloc;
+  edp_free_fn fr = ctx->cfg.free ? ctx->cfg.free : default_free;
+  if (ctx->perm_scratch) {
+    cudaDeviceSynchronize();
+    fr(ctx->cfg.alloc_user, ctx->perm_scratch);
+    ctx->perm_scratch = nullptr;
+    ctx->perm_bytes = 0;
+  }
+  bytes = (bytes + 255) & ~(size_t)255;
+  void *p = al(ctx->cfg.alloc_user, bytes);
+  if (!p) return nullptr;
+  if (cudaMemset(p, 0, perm_zeroed_bytes()) != cudaSuccess) {
+    cudaGetLastError();
+    fr(ctx->cfg.alloc_user, p);
+    return nullptr;
+  }
+  ctx->perm_scratch = p;
+  ctx->perm_bytes = bytes;
   return p;
 }
 
@@ -473,6 +498,8 @@ edp_status edp_sample(edp_ctx *ctx, edp_sample_mode mode, uint32_t batch,
     default:
       return fail(ctx, EDP_ERR_INVALID, "edp_sample: unknown mode %d", (int)mode);
   }
+  if (e == cudaErrorMemoryAllocation)
+    return fail(ctx, EDP_ERR_OOM, "edp_sample: scratch allocation failed");
   if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_sample");
   return EDP_OK;
 }

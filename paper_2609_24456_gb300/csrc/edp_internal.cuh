@@ -17,7 +17,7 @@ namespace edp {
 enum : uint32_t {
   DEVERR_INDEX = 1u,    // a slot index outside the sampleable range
   DEVERR_EMPTY = 2u,    // total priority 0 at sampling time
-  DEVERR_TIMEOUT = 4u,  // a bounded wait (grid barrier, bulk copy) expired
+  DEVERR_TIMEOUT = 4u,  // a bounded wait (bulk-copy barrier) expired
   DEVERR_TREE = 8u,     // a tree descent found no child holding its target
 };
 
@@ -26,8 +26,7 @@ struct Ctrl {
   uint32_t err;
   uint32_t pending_q;  // deferred priority of the newest transition
   uint32_t max_q;      // running maximum priority
-  uint32_t bar_count;  // grid barrier: arrivals
-  uint32_t bar_gen;    // grid barrier: generation
+  uint32_t pad0[2];
   uint32_t upd_count;  // priority update: CTAs done with phase 1
   uint32_t pad[2];
   unsigned long long bad_index;  // first offending index (diagnostics)
@@ -55,6 +54,8 @@ struct edp_ctx {
   // lazily grown scratch (shuffle, GAE partials)
   void *scratch = nullptr;
   size_t scratch_bytes = 0;
+  void *perm_scratch = nullptr;
+  size_t perm_bytes = 0;
   // priorities computed from TD errors before they are applied
   uint32_t *qbuf = nullptr;
   size_t qbuf_n = 0;
@@ -329,41 +330,13 @@ __device__ __forceinline__ void flag(Ctrl *c, uint32_t bits,
     atomicCAS(&c->bad_index, 0ull, detail + 1);
 }
 
-// Grid-wide barrier for cooperative launches (all CTAs co-resident by
-// construction).  The wait is bounded: after ~`budget` clock cycles the CTA
-// records DEVERR_TIMEOUT and proceeds, so a fault can never hang the GPU.
-__device__ __forceinline__ void grid_barrier(Ctrl *c, unsigned nblocks) {
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    volatile uint32_t *gen = &c->bar_gen;
-    const uint32_t g = *gen;
-    __threadfence();
-    const uint32_t arrived = atomicAdd(&c->bar_count, 1u) + 1u;
-    if (arrived == nblocks) {
-      c->bar_count = 0;
-      __threadfence();
-      atomicAdd(&c->bar_gen, 1u);
-    } else {
-      const long long t0 = clock64();
-      while (*gen == g) {
-        __nanosleep(64);
-        if (clock64() - t0 > 4000000000ll) {  // ~2 s at 2 GHz
-          atomicOr(&c->err, DEVERR_TIMEOUT);
-          break;
-        }
-      }
-    }
-    __threadfence();
-  }
-  __syncthreads();
-}
-
 // Programmatic dependent launch (sm_90+): a kernel launched with
 // launch_pdl may be scheduled while its predecessor in the stream is still
 // running; pdl_wait() blocks until the predecessor has completed and its
-// writes are visible, so every such kernel calls it before touching memory.
-// pdl_launch() lets the next kernel in the stream start launching.  Both are
-// no-ops for a kernel launched without the attribute.
+// writes are visible, so every such kernel calls it before touching memory
+// the predecessor may write.  pdl_launch() lets the next kernel in the
+// stream start launching.  Both are no-ops for a kernel launched without
+// the attribute.
 __device__ __forceinline__ void pdl_wait() {
   asm volatile("griddepcontrol.wait;" ::: "memory");
 }
@@ -430,6 +403,11 @@ cudaError_t launch_probe_read(const void *src, uint64_t bytes, uint64_t *fold,
 // scratch owned by the context, grown on demand (not stream-ordered: the
 // caller makes the first call of a given size outside graph capture)
 void *ctx_scratch(edp_ctx *ctx, size_t bytes);
+// shuffle scratch: its first perm_zeroed_bytes() start zeroed and are left
+// zeroed by every shuffle
+void *ctx_perm_scratch(edp_ctx *ctx, size_t bytes);
+size_t perm_scratch_bytes(uint32_t n);
+size_t perm_zeroed_bytes();
 uint32_t *ctx_qbuf(edp_ctx *ctx, size_t n);
 
 }  // namespace edp

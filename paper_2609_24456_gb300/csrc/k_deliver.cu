@@ -69,6 +69,25 @@ __device__ __forceinline__ bool sample_slot(const Common &c, uint32_t k,
   return true;
 }
 
+// Minimum of q over the batch (one warp): loads are issued 8 per lane at a
+// time so a batch of 512 costs two memory round trips, not sixteen.
+__device__ __forceinline__ uint32_t batch_qmin(const Common &c, int lane) {
+  uint32_t m = 0xffffffffu;
+  for (uint32_t i0 = lane; i0 < c.B; i0 += 32 * 8) {
+    uint32_t v[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const uint32_t i = i0 + u * 32;
+      v[u] = i < c.B ? __ldg(c.q + i) : 0xffffffffu;
+    }
+#pragma unroll
+    for (int u = 0; u < 8; ++u) m = min(m, v[u]);
+  }
+#pragma unroll
+  for (int o = 16; o; o >>= 1) m = min(m, __shfl_xor_sync(kFull, m, o));
+  return m;
+}
+
 // Per-sample collate, importance weight and scalar gathers (one warp).  The
 // head warp of each sample runs this before its payload span, so the fp64
 // chain of the weight overlaps the other warps' streaming.
@@ -83,10 +102,7 @@ __device__ void collate(const Common &c, uint32_t k, bool ok, uint64_t slot,
   }
   if (c.isw) {
     // PER: w = (q_min / q_k)^beta, q_min over the batch; fp64, one rounding
-    uint32_t m = 0xffffffffu;
-    for (uint32_t i = lane; i < c.B; i += 32) m = min(m, c.q[i]);
-#pragma unroll
-    for (int o = 16; o; o >>= 1) m = min(m, __shfl_xor_sync(kFull, m, o));
+    const uint32_t m = batch_qmin(c, lane);
     if (lane == 0) {
       const uint32_t qk = c.q[k];
       float w = 0.f;

@@ -11,12 +11,21 @@
 // scan composes lanes (5 levels), and each lane then replays its own steps
 // from the value handed over by its right neighbour.  Chunks of 32*J steps
 // are processed from the end of the rollout backwards, carrying A across.
-// All arithmetic is fp64; outputs are rounded once to fp32.
 //
-// One cooperative launch: phase 1 computes A and returns and per-CTA fp64
-// sums of A and A^2; a bounded grid barrier; phase 2 forms mean and the
-// unbiased standard deviation (every CTA reduces the partials in the same
-// fixed order, so all agree bit for bit) and writes the normalised values.
+// Arithmetic: GB300's fp64 pipe is narrow (a dependent fp64 FMA costs ~64
+// cycles, fp32 ~4), so the scan runs in double-float arithmetic -- a value
+// is an unevaluated pair hi + lo of fp32 numbers, combined with the
+// error-free transformations TwoSum (Knuth) and TwoProd via FMA (Dekker),
+// as in the double-double arithmetic of Hida, Li and Bailey -- which keeps
+// ~44 significant bits (relative error ~2^-44 per operation); gamma and
+// gamma*lambda enter as pairs split from fp64.  Only the mean / variance
+// reduction and the normalisation use fp64.  Outputs are rounded to fp32.
+//
+// Two kernels chained with programmatic dependent launch: the scan writes A,
+// the returns and per-CTA fp64 sums of A and A^2; the normalisation kernel
+// forms mean and the unbiased standard deviation (every CTA reduces the
+// partials in the same fixed order, so all agree bit for bit) and writes
+// the normalised values, one thread per element.
 #include "edp_internal.cuh"
 
 namespace edp {
@@ -26,71 +35,128 @@ constexpr unsigned kFull = 0xffffffffu;
 constexpr int kJ = 4;          // steps per lane per chunk
 constexpr int kGaeWarps = 4;   // environments per CTA
 constexpr int kGaeThreads = kGaeWarps * 32;
+constexpr int kNormThreads = 256;
+
+// ---- double-float arithmetic (every operation one IEEE rounding: the
+// intrinsics are never contracted or reassociated by the compiler)
+struct df {
+  float hi, lo;
+};
+__device__ __forceinline__ df two_sum(float a, float b) {
+  const float s = __fadd_rn(a, b);
+  const float bb = __fsub_rn(s, a);
+  const float e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
+  return {s, e};
+}
+__device__ __forceinline__ df quick_two_sum(float a, float b) {  // |a| >= |b|
+  const float s = __fadd_rn(a, b);
+  return {s, __fsub_rn(b, __fsub_rn(s, a))};
+}
+__device__ __forceinline__ df df_add(df a, df b) {
+  df s = two_sum(a.hi, b.hi);
+  const df t = two_sum(a.lo, b.lo);
+  s.lo = __fadd_rn(s.lo, t.hi);
+  s = quick_two_sum(s.hi, s.lo);
+  s.lo = __fadd_rn(s.lo, t.lo);
+  return quick_two_sum(s.hi, s.lo);
+}
+__device__ __forceinline__ df df_add_f(df a, float b) {
+  df s = two_sum(a.hi, b);
+  s.lo = __fadd_rn(s.lo, a.lo);
+  return quick_two_sum(s.hi, s.lo);
+}
+__device__ __forceinline__ df df_mul(df a, df b) {
+  const float p = __fmul_rn(a.hi, b.hi);
+  float e = __fmaf_rn(a.hi, b.hi, -p);
+  e = __fmaf_rn(a.hi, b.lo, e);
+  e = __fmaf_rn(a.lo, b.hi, e);
+  return quick_two_sum(p, e);
+}
+__device__ __forceinline__ df df_mul_f(df a, float b) {
+  const float p = __fmul_rn(a.hi, b);
+  float e = __fmaf_rn(a.hi, b, -p);
+  e = __fmaf_rn(a.lo, b, e);
+  return quick_two_sum(p, e);
+}
+__device__ __forceinline__ df df_shfl_down(df a, int o) {
+  return {__shfl_down_sync(kFull, a.hi, o), __shfl_down_sync(kFull, a.lo, o)};
+}
+__device__ __forceinline__ df df_split(double x) {
+  const float hi = (float)x;
+  return {hi, (float)(x - (double)hi)};
+}
+__device__ __forceinline__ double df_to_d(df a) {
+  return (double)a.hi + (double)a.lo;
+}
 
 __global__ void __launch_bounds__(kGaeThreads)
-k_gae(const float *__restrict__ r, const float *__restrict__ v,
-      const uint8_t *__restrict__ d, uint32_t T, uint32_t E, double gamma,
-      double lambda, float *__restrict__ adv, float *__restrict__ ret,
-      float *__restrict__ adv_norm, double *__restrict__ partial, Ctrl *ctrl) {
+k_gae_scan(const float *__restrict__ r, const float *__restrict__ v,
+           const uint8_t *__restrict__ d, uint32_t T, uint32_t E, double gamma,
+           double lambda, float *__restrict__ A_out, float *__restrict__ ret,
+           double *__restrict__ partial) {
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-  const double gl = gamma * lambda;
-  // where A is kept between the phases (fp32; the normalisation error this
-  // adds is below 2^-24 |A| / std)
-  float *A_out = adv ? adv : adv_norm;
+  pdl_wait();
+  const df g = df_split(gamma);
+  const df gl = df_split(gamma * lambda);
+  const df one = {1.f, 0.f}, zero = {0.f, 0.f};
   double s1 = 0.0, s2 = 0.0;
   for (uint32_t e = blockIdx.x * kGaeWarps + wid; e < E; e += gridDim.x * kGaeWarps) {
-    double carry = 0.0;  // A at the step after the current chunk
+    df carry = zero;  // A at the step after the current chunk
     for (int64_t te = T; te > 0; te -= 32 * kJ) {
       const int64_t ts = te - 32 * kJ > 0 ? te - 32 * kJ : 0;
-      double del[kJ], cc[kJ];
-      double a = 1.0, b = 0.0;  // this lane's steps composed
+      df del[kJ], cc[kJ];
+      df a = one, b = zero;  // this lane's steps composed: x -> b + a x
 #pragma unroll
       for (int i = kJ - 1; i >= 0; --i) {
         const int64_t t = ts + (int64_t)lane * kJ + i;
         if (t < te) {
           const uint64_t at = (uint64_t)t * E + e;
-          const double nd = d[at] ? 0.0 : 1.0;
-          del[i] = (double)r[at] + gamma * (double)v[at + E] * nd - (double)v[at];
-          cc[i] = gl * nd;
-          b = del[i] + cc[i] * b;
-          a = cc[i] * a;
+          const bool dn = d[at] != 0;
+          // delta = r + gamma V' (1 - d) - V
+          df x = dn ? df{r[at], 0.f} : df_add_f(df_mul_f(g, v[at + E]), r[at]);
+          del[i] = df_add_f(x, -v[at]);
+          cc[i] = dn ? zero : gl;
+          b = df_add(del[i], df_mul(cc[i], b));
+          a = df_mul(cc[i], a);
         } else {
-          del[i] = 0.0;
-          cc[i] = 1.0;
+          del[i] = zero;
+          cc[i] = one;
         }
       }
       // inclusive suffix scan: lane l gets lanes l..31 composed
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
-        const double a2 = __shfl_down_sync(kFull, a, o);
-        const double b2 = __shfl_down_sync(kFull, b, o);
+        const df a2 = df_shfl_down(a, o);
+        const df b2 = df_shfl_down(b, o);
         if (lane + o < 32) {
-          b = b + a * b2;
-          a = a * a2;
+          b = df_add(b, df_mul(a, b2));
+          a = df_mul(a, a2);
         }
       }
-      const double an = __shfl_down_sync(kFull, a, 1);
-      const double bn = __shfl_down_sync(kFull, b, 1);
-      double A = lane < 31 ? bn + an * carry : carry;  // A after my steps
+      const df an = df_shfl_down(a, 1);
+      const df bn = df_shfl_down(b, 1);
+      df A = lane < 31 ? df_add(bn, df_mul(an, carry)) : carry;  // A after my steps
 #pragma unroll
       for (int i = kJ - 1; i >= 0; --i) {
         const int64_t t = ts + (int64_t)lane * kJ + i;
         if (t < te) {
-          A = del[i] + cc[i] * A;
+          A = df_add(del[i], df_mul(cc[i], A));
           const uint64_t at = (uint64_t)t * E + e;
-          if (A_out) A_out[at] = (float)A;
-          if (ret) ret[at] = (float)(A + (double)v[at]);
-          s1 += A;
-          s2 += A * A;
+          if (A_out) A_out[at] = A.hi;
+          if (ret) ret[at] = df_add_f(A, v[at]).hi;
+          const double Ad = df_to_d(A);
+          s1 += Ad;
+          s2 = fma(Ad, Ad, s2);
         }
       }
-      carry = __shfl_sync(kFull, b + a * carry, 0);
+      const df c0 = df_add(b, df_mul(a, carry));
+      carry = {__shfl_sync(kFull, c0.hi, 0), __shfl_sync(kFull, c0.lo, 0)};
     }
   }
-  if (!adv_norm) return;  // no normalisation requested: no barrier needed
+  pdl_launch();
+  if (!partial) return;  // no normalisation requested
   // per-CTA partial sums (fixed order: warps, then lanes by xor tree)
   __shared__ double ws1[kGaeWarps], ws2[kGaeWarps];
-  __shared__ double stat[2];
 #pragma unroll
   for (int o = 16; o; o >>= 1) {
     s1 += __shfl_xor_sync(kFull, s1, o);
@@ -110,27 +176,46 @@ k_gae(const float *__restrict__ r, const float *__restrict__ v,
     partial[2 * blockIdx.x] = t1;
     partial[2 * blockIdx.x + 1] = t2;
   }
-  grid_barrier(ctrl, gridDim.x);
-  if (threadIdx.x == 0) {
-    double t1 = 0.0, t2 = 0.0;
-    for (unsigned bI = 0; bI < gridDim.x; ++bI) {
-      t1 += *((volatile double *)&partial[2 * bI]);
-      t2 += *((volatile double *)&partial[2 * bI + 1]);
+}
+
+// Normalisation: every CTA reduces the per-CTA partials of the scan in the
+// same fixed order, then one thread per element writes (A - mean) * inv_std.
+// A is read from A_src (the caller's adv, or adv_norm itself).
+__global__ void __launch_bounds__(kNormThreads)
+k_gae_norm(const float *A_src, float *adv_norm, uint64_t n, const double *partial,
+           uint32_t nparts) {
+  __shared__ double r1[kNormThreads], r2[kNormThreads];
+  __shared__ double stat[2];
+  pdl_wait();
+  pdl_launch();
+  double t1 = 0.0, t2 = 0.0;
+  for (unsigned i = threadIdx.x; i < nparts; i += kNormThreads) {
+    t1 += __ldcg(&partial[2 * i]);
+    t2 += __ldcg(&partial[2 * i + 1]);
+  }
+  r1[threadIdx.x] = t1;
+  r2[threadIdx.x] = t2;
+  __syncthreads();
+  for (int w = kNormThreads / 2; w > 0; w >>= 1) {
+    if ((int)threadIdx.x < w) {
+      r1[threadIdx.x] += r1[threadIdx.x + w];
+      r2[threadIdx.x] += r2[threadIdx.x + w];
     }
-    const double n = (double)T * (double)E;
-    const double mean = t1 / n;
-    double var = (t2 - t1 * mean) / (n - 1.0);
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) {
+    const double nn = (double)n;
+    const double mean = r1[0] / nn;
+    double var = (r2[0] - r1[0] * mean) / (nn - 1.0);
     if (var < 0.0) var = 0.0;
     stat[0] = mean;
     stat[1] = 1.0 / (sqrt(var) + 1e-8);
   }
   __syncthreads();
   const double mean = stat[0], inv = stat[1];
-  for (uint32_t e = blockIdx.x * kGaeWarps + wid; e < E; e += gridDim.x * kGaeWarps)
-    for (uint32_t t = lane; t < T; t += 32) {
-      const uint64_t at = (uint64_t)t * E + e;
-      adv_norm[at] = (float)(((double)A_out[at] - mean) * inv);
-    }
+  for (uint64_t i = blockIdx.x * (uint64_t)kNormThreads + threadIdx.x; i < n;
+       i += (uint64_t)gridDim.x * kNormThreads)
+    adv_norm[i] = (float)(((double)__ldcg(&A_src[i]) - mean) * inv);
 }
 
 }  // namespace
@@ -139,19 +224,24 @@ cudaError_t launch_gae(edp_ctx *c, const float *r, const float *v,
                        const uint8_t *d, uint32_t T, uint32_t E, double gamma,
                        double lambda, float *adv, float *ret, float *adv_norm,
                        cudaStream_t s) {
-  int per_sm = 0;
-  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_gae, kGaeThreads, 0);
-  uint64_t grid = (E + kGaeWarps - 1) / kGaeWarps;
-  const uint64_t cap = (uint64_t)per_sm * c->coop_sms;
-  if (grid > cap) grid = cap;
-  if (grid == 0) grid = 1;
-  double *partial = (double *)ctx_scratch(c, grid * 2 * sizeof(double));
-  if (!partial) return cudaErrorMemoryAllocation;
-  unsigned g = (unsigned)grid;
-  void *args[] = {(void *)&r, (void *)&v, (void *)&d, &T, &E, &gamma, &lambda,
-                  &adv, &ret, &adv_norm, &partial, &c->ctrl};
-  return cudaLaunchCooperativeKernel((const void *)k_gae, dim3(g),
-                                     dim3(kGaeThreads), args, 0, s);
+  const uint64_t grid = (E + kGaeWarps - 1) / kGaeWarps;
+  double *partial = nullptr;
+  if (adv_norm) {
+    partial = (double *)ctx_scratch(c, grid * 2 * sizeof(double));
+    if (!partial) return cudaErrorMemoryAllocation;
+  }
+  // A is kept between the kernels in adv, or in adv_norm itself (fp32; the
+  // normalisation error this adds is below 2^-24 |A| / std)
+  float *A_out = adv ? adv : adv_norm;
+  cudaError_t e = launch_pdl(k_gae_scan, dim3((unsigned)grid), dim3(kGaeThreads), s,
+                             r, v, d, T, E, gamma, lambda, A_out, ret, partial);
+  if (e != cudaSuccess || !adv_norm) return e;
+  const uint64_t n = (uint64_t)T * E;
+  uint64_t ng = (n + kNormThreads - 1) / kNormThreads;
+  if (ng > 4ull * c->coop_sms) ng = 4ull * c->coop_sms;
+  return launch_pdl(k_gae_norm, dim3((unsigned)ng), dim3(kNormThreads), s,
+                    (const float *)A_out, adv_norm, n, (const double *)partial,
+                    (uint32_t)grid);
 }
 
 }  // namespace edp

@@ -78,9 +78,19 @@ k_sample_prio(TreeView t, uint32_t B, uint64_t seed, uint64_t round,
   pdl_launch();
   const uint32_t cached = t.depth - 1 < (uint32_t)kSmemLevels ? t.depth - 1 : kSmemLevels;
   const uint32_t ncached = cached == 0 ? 0 : (cached == 1 ? 32 : 32 + 1024);
-  for (uint32_t i = threadIdx.x; i < ncached; i += blockDim.x)
-    top[i] = t.nodes[1 + i];  // levels 1.. start right after the root
+  // levels 1.. start right after the root; all loads issued before any use
+  uint64_t v5[5];
+#pragma unroll
+  for (int u = 0; u < 5; ++u) {
+    const uint32_t i = threadIdx.x + u * 256;
+    v5[u] = i < ncached ? ld_keep(t.nodes + 1 + i, keep) : 0ull;
+  }
   const uint64_t S = t.nodes[0];
+#pragma unroll
+  for (int u = 0; u < 5; ++u) {
+    const uint32_t i = threadIdx.x + u * 256;
+    if (i < ncached) top[i] = v5[u];
+  }
   __syncthreads();
   const uint32_t warps = (gridDim.x * blockDim.x) >> 5;
   for (uint32_t k = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; k < B;
