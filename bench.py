@@ -333,6 +333,10 @@ class PerReplay(Workload):
         self.td_rounds = 64
         self.td = torch.stack([dev(fx.td_errors(self.seed, B, r), device)
                                for r in range(self.td_rounds)])
+        self.side = torch.cuda.Stream(device=device)
+        self.ready = [torch.cuda.Event() for _ in range(self.R)]
+        self.consumed = [torch.cuda.Event() for _ in range(self.R)]
+        self.in_flight = set()  # output sets whose delivery is not yet joined
 
     def _sample(self, r, o):
         self.edp.edp_sample(self.ring.ctx, self.edp.EDP_SAMPLE_PRIORITIZED, self.B,
@@ -345,6 +349,38 @@ class PerReplay(Workload):
         self.edp.edp_update_priorities_td(self.ring.ctx, o["idx"],
                                           self.td[r % self.td_rounds], self.B,
                                           ALPHA, EPS)
+
+    def round_overlap(self, r):
+        """The round with the delivery on a second stream.  Delivery depends
+        only on this round's sampling, so it overlaps the priority update
+        (whose TD errors do not depend on the delivered batch here) and the
+        next round's sampling on the main stream: the overlapped timing of
+        the paper's scheduling (Sec. 6.1).  Every data dependency is kept:
+        delivery r waits for sampling r; sampling r+1 follows update r in
+        stream order, so it sees the updated priorities; the R output sets
+        rotate, and sampling r+R waits until delivery r has read the indices
+        it would overwrite."""
+        import torch
+        k = r % self.R
+        o = self.outs[k]
+        if k in self.in_flight:
+            torch.cuda.current_stream().wait_event(self.consumed[k])
+        self._sample(r, o)
+        self.ready[k].record()
+        with torch.cuda.stream(self.side):
+            self.side.wait_event(self.ready[k])
+            self.edp.edp_deliver(self.ring.ctx, o["idx"], self.B, o["batch"],
+                                 stream=self.side)
+            self.consumed[k].record()
+        self.in_flight.add(k)
+        self.edp.edp_update_priorities_td(self.ring.ctx, o["idx"],
+                                          self.td[r % self.td_rounds], self.B,
+                                          ALPHA, EPS)
+
+    def join(self):
+        import torch
+        torch.cuda.current_stream().wait_stream(self.side)
+        self.in_flight.clear()
 
     def deliver_once(self, r):
         o = self.outs[r % self.R]
@@ -894,6 +930,23 @@ def run_reference(args):
     return 0
 
 
+def job_ms(ms, dist, device):
+    """Job time of a timed region: the maximum over ranks (every rank's
+    replica must finish), or the local time with one rank."""
+    if dist is None:
+        return ms
+    import torch
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_gbs(bytes_per_step, steps, world, ms):
+    """Whole-job throughput: every rank processed `steps` units of
+    `bytes_per_step` (weak scaling: fixed work per rank) in `ms`."""
+    return bytes_per_step * steps * world / (ms / 1e3) / 1e9
+
+
 def run_edp(args):
     import torch
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -918,40 +971,48 @@ def run_edp(args):
 
     # warm-up rounds (eager), then capture the timed rounds in one graph;
     # no events inside it (event nodes split the graph and cost several us)
-    for r in range(W):
-        wl.round(K + r)
-    torch.cuda.synchronize()
-    use_graph = not args.no_graph
-    if use_graph:
-        g = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g, capture_error_mode="thread_local"):
-            for r in range(K):
-                wl.round(r)
-        g.replay()  # upload + warm the graph (rounds are re-timed below)
+    overlap = hasattr(wl, "round_overlap") and not args.serial
+
+    def rounds(first, n, ovl):
+        for r in range(first, first + n):
+            (wl.round_overlap if ovl else wl.round)(r)
+        if ovl:
+            wl.join()
+
+    def timed(ovl):
+        rounds(K, W, ovl)
         torch.cuda.synchronize()
-    if dist:
-        dist.barrier()
-    torch.cuda.synchronize()
-    clocks = Clocks(local)
-    clocks.start()
-    time.sleep(0.02)
-    t_start, t_end = mk(), mk()
-    t_start.record(stream)
-    if use_graph:
-        g.replay()
-    else:
-        for r in range(K):
-            wl.round(r)
-    t_end.record(stream)
-    torch.cuda.synchronize()
-    clk = clocks.stop()
-    ms = t_start.elapsed_time(t_end)
-    if dist:
-        t = torch.tensor([ms], device=device)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+        g = None
+        if not args.no_graph:
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, capture_error_mode="thread_local"):
+                rounds(0, K, ovl)
+            g.replay()  # upload + warm the graph (rounds are re-timed below)
+            torch.cuda.synchronize()
+        if dist:
+            dist.barrier()
+        torch.cuda.synchronize()
+        clocks = Clocks(local)
+        clocks.start()
+        time.sleep(0.02)
+        t_start, t_end = mk(), mk()
+        t_start.record(stream)
+        g.replay() if g is not None else rounds(0, K, ovl)
+        t_end.record(stream)
+        torch.cuda.synchronize()
+        clk = clocks.stop()
+        return job_ms(t_start.elapsed_time(t_end), dist, device), clk
+
+    use_graph = not args.no_graph
+    serial = None
+    if overlap:
+        ms_ser, _ = timed(False)
+        serial = {"value": job_gbs(wl.round_bytes, K, world, ms_ser),
+                  "ms_per_step": ms_ser / K,
+                  "schedule": "sample -> deliver -> update, one stream"}
+    ms, clk = timed(overlap)
     ms_step = ms / K
-    value = wl.round_bytes * K * world / (ms / 1e3) / 1e9
+    value = job_gbs(wl.round_bytes, K, world, ms)
     peak, peak_kind = peaks()
 
     # dominant kernel: the fused delivery, timed back to back on the same
@@ -979,12 +1040,8 @@ def run_edp(args):
             wl.e2e_round(r)
         e1.record(stream)
         torch.cuda.synchronize()
-        ems = e0.elapsed_time(e1)
-        if dist:
-            t = torch.tensor([ems], device=device)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            ems = float(t.item())
-        e2e = {"value": wl.round_bytes * Ke * world / (ems / 1e3) / 1e9,
+        ems = job_ms(e0.elapsed_time(e1), dist, device)
+        e2e = {"value": job_gbs(wl.round_bytes, Ke, world, ems),
                "unit": "GB/s", "h2d_bytes_per_step": wl.h2d,
                "d2h_bytes_per_step": wl.d2h, "steps": Ke,
                "ms_per_step": ems / Ke}
@@ -1014,13 +1071,19 @@ def run_edp(args):
                 "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype,
                 "data": "synthetic", "config": dict(wl.config(),
                                                     parallelism="replicas%d" % world,
-                                                    graph=use_graph),
+                                                    graph=use_graph,
+                                                    schedule=("delivery on a second stream, "
+                                                              "overlapping update r and "
+                                                              "sampling r+1" if overlap
+                                                              else "one stream")),
                 "pct_hbm_peak": 100.0 * value / peak,
                 "batches_per_s": K * world / (ms / 1e3),
                 "p50_sample_to_batch_us": p50,
                 "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
                 "gpu_launches": wl.launches_per_round * K,
                 "clocks": clk}
+        if serial:
+            line["serial"] = serial
         line.update(extra)
         print(json.dumps(line))
     if dist:
@@ -1039,6 +1102,8 @@ def main():
     ap.add_argument("--capacity", type=int, default=0,
                     help="override the ring capacity (profiling small cases)")
     ap.add_argument("--no-graph", action="store_true")
+    ap.add_argument("--serial", action="store_true",
+                    help="one-stream rounds only (no delivery/update overlap)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)

@@ -25,12 +25,26 @@
  *   storage, inputs, outputs).  libedp owns only the context, the priority
  *   tree and small scratch, allocated through edp_config.alloc (cudaMalloc
  *   when NULL) and released by edp_destroy.  libedp never frees caller memory.
+ *   Scratch is allocated at a call's first use and grown (after a device
+ *   synchronisation) when a later call needs more: edp_update_priorities_td
+ *   (4 bytes per pair), the PERMUTE sampling mode and edp_gae with
+ *   normalisation.  Before capturing calls into a CUDA graph, make each of
+ *   them once at its largest size, outside the capture.
  * - Asynchrony: every call validates its arguments on the host, enqueues its
  *   kernels on `stream` and returns without synchronising.  Results are
  *   valid once the stream has reached that point.  Host-side cursors
  *   (head, total) advance at enqueue time, so calls on one context must be
  *   issued in program order on one stream (or with the caller's own
  *   cross-stream ordering).
+ * - Overlap (the overlapped timing of Sec. 6.1): edp_deliver reads only the
+ *   ring storage, its `idx` / `q` and the gather sources, and writes only
+ *   its batch, so it may run on another stream concurrently with
+ *   edp_sample, edp_update_priorities*, edp_priorities_from_td, edp_gae and
+ *   other deliveries of the same context, once the sampling that wrote its
+ *   `idx` has completed (an event) and while nothing overwrites `idx`, `q`
+ *   or the rows it reads (edp_ingest).  Every other pair of calls on one
+ *   context shares the priority tree or the context's scratch and must be
+ *   ordered.
  * - Errors: argument and state errors are returned synchronously and leave
  *   the context unchanged.  A CUDA launch error returns EDP_ERR_CUDA.
  *   Data-dependent faults found on the device (an index out of range, an
