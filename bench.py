@@ -205,6 +205,51 @@ class Workload:
     def config(self):
         return {"workload": self.name}
 
+    def schedules(self):
+        """[(name, round function, description)], the main schedule first;
+        every schedule runs the same work per round."""
+        return [("one stream", self.round, "one stream")]
+
+    def join(self):
+        """Make the current stream wait for the workload's side streams."""
+        import torch
+        if getattr(self, "side_used", False):
+            for st in self.sides:
+                torch.cuda.current_stream().wait_stream(st)
+        self.side_used = False
+        self.in_flight = set()
+
+    def _init_overlap(self, device, sets, sides=2):
+        import torch
+        self.sides = [torch.cuda.Stream(device=device) for _ in range(sides)]
+        self.ready = [torch.cuda.Event() for _ in range(sets)]
+        self.consumed = [torch.cuda.Event() for _ in range(sets)]
+        self.in_flight = set()  # output sets whose delivery is not yet joined
+
+    def _overlapped(self, k, sample, deliver, after=None):
+        """One round with its delivery on a side stream: sample() on the
+        current stream; deliver(stream) on side stream k mod (number of side
+        streams) once the sampling has finished; after() (if any) on the
+        current stream meanwhile.  Consecutive deliveries alternate between
+        the side streams, so one's ramp-up overlaps the previous one's tail.
+        Output set k is reused only after its previous delivery has read
+        its indices."""
+        import torch
+        main = torch.cuda.current_stream()
+        if k in self.in_flight:
+            main.wait_event(self.consumed[k])
+        sample()
+        self.ready[k].record()
+        side = self.sides[k % len(self.sides)]
+        with torch.cuda.stream(side):
+            side.wait_event(self.ready[k])
+            deliver(side)
+            self.consumed[k].record()
+        self.in_flight.add(k)
+        self.side_used = True
+        if after is not None:
+            after()
+
     def _graph_or_eager(self, body, graph):
         import torch
         body()
@@ -333,10 +378,7 @@ class PerReplay(Workload):
         self.td_rounds = 64
         self.td = torch.stack([dev(fx.td_errors(self.seed, B, r), device)
                                for r in range(self.td_rounds)])
-        self.side = torch.cuda.Stream(device=device)
-        self.ready = [torch.cuda.Event() for _ in range(self.R)]
-        self.consumed = [torch.cuda.Event() for _ in range(self.R)]
-        self.in_flight = set()  # output sets whose delivery is not yet joined
+        self._init_overlap(device, self.R)
 
     def _sample(self, r, o):
         self.edp.edp_sample(self.ring.ctx, self.edp.EDP_SAMPLE_PRIORITIZED, self.B,
@@ -351,7 +393,7 @@ class PerReplay(Workload):
                                           ALPHA, EPS)
 
     def round_overlap(self, r):
-        """The round with the delivery on a second stream.  Delivery depends
+        """The round with the delivery on a side stream.  Delivery depends
         only on this round's sampling, so it overlaps the priority update
         (whose TD errors do not depend on the delivered batch here) and the
         next round's sampling on the main stream: the overlapped timing of
@@ -360,27 +402,20 @@ class PerReplay(Workload):
         stream order, so it sees the updated priorities; the R output sets
         rotate, and sampling r+R waits until delivery r has read the indices
         it would overwrite."""
-        import torch
         k = r % self.R
         o = self.outs[k]
-        if k in self.in_flight:
-            torch.cuda.current_stream().wait_event(self.consumed[k])
-        self._sample(r, o)
-        self.ready[k].record()
-        with torch.cuda.stream(self.side):
-            self.side.wait_event(self.ready[k])
-            self.edp.edp_deliver(self.ring.ctx, o["idx"], self.B, o["batch"],
-                                 stream=self.side)
-            self.consumed[k].record()
-        self.in_flight.add(k)
-        self.edp.edp_update_priorities_td(self.ring.ctx, o["idx"],
-                                          self.td[r % self.td_rounds], self.B,
-                                          ALPHA, EPS)
+        self._overlapped(
+            k, lambda: self._sample(r, o),
+            lambda st: self.edp.edp_deliver(self.ring.ctx, o["idx"], self.B,
+                                            o["batch"], stream=st),
+            lambda: self.edp.edp_update_priorities_td(
+                self.ring.ctx, o["idx"], self.td[r % self.td_rounds], self.B,
+                ALPHA, EPS))
 
-    def join(self):
-        import torch
-        torch.cuda.current_stream().wait_stream(self.side)
-        self.in_flight.clear()
+    def schedules(self):
+        return [("overlapped", self.round_overlap,
+                 "delivery on side streams, overlapping update r and sampling r+1"),
+                ("serial", self.round, "sample -> deliver -> update, one stream")]
 
     def deliver_once(self, r):
         o = self.outs[r % self.R]
@@ -580,12 +615,14 @@ class PpoIteration(Workload):
         self.mb = self.n // self.M
         F = self.H * self.W * self.C
         self.F = F
-        # one mini-batch delivery: obs read + bf16 write + adv/ret gathers
-        self.deliver_bytes = self.mb * (F + 2 * F + 8 + 8 + 8)
+        # per delivered sample: obs read + bf16 write + adv/ret gathers + idx
+        self.sample_bytes = F + 2 * F + 8 + 8 + 8
+        # the main schedule delivers the whole iteration in one call
+        self.deliver_bytes = self.n * self.sample_bytes
         gae = self.T * self.E * (4 + 1 + 4) + self.E * 4 + 3 * self.T * self.E * 4
         perm = self.n * (8 + 8 + 8 + 4 + 8 + 4 + 8) + 3 * 4 * (self.n // 4)
-        self.round_bytes = gae + perm + self.M * self.deliver_bytes
-        self.launches_per_round = 2 + self.M
+        self.round_bytes = gae + perm + self.n * self.sample_bytes
+        self.launches_per_round = 2 + 3 + 1  # GAE, shuffle, delivery
 
     def config(self):
         return {"workload": self.name, "envs": self.E, "steps": self.T,
@@ -615,6 +652,16 @@ class PpoIteration(Workload):
                                 device=device) for _ in range(2)]
         self.a_out = torch.empty(self.mb, device=device)
         self.r_out = torch.empty(self.mb, device=device)
+        # all M mini-batches of one iteration, mini-batch m = rows
+        # [m * 4096, (m + 1) * 4096) (805 MB, larger than L2)
+        self.out_all = torch.empty((self.n, self.C, self.H, self.W), dtype=torch.bfloat16,
+                                   device=device)
+        self.a_all = torch.empty(self.n, device=device)
+        self.r_all = torch.empty(self.n, device=device)
+        self.side = torch.cuda.Stream(device=device)
+        self.sides = [self.side]
+        self.fork = torch.cuda.Event()
+        self.gae_done = torch.cuda.Event()
         # first calls allocate scratch outside any capture
         self._gae()
         edp.edp_sample(self.ring.ctx, edp.EDP_SAMPLE_PERMUTE, self.n, self.seed, 0, self.idx)
@@ -638,8 +685,43 @@ class PpoIteration(Workload):
         for m in range(self.M):
             self._mb(m, r)
 
+    def _deliver_all(self):
+        b = self.edp.make_batch(self.out_all,
+                                gather=[(self.nrm.view(-1), self.a_all),
+                                        (self.ret.view(-1), self.r_all)])
+        self.edp.edp_deliver(self.ring.ctx, self.idx, self.n, b)
+
+    def round_batched(self, r):
+        """GAE on a side stream beside the shuffle (the two are independent:
+        GAE reads the rollout scalars, the shuffle only its keys), then one
+        delivery call for the whole iteration: the delivery granularity
+        g_del = 1 of Sec. 4.2 instead of one call per mini-batch.  Mini-batch
+        m is rows [4096 m, 4096 (m + 1)) of the output, equal to what the
+        m-th per-mini-batch call delivers."""
+        import torch
+        main = torch.cuda.current_stream()
+        self.fork.record()  # the side stream starts after prior work
+        self.side_used = True
+        with torch.cuda.stream(self.side):
+            self.side.wait_event(self.fork)
+            self.edp.edp_gae(self.ring.ctx, self.r, self.v, self.d, self.T, self.E,
+                             0.99, 0.95, self.adv, self.ret, self.nrm, stream=self.side)
+            self.gae_done.record()
+        self.edp.edp_sample(self.ring.ctx, self.edp.EDP_SAMPLE_PERMUTE, self.n,
+                            self.seed, r, self.idx)
+        main.wait_event(self.gae_done)
+        self._deliver_all()
+
+    def schedules(self):
+        return [("batched", self.round_batched,
+                 "GAE on a side stream beside the shuffle; one delivery call "
+                 "for all 8 mini-batches (g_del = 1)"),
+                ("per-minibatch", self.round,
+                 "GAE, shuffle, 8 mini-batch deliveries of 4,096, one stream "
+                 "(g_del = 1/8)")]
+
     def deliver_once(self, r):
-        self._mb(r % self.M, r)
+        self._deliver_all()
 
     def latency_step(self, r, ev_end):
         self._gae()
@@ -780,6 +862,7 @@ class MmReplay(Workload):
                      rew=torch.empty(B, device=device))
             o["batch"] = edp.make_batch(o["obs"], tokens=o["tok"], reward=o["rew"])
             self.outs.append(o)
+        self._init_overlap(device, len(self.outs))
 
     def round(self, r):
         ctx = self.ring.ctx
@@ -789,6 +872,24 @@ class MmReplay(Workload):
         o = self.outs[r % 2]
         self.edp.edp_sample(ctx, self.edp.EDP_SAMPLE_UNIFORM, self.B, self.seed, r, o["idx"])
         self.edp.edp_deliver(ctx, o["idx"], self.B, o["batch"])
+
+    def round_overlap(self, r):
+        """Delivery r on a side stream while round r+1 samples (no ingest:
+        an ingest would overwrite rows a pending delivery reads)."""
+        k = r % 2
+        o = self.outs[k]
+        self._overlapped(
+            k, lambda: self.edp.edp_sample(self.ring.ctx, self.edp.EDP_SAMPLE_UNIFORM,
+                                           self.B, self.seed, r, o["idx"]),
+            lambda st: self.edp.edp_deliver(self.ring.ctx, o["idx"], self.B, o["batch"],
+                                            stream=st))
+
+    def schedules(self):
+        one = ("one stream", self.round, "sample -> deliver, one stream")
+        if self.ingest:
+            return [one]
+        return [("overlapped", self.round_overlap,
+                 "delivery on side streams, overlapping sampling r+1"), one]
 
     def deliver_once(self, r):
         o = self.outs[r % 2]
@@ -971,22 +1072,26 @@ def run_edp(args):
 
     # warm-up rounds (eager), then capture the timed rounds in one graph;
     # no events inside it (event nodes split the graph and cost several us)
-    overlap = hasattr(wl, "round_overlap") and not args.serial
+    scheds = wl.schedules()
+    if args.schedule:
+        names = [n for n, _, _ in scheds]
+        if args.schedule not in names:
+            raise SystemExit("--schedule: one of %s" % names)
+        scheds.sort(key=lambda x: x[0] != args.schedule)
 
-    def rounds(first, n, ovl):
+    def rounds(first, n, fn):
         for r in range(first, first + n):
-            (wl.round_overlap if ovl else wl.round)(r)
-        if ovl:
-            wl.join()
+            fn(r)
+        wl.join()
 
-    def timed(ovl):
-        rounds(K, W, ovl)
+    def timed(fn):
+        rounds(K, W, fn)
         torch.cuda.synchronize()
         g = None
         if not args.no_graph:
             g = torch.cuda.CUDAGraph()
             with torch.cuda.graph(g, capture_error_mode="thread_local"):
-                rounds(0, K, ovl)
+                rounds(0, K, fn)
             g.replay()  # upload + warm the graph (rounds are re-timed below)
             torch.cuda.synchronize()
         if dist:
@@ -997,20 +1102,19 @@ def run_edp(args):
         time.sleep(0.02)
         t_start, t_end = mk(), mk()
         t_start.record(stream)
-        g.replay() if g is not None else rounds(0, K, ovl)
+        g.replay() if g is not None else rounds(0, K, fn)
         t_end.record(stream)
         torch.cuda.synchronize()
         clk = clocks.stop()
         return job_ms(t_start.elapsed_time(t_end), dist, device), clk
 
     use_graph = not args.no_graph
-    serial = None
-    if overlap:
-        ms_ser, _ = timed(False)
-        serial = {"value": job_gbs(wl.round_bytes, K, world, ms_ser),
-                  "ms_per_step": ms_ser / K,
-                  "schedule": "sample -> deliver -> update, one stream"}
-    ms, clk = timed(overlap)
+    others = []
+    for name, fn, desc in scheds[1:]:
+        ms_o, _ = timed(fn)
+        others.append({"schedule": name, "value": job_gbs(wl.round_bytes, K, world, ms_o),
+                       "ms_per_step": ms_o / K, "description": desc})
+    ms, clk = timed(scheds[0][1])
     ms_step = ms / K
     value = job_gbs(wl.round_bytes, K, world, ms)
     peak, peak_kind = peaks()
@@ -1072,18 +1176,15 @@ def run_edp(args):
                 "data": "synthetic", "config": dict(wl.config(),
                                                     parallelism="replicas%d" % world,
                                                     graph=use_graph,
-                                                    schedule=("delivery on a second stream, "
-                                                              "overlapping update r and "
-                                                              "sampling r+1" if overlap
-                                                              else "one stream")),
+                                                    schedule="%s: %s" % scheds[0][::2]),
                 "pct_hbm_peak": 100.0 * value / peak,
                 "batches_per_s": K * world / (ms / 1e3),
                 "p50_sample_to_batch_us": p50,
                 "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
                 "gpu_launches": wl.launches_per_round * K,
                 "clocks": clk}
-        if serial:
-            line["serial"] = serial
+        if others:
+            line["other_schedules"] = others
         line.update(extra)
         print(json.dumps(line))
     if dist:
@@ -1102,8 +1203,9 @@ def main():
     ap.add_argument("--capacity", type=int, default=0,
                     help="override the ring capacity (profiling small cases)")
     ap.add_argument("--no-graph", action="store_true")
-    ap.add_argument("--serial", action="store_true",
-                    help="one-stream rounds only (no delivery/update overlap)")
+    ap.add_argument("--schedule", default="",
+                    help="the workload's schedule timed as the main number "
+                         "(default: its first); the others are reported too")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)

@@ -17,11 +17,16 @@ namespace edp {
 enum : uint32_t {
   DEVERR_INDEX = 1u,    // a slot index outside the sampleable range
   DEVERR_EMPTY = 2u,    // total priority 0 at sampling time
-  DEVERR_TIMEOUT = 4u,  // a bounded wait (bulk-copy barrier) expired
+  DEVERR_TIMEOUT = 4u,  // a bounded device-side wait expired (no kernel waits now)
   DEVERR_TREE = 8u,     // a tree descent found no child holding its target
 };
 
 // Small device-resident control block (one per context).
+// Work counters of the dynamically scheduled delivery kernels: launch n of
+// a context uses pair n mod kWorkSlots (chunks handed out, CTAs retired);
+// the last CTA of the launch resets its pair to zero.
+constexpr int kWorkSlots = 32;
+
 struct Ctrl {
   uint32_t err;
   uint32_t pending_q;  // deferred priority of the newest transition
@@ -30,6 +35,7 @@ struct Ctrl {
   uint32_t upd_count;  // priority update: CTAs done with phase 1
   uint32_t pad[2];
   unsigned long long bad_index;  // first offending index (diagnostics)
+  uint32_t work[2 * kWorkSlots];
 };
 
 constexpr int kFanout = 32;
@@ -65,6 +71,7 @@ struct edp_ctx {
   float nmean[4] = {}, ns1[4] = {}, ns2[4] = {}, nstd[4] = {};
   int norm_fast = 1;  // 0: the constants do not reproduce t/std -> divide
   int coop_sms = 0;
+  uint32_t work_seq = 0;  // delivery launches so far (work counter pairs)
   std::string err;
 };
 
@@ -198,83 +205,6 @@ __device__ __forceinline__ double pow_pos(double x, double a) {
   q = fma(q, r, 1.0);
   const long long ni = (long long)n;
   return q * __longlong_as_double((ni + 1023) << 52);
-}
-
-// ---------------------------------------------------------------------------
-// Bulk asynchronous copies (TMA, cp.async.bulk) and mbarriers.  Addresses
-// and sizes are multiples of 16 bytes.  Every wait on an mbarrier is bounded:
-// after ~1 s of clock cycles it records DEVERR_TIMEOUT and gives up.
-// ---------------------------------------------------------------------------
-__device__ __forceinline__ uint32_t smem_u32(const void *p) {
-  return (uint32_t)__cvta_generic_to_shared(p);
-}
-__device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)),
-               "r"(count)
-               : "memory");
-}
-__device__ __forceinline__ void fence_mbar_init() {
-  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-}
-// make this thread's shared-memory writes visible to the bulk-copy engine
-__device__ __forceinline__ void fence_proxy_async() {
-  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
-// arrive once and expect `bytes` of bulk-copy transactions (0: plain arrive)
-__device__ __forceinline__ void mbar_expect_tx(uint64_t *bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(
-                   smem_u32(bar)),
-               "r"(bytes)
-               : "memory");
-}
-__device__ __forceinline__ void tma_load(void *dst_smem, const void *src,
-                                         uint32_t bytes, uint64_t *bar,
-                                         uint64_t policy) {
-  asm volatile(
-      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
-      " [%0], [%1], %2, [%3], %4;" ::"r"(smem_u32(dst_smem)),
-      "l"(src), "r"(bytes), "r"(smem_u32(bar)), "l"(policy)
-      : "memory");
-}
-__device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;"
-      " selp.u32 %0, 1, 0, p; }"
-      : "=r"(ok)
-      : "r"(smem_u32(bar)), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity,
-                                          Ctrl *ctrl) {
-  if (mbar_try_wait(bar, parity)) return true;
-  const long long t0 = clock64();
-  while (!mbar_try_wait(bar, parity)) {
-    if (clock64() - t0 > 2000000000ll) {
-      atomicOr(&ctrl->err, DEVERR_TIMEOUT);
-      return false;
-    }
-  }
-  return true;
-}
-__device__ __forceinline__ void tma_store(void *dst, const void *src_smem,
-                                          uint32_t bytes, uint64_t policy) {
-  asm volatile(
-      "cp.async.bulk.global.shared::cta.bulk_group.L2::cache_hint [%0], [%1], %2, %3;" ::"l"(dst),
-      "r"(smem_u32(src_smem)), "r"(bytes), "l"(policy)
-      : "memory");
-}
-__device__ __forceinline__ void tma_commit() {
-  asm volatile("cp.async.bulk.commit_group;" ::: "memory");
-}
-// wait until at most N committed store groups still read shared memory
-template <int N>
-__device__ __forceinline__ void tma_wait_read() {
-  asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
-}
-__device__ __forceinline__ void tma_wait_all() {
-  asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
 }
 
 // L2 residency hints: payload streams through (an evict_first policy) so

@@ -1,24 +1,26 @@
 // k_deliver.cu -- fused delivery: gather the sampled transitions, transform
 // their uint8 payload into the learner layout, collate metadata, and
-// compute importance weights, in one pass over the payload (Sec. 2.2:
-// delivery "materializes the selected transitions and performs batch/layout
-// transformations").
+// compute importance weights, in one pass over the payload (the delivery
+// operator of Sec. 2.2: the chosen transitions are materialised in the
+// layout and batch shape the learner consumes).
 //
 // Work decomposition: the batch's output is a flat sequence of units (a
-// 32-bit word of a frame, an 8-pixel group, an 8-byte run of a plane).  The
-// grid is one wave of persistent CTAs (occupancy x SMs) and each warp takes
-// one contiguous, equal span of that sequence, so every SM finishes at the
-// same time.  A warp walks its span segment by segment (a segment never
-// crosses a frame or image), resolving the sample's slot, episode-boundary
-// mask and source pointer once per segment.  Loads are the payload bytes a
-// lane needs for one 16-byte output store, so every warp-wide store
-// instruction writes 512 contiguous bytes.  The byte->float step is
-// x = b (exact), fl32(b/255) = fma(x, r1, x*r2) with one rounding (see
-// unit_f32), then optionally the per-channel normalisation and the
-// round-to-nearest-even bfloat16 conversion.
+// 32-bit word of a frame, an 8-pixel group, an 8-byte run of a plane), cut
+// into warp spans whose size is set from the work, not from the grid: a
+// warp runs a few iterations of its unrolled loop per span and the grid
+// holds as many CTAs as that takes (several waves), so the block scheduler,
+// or for the frame stack a work counter, balances the tail.  A warp walks
+// its span segment by segment (a segment never crosses a frame or image),
+// resolving the sample's slot, episode-boundary mask and source pointer
+// once per segment.  Loads are the payload bytes a lane needs for one
+// 16-byte output store, so every warp-wide store instruction writes 512
+// contiguous bytes.  The byte->float step is x = b (exact),
+// fl32(b/255) = fma(x, r1, x*r2) with one rounding (see unit_f32), then
+// optionally the per-channel normalisation and the round-to-nearest-even
+// bfloat16 conversion.
 //
-// This kernel is HBM-bound: per sample it reads the unique source bytes once
-// and writes the (2-4x larger) float output once.
+// These kernels are HBM-bound: per sample they read the unique source bytes
+// once and write the (2-8x larger) output once.
 #include "edp_internal.cuh"
 
 namespace edp {
@@ -46,6 +48,7 @@ struct Common {
   const float *gsrc0, *gsrc1;
   float *gdst0, *gdst1;
   Ctrl *ctrl;
+  uint32_t *work;  // this launch's work counter pair, or null (one chunk per CTA)
   float r1, r2;
 };
 
@@ -138,189 +141,135 @@ __device__ __forceinline__ float byte_f(uint32_t w, int i) {
 }
 
 // ---------------------------------------------------------------------------
-// Frame stack, float32 (DQN), on the bulk-copy engine.  A unit is one part
-// (<= 2400 bytes) of frame m in [0, K] of sample k -- the frame at logical
+// Frame stack, float32 (DQN), on the load / store units.  A unit is one
+// 32-bit word of frame m in [0, U) of sample k -- the frame at logical
 // offset j = off - K + 1 + m, which is obs slot m (m < K) and next_obs slot
-// m - 1 (m >= 1).  Each persistent CTA owns a contiguous range of units and
-// runs a kStages-deep pipeline over it:
-//   thread 0  bulk-loads the part of unit i + kStages - 1 into its stage
-//             (mbarrier with transaction count; units needing no load arrive
-//             on the barrier without bytes so the phases stay in step);
-//   all       wait for unit i's stage, convert its bytes to fp32 in shared
-//             memory, fence the async proxy;
-//   thread 0  bulk-stores the fp32 tile to obs and/or next_obs (a zero tile
-//             for zero-padded frames) and commits one store group per unit;
-//             before a stage's tile is rewritten, at most kStages - 1 groups
-//             may still be reading shared memory.
-// The per-unit control (slot, episode-boundary mask, source and destination
-// offsets) is resolved for 256 units at a time, one thread per unit, before
-// the pipeline; the head unit of each sample also runs the collate.
+// m - 1 (m >= 1).  A lane turns its word into one float4 and stores it to
+// obs and / or next_obs, so every warp-wide store writes 512 contiguous
+// bytes.  Per segment (the part of one frame inside a warp's span) the warp
+// resolves the slot and the episode mask once: lanes 0..K-m-1 load the done
+// flags of offsets j..off and a ballot gives "an episode end before the
+// anchor" (zeroes the frame in obs and next_obs) and "at the anchor" (zeroes
+// it in next_obs only).
+//
+// Scheduling: the work is cut into chunks of kWarps spans.  A batch with
+// more chunks than the grid holds runs on a persistent grid that leaves
+// kStackHeadroom CTA slots of every SM free -- so the small sampling and
+// priority-update kernels of the next round find room beside a running
+// delivery (the overlapped timing of Sec. 6.1) -- and its CTAs take chunks
+// from the launch's work counter until the batch is done, which balances
+// the tail without relying on all CTAs being resident.  A smaller batch
+// runs one chunk per CTA with no counter.
 // ---------------------------------------------------------------------------
-constexpr int kStages = 4;
-constexpr int kCtlUnits = 256;
-
 struct StackArgs {
   const uint8_t *frames;
-  uint32_t F;     // bytes per frame
+  uint32_t F;     // bytes per frame (multiple of 16)
+  uint32_t W;     // 32-bit words per frame
   uint32_t K;
   uint32_t U;     // frames per sample (K, or K + 1 with next_obs)
-  uint32_t P;     // parts per frame
-  uint32_t part;  // bytes per part (multiple of 16; the last may be shorter)
+  uint32_t span;  // units per warp per chunk (multiple of 32)
   float *obs;
   float *next;
 };
 
-struct UnitCtl {
-  uint64_t src;    // byte offset of the part in the frame ring
-  uint64_t dobs;   // float offset in obs, or ~0
-  uint64_t dnext;  // float offset in next_obs, or ~0
-  uint32_t bytes;  // bytes of this part
-  uint32_t flags;  // kLoad | kZeroObs | kZeroNext
-};
-constexpr uint32_t kLoad = 1u, kZeroObs = 2u, kZeroNext = 4u;
-
-__host__ __device__ constexpr size_t align_up(size_t x, size_t a) {
-  return (x + a - 1) / a * a;
+// Stack units [f, end) of one warp.
+template <int UN>
+__device__ __forceinline__ void stack_span(const Common &c, const StackArgs &a,
+                                           uint64_t f, uint64_t end, int lane,
+                                           uint64_t pol) {
+  const uint64_t per = (uint64_t)a.U * a.W;  // units per sample
+  const float4 zero4 = make_float4(0.f, 0.f, 0.f, 0.f);
+  while (f < end) {
+    const uint32_t k = (uint32_t)(f / per);
+    const uint32_t rem = (uint32_t)(f - (uint64_t)k * per);
+    const uint32_t m = rem / a.W;
+    const uint32_t w_lo = rem - m * a.W;
+    const uint64_t seg_end = min(end, (uint64_t)k * per + (uint64_t)(m + 1) * a.W);
+    const uint32_t w_hi = (uint32_t)(seg_end - (uint64_t)k * per - (uint64_t)m * a.W);
+    const bool head = rem == 0;
+    uint64_t slot = 0, off = 0;
+    const bool ok = sample_slot(c, k, &slot, &off, head && lane == 0);
+    if (head) collate(c, k, ok, slot, off, lane);
+    const int64_t j = (int64_t)off - (int64_t)(a.K - 1) + (int64_t)m;
+    bool end_before = false, end_at = false;
+    if (ok && j >= 0 && (int64_t)off >= j) {
+      const uint32_t span = (uint32_t)((int64_t)off - j + 1);  // 1..K
+      bool d = false;
+      if ((uint32_t)lane < span) {
+        const uint64_t t2 = c.oldest + (uint64_t)j + lane;
+        d = c.done[t2 >= c.cap ? t2 - c.cap : t2] != 0;
+      }
+      const unsigned bal = __ballot_sync(kFull, d);
+      end_at = (bal >> (span - 1)) & 1u;
+      end_before = (bal & ((1u << (span - 1)) - 1u)) != 0;
+    }
+    const bool has_obs = m < a.K;
+    const bool has_next = a.next && m >= 1;
+    const bool zo = !ok || j < 0 || end_before;
+    const bool zn = zo || end_at;
+    const bool load = (has_obs && !zo) || (has_next && !zn);
+    const uint64_t js = c.oldest + (uint64_t)(j < 0 ? 0 : j);
+    const uint32_t *src = reinterpret_cast<const uint32_t *>(
+        a.frames + (js >= c.cap ? js - c.cap : js) * a.F);
+    float4 *dobs = has_obs ? reinterpret_cast<float4 *>(
+                                 a.obs + ((uint64_t)k * a.K + m) * a.F)
+                           : nullptr;
+    float4 *dnext = has_next ? reinterpret_cast<float4 *>(
+                                   a.next + ((uint64_t)k * a.K + m - 1) * a.F)
+                             : nullptr;
+    for (uint32_t u0 = w_lo + lane; u0 < w_hi; u0 += 32 * UN) {
+      uint32_t v[UN];
+#pragma unroll
+      for (int u = 0; u < UN; ++u) {
+        const uint32_t w = u0 + u * 32;
+        v[u] = (load && w < w_hi) ? ld_stream(src + w, pol) : 0u;
+      }
+#pragma unroll
+      for (int u = 0; u < UN; ++u) {
+        const uint32_t w = u0 + u * 32;
+        if (w >= w_hi) continue;
+        float4 fv;
+        fv.x = unit_f32(byte_f(v[u], 0), c.r1, c.r2);
+        fv.y = unit_f32(byte_f(v[u], 1), c.r1, c.r2);
+        fv.z = unit_f32(byte_f(v[u], 2), c.r1, c.r2);
+        fv.w = unit_f32(byte_f(v[u], 3), c.r1, c.r2);
+        if (dobs) st_stream(dobs + w, zo ? zero4 : fv, pol);
+        if (dnext) st_stream(dnext + w, zn ? zero4 : fv, pol);
+      }
+    }
+    f = seg_end;
+  }
 }
-// shared memory: barriers | control | kStages input parts | kStages fp32
-// tiles | one zero tile
-__host__ __device__ inline size_t stack_smem(uint32_t part) {
-  return 128 + align_up(kCtlUnits * sizeof(UnitCtl), 128) +
-         align_up((size_t)kStages * part, 128) + (size_t)kStages * part * 4 +
-         (size_t)part * 4;
-}
 
+template <int UN>
 __global__ void __launch_bounds__(kThreads)
 k_deliver_stack(Common c, StackArgs a) {
-  extern __shared__ __align__(128) uint8_t sm[];
-  uint64_t *bar = reinterpret_cast<uint64_t *>(sm);
-  UnitCtl *ctl = reinterpret_cast<UnitCtl *>(sm + 128);
-  uint8_t *in = sm + 128 + align_up(kCtlUnits * sizeof(UnitCtl), 128);
-  float *tile = reinterpret_cast<float *>(in + align_up((size_t)kStages * a.part, 128));
-  float *zero = tile + (size_t)kStages * a.part;
-  __shared__ int s_abort;  // a bounded wait expired: stop the pipeline
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  __shared__ uint32_t s_chunk;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const uint64_t pol = policy_stream();
-  if (tid == 0) {
-    for (int i = 0; i < kStages; ++i) mbar_init(&bar[i], 1);
-    fence_mbar_init();
-    s_abort = 0;
-  }
-  for (uint32_t i = tid; i < a.part; i += kThreads) zero[i] = 0.f;
   pdl_wait();
   pdl_launch();
-  fence_proxy_async();
-  __syncthreads();
-
-  const uint64_t total = (uint64_t)c.B * a.U * a.P;
-  const uint64_t per = (total + gridDim.x - 1) / gridDim.x;
-  const uint64_t u0 = (uint64_t)blockIdx.x * per;
-  const uint64_t u1 = min(total, u0 + per);
-  uint32_t it = 0;  // pipeline position across control batches
-  for (uint64_t ub = u0; ub < u1; ub += kCtlUnits) {
-    const uint32_t nu = (uint32_t)min((uint64_t)kCtlUnits, u1 - ub);
-    // ---- control, one thread per unit
-    for (uint32_t t = tid; t < nu; t += kThreads) {
-      const uint64_t u = ub + t;
-      const uint32_t k = (uint32_t)(u / (a.U * a.P));
-      const uint32_t rem = (uint32_t)(u % (a.U * a.P));
-      const uint32_t m = rem / a.P, p = rem % a.P;
-      uint64_t slot = 0, off = 0;
-      const bool ok = sample_slot(c, k, &slot, &off, m == 0 && p == 0);
-      const int64_t j = (int64_t)off - (int64_t)(a.K - 1) + (int64_t)m;
-      // an episode end at offsets [j, off - 1] zeroes the frame in obs,
-      // one at [j, off] in next_obs
-      bool end_before = false, end_at = false;
-      if (ok && j >= 0) {
-        for (int64_t o = j; o <= (int64_t)off; ++o) {
-          const uint64_t t2 = c.oldest + (uint64_t)o;
-          const bool d = c.done[t2 >= c.cap ? t2 - c.cap : t2] != 0;
-          if (o < (int64_t)off) end_before |= d; else end_at = d;
-        }
-      }
-      const bool has_obs = m < a.K;
-      const bool has_next = a.next && m >= 1;
-      const bool zo = !ok || j < 0 || end_before;
-      const bool zn = !ok || j < 0 || end_before || end_at;
-      UnitCtl e;
-      e.bytes = p + 1 < a.P ? a.part : a.F - (a.P - 1) * a.part;
-      const uint64_t js = c.oldest + (uint64_t)(j < 0 ? 0 : j);
-      e.src = (js >= c.cap ? js - c.cap : js) * a.F + (uint64_t)p * a.part;
-      e.dobs = has_obs ? ((uint64_t)k * a.K + m) * a.F + (uint64_t)p * a.part : ~0ull;
-      e.dnext = has_next ? ((uint64_t)k * a.K + m - 1) * a.F + (uint64_t)p * a.part : ~0ull;
-      e.flags = ((has_obs && !zo) || (has_next && !zn) ? kLoad : 0u) |
-                (zo ? kZeroObs : 0u) | (zn ? kZeroNext : 0u);
-      ctl[t] = e;
-    }
-    __syncthreads();
-    // ---- bulk loads of the first kStages - 1 units
-    if (tid == 0)
-      for (uint32_t i = 0; i + 1 < kStages && i < nu; ++i) {
-        const UnitCtl &e = ctl[i];
-        const uint32_t st = (it + i) % kStages;
-        if (e.flags & kLoad) {
-          mbar_expect_tx(&bar[st], e.bytes);
-          tma_load(in + (size_t)st * a.part, a.frames + e.src, e.bytes, &bar[st], pol);
-        } else {
-          mbar_expect_tx(&bar[st], 0);
-        }
-      }
-    // ---- collate of the samples whose head unit is in this batch
-    for (uint32_t t = warp; t < nu; t += kWarps) {
-      const uint64_t u = ub + t;
-      if (u % ((uint64_t)a.U * a.P) != 0) continue;
-      const uint32_t k = (uint32_t)(u / (a.U * a.P));
-      uint64_t slot = 0, off = 0;
-      const bool ok = sample_slot(c, k, &slot, &off, false);
-      collate(c, k, ok, slot, off, lane);
-    }
-    // ---- pipeline
-    for (uint32_t i = 0; i < nu; ++i, ++it) {
-      const uint32_t st = it % kStages;
-      if (tid == 0 && i + kStages - 1 < nu) {
-        const UnitCtl &e = ctl[i + kStages - 1];
-        const uint32_t sn = (it + kStages - 1) % kStages;
-        if (e.flags & kLoad) {
-          mbar_expect_tx(&bar[sn], e.bytes);
-          tma_load(in + (size_t)sn * a.part, a.frames + e.src, e.bytes, &bar[sn], pol);
-        } else {
-          mbar_expect_tx(&bar[sn], 0);
-        }
-      }
-      const UnitCtl e = ctl[i];
-      if (!mbar_wait(&bar[st], (it / kStages) & 1u, c.ctrl)) s_abort = 1;
-      if (tid == 0) tma_wait_read<kStages - 1>();  // tile st is free again
-      __syncthreads();
-      if (s_abort) break;
-      float4 *tl = reinterpret_cast<float4 *>(tile + (size_t)st * a.part);
-      if (e.flags & kLoad) {
-        const uint32_t *src = reinterpret_cast<const uint32_t *>(in + (size_t)st * a.part);
-        for (uint32_t w = tid; w < e.bytes / 4; w += kThreads) {
-          const uint32_t v = src[w];
-          float4 fv;
-          fv.x = unit_f32(byte_f(v, 0), c.r1, c.r2);
-          fv.y = unit_f32(byte_f(v, 1), c.r1, c.r2);
-          fv.z = unit_f32(byte_f(v, 2), c.r1, c.r2);
-          fv.w = unit_f32(byte_f(v, 3), c.r1, c.r2);
-          tl[w] = fv;
-        }
-      }
-      fence_proxy_async();
-      __syncthreads();
-      if (tid == 0) {
-        if (e.dobs != ~0ull)
-          tma_store(a.obs + e.dobs, (e.flags & kZeroObs) ? zero : (float *)tl,
-                    e.bytes * 4, pol);
-        if (e.dnext != ~0ull)
-          tma_store(a.next + e.dnext, (e.flags & kZeroNext) ? zero : (float *)tl,
-                    e.bytes * 4, pol);
-        tma_commit();
-      }
-    }
-    __syncthreads();  // the control table is rewritten by the next batch
-    if (s_abort) break;
+  const uint64_t total = (uint64_t)c.B * a.U * a.W;
+  const uint64_t per_chunk = (uint64_t)kWarps * a.span;
+  if (!c.work) {  // one chunk per CTA
+    const uint64_t f = (uint64_t)blockIdx.x * per_chunk + (uint64_t)warp * a.span;
+    if (f < total) stack_span<UN>(c, a, f, min(total, f + a.span), lane, pol);
+    return;
   }
-  if (tid == 0) tma_wait_all();
+  for (;;) {
+    if (threadIdx.x == 0) s_chunk = atomicAdd(&c.work[0], 1u);
+    __syncthreads();
+    const uint64_t f0 = (uint64_t)s_chunk * per_chunk;
+    __syncthreads();  // s_chunk is rewritten by the next grab
+    if (f0 >= total) break;  // uniform across the CTA
+    const uint64_t f = f0 + (uint64_t)warp * a.span;
+    if (f < total) stack_span<UN>(c, a, f, min(total, f + a.span), lane, pol);
+  }
+  // every CTA has made its last grab: the last to retire resets the pair
+  if (threadIdx.x == 0 && atomicAdd(&c.work[1], 1u) == gridDim.x - 1) {
+    c.work[0] = 0u;
+    c.work[1] = 0u;
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -491,21 +440,34 @@ k_deliver_norm(Common c, NormArgs a) {
   }
 }
 
-// One wave of persistent CTAs: blocks resident per SM x SMs (queried once
-// per kernel), never more CTAs than there are 32-unit rows of work.
+// Grid size from the work: enough CTAs that each warp runs about `iters`
+// iterations of its unrolled loop (`per_iter` units each), so the block
+// scheduler balances the tail and a CTA that starts late (its SM still busy
+// with another kernel) holds up little work; a small batch is spread over up
+// to one wave (blocks resident per SM x SMs, queried once per kernel) with
+// at least one iteration per warp.
 template <typename Kern>
-unsigned one_wave(Kern kern, uint64_t total_units, int sms) {
+unsigned grid_for(Kern kern, uint64_t units, uint64_t per_iter, int iters, int sms) {
   static int per_sm = 0;  // per template instantiation
   if (!per_sm) {
     cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, 0);
     if (per_sm < 1) per_sm = 1;
   }
-  const uint64_t rows = (total_units + 31) / 32;
-  uint64_t blocks = (uint64_t)per_sm * sms;
-  const uint64_t need = (rows + kWarps - 1) / kWarps;
-  if (blocks > need) blocks = need;
+  const uint64_t wave = (uint64_t)per_sm * sms;
+  const uint64_t warp_iters = (units + per_iter - 1) / per_iter;
+  uint64_t blocks = (warp_iters + (uint64_t)kWarps * iters - 1) / ((uint64_t)kWarps * iters);
+  if (blocks < wave) {
+    const uint64_t most = (warp_iters + kWarps - 1) / kWarps;
+    blocks = most < wave ? most : wave;
+  }
   return (unsigned)(blocks ? blocks : 1);
 }
+
+// unrolled rows per warp iteration and iterations per warp (chunk span) of
+// each kernel; CTA slots per SM the frame-stack delivery leaves free
+constexpr int kStackUnroll = 4, kStackIters = 3, kStackHeadroom = 2;
+constexpr int kHwcUnroll = 2, kHwcIters = 2;
+constexpr int kNormIters = 3;
 
 }  // namespace
 
@@ -540,57 +502,63 @@ cudaError_t launch_deliver(edp_ctx *ctx, const int64_t *idx, uint32_t B,
     StackArgs a{};
     a.frames = ctx->st.obs;
     a.F = (uint32_t)ctx->obs_bytes;
+    a.W = a.F / 4;
     a.K = cfg.frame_stack;
     a.obs = (float *)out->obs;
     a.next = (float *)out->next_obs;
     a.U = a.K + (a.next ? 1 : 0);
-    // parts of at most ~2.4 KB, each a multiple of 16 bytes
-    a.P = (a.F + 2399) / 2400;
-    a.part = (uint32_t)(((a.F / 16) + a.P - 1) / a.P * 16);
-    a.P = (a.F + a.part - 1) / a.part;
-    const size_t smem = stack_smem(a.part);
+    const uint64_t units = (uint64_t)B * a.U * a.W;
+    auto kern = k_deliver_stack<kStackUnroll>;
     static int per_sm = 0;
-    static size_t smem_set = 0;
-    if (smem_set != smem) {
-      cudaFuncSetAttribute(k_deliver_stack, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           (int)smem);
-      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_deliver_stack, kThreads, smem);
+    if (!per_sm) {
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, 0);
       if (per_sm < 1) per_sm = 1;
-      smem_set = smem;
     }
-    const uint64_t units = (uint64_t)B * a.U * a.P;
-    uint64_t grid = (uint64_t)per_sm * sms;
-    if (grid > units) grid = units;
-    cudaLaunchConfig_t lc = {};
-    lc.gridDim = dim3((unsigned)grid);
-    lc.blockDim = dim3(kThreads);
-    lc.dynamicSmemBytes = smem;
-    lc.stream = s;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    lc.attrs = attr;
-    lc.numAttrs = 1;
-    return cudaLaunchKernelEx(&lc, k_deliver_stack, c, a);
+    const int resident = per_sm > kStackHeadroom ? per_sm - kStackHeadroom : 1;
+    uint64_t grid = (uint64_t)resident * sms;
+    auto n_chunks = [&](uint32_t span) {
+      return (units + (uint64_t)kWarps * span - 1) / ((uint64_t)kWarps * span);
+    };
+    a.span = 32 * kStackUnroll * kStackIters;
+    uint64_t chunks = n_chunks(a.span);
+    if (chunks < grid) {  // a small batch: one iteration per warp, more CTAs
+      a.span = 32 * kStackUnroll;
+      chunks = n_chunks(a.span);
+    }
+    if (grid >= chunks) {
+      grid = chunks;  // one chunk per CTA, no work counter
+    } else {
+      c.work = ctx->ctrl->work + 2 * (ctx->work_seq++ % kWorkSlots);
+    }
+    return launch_pdl(kern, dim3((unsigned)grid), dim3(kThreads), s, c, a);
   } else if (cfg.transform == EDP_XFORM_HWC_CHW_BF16) {
     ChwArgs a{};
     a.obs = ctx->st.obs;
     a.HW = cfg.obs_h * cfg.obs_w;
     a.out = (__nv_bfloat16 *)out->obs;
     const uint64_t units = (uint64_t)B * (a.HW / 8);
+    constexpr uint64_t it = 32 * kHwcUnroll;
     switch (cfg.obs_c) {
-      case 1:
-        return launch_pdl(k_deliver_hwc<1, 2>, dim3(one_wave(k_deliver_hwc<1, 2>, units, sms)),
+      case 1: {
+        auto kern = k_deliver_hwc<1, kHwcUnroll>;
+        return launch_pdl(kern, dim3(grid_for(kern, units, it, kHwcIters, sms)),
                           dim3(kThreads), s, c, a);
-      case 2:
-        return launch_pdl(k_deliver_hwc<2, 2>, dim3(one_wave(k_deliver_hwc<2, 2>, units, sms)),
+      }
+      case 2: {
+        auto kern = k_deliver_hwc<2, kHwcUnroll>;
+        return launch_pdl(kern, dim3(grid_for(kern, units, it, kHwcIters, sms)),
                           dim3(kThreads), s, c, a);
-      case 3:
-        return launch_pdl(k_deliver_hwc<3, 2>, dim3(one_wave(k_deliver_hwc<3, 2>, units, sms)),
+      }
+      case 3: {
+        auto kern = k_deliver_hwc<3, kHwcUnroll>;
+        return launch_pdl(kern, dim3(grid_for(kern, units, it, kHwcIters, sms)),
                           dim3(kThreads), s, c, a);
-      default:
-        return launch_pdl(k_deliver_hwc<4, 2>, dim3(one_wave(k_deliver_hwc<4, 2>, units, sms)),
+      }
+      default: {
+        auto kern = k_deliver_hwc<4, kHwcUnroll>;
+        return launch_pdl(kern, dim3(grid_for(kern, units, it, kHwcIters, sms)),
                           dim3(kThreads), s, c, a);
+      }
     }
   } else {
     NormArgs a{};
@@ -615,8 +583,8 @@ cudaError_t launch_deliver(edp_ctx *ctx, const int64_t *idx, uint32_t B,
     a.out = (__nv_bfloat16 *)out->obs;
     a.tok_out = out->tokens;
     const uint64_t units = (uint64_t)B * a.F8;
-    return launch_pdl(k_deliver_norm<kNormUnroll>,
-                      dim3(one_wave(k_deliver_norm<kNormUnroll>, units, sms)),
+    auto kern = k_deliver_norm<kNormUnroll>;
+    return launch_pdl(kern, dim3(grid_for(kern, units, 32 * kNormUnroll, kNormIters, sms)),
                       dim3(kThreads), s, c, a);
   }
   return cudaGetLastError();

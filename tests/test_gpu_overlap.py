@@ -3,7 +3,8 @@
 A round of prioritized replay is sample -> deliver -> priority update.  The
 delivery depends only on the sampled indices, so it may run on a second
 stream while the update and the next round's sampling run on the first (the
-overlapped timing of Sec. 6.1).  With the dependencies kept -- delivery r
+overlapped timing of Sec. 6.1); with two side streams consecutive deliveries
+may also overlap each other.  With the dependencies kept -- delivery r
 after sampling r, sampling r+1 after update r, and sampling r+R after
 delivery r has read the R-th previous index set -- every sampled index, every
 delivered batch and the final priority tree must equal, bit for bit, those of
@@ -38,7 +39,7 @@ class _Rounds:
             idx_copy = torch.zeros(B, dtype=torch.int64, device=dev)
             self.out.append((obs, nxt, act, rew, dn, isw, idx_copy))
         self.td = [torch.from_numpy(fx.td_errors(31, B, r)).cuda() for r in range(ROUNDS)]
-        self.side = torch.cuda.Stream()
+        self.sides = [torch.cuda.Stream(), torch.cuda.Stream()]
         self.ready = [torch.cuda.Event() for _ in range(R)]
         self.consumed = [torch.cuda.Event() for _ in range(R)]
 
@@ -77,7 +78,7 @@ class _Rounds:
             self._deliver(r)
             self._update(r)
 
-    def overlapped(self):
+    def overlapped(self, nsides):
         main = torch.cuda.current_stream()
         for r in range(ROUNDS):
             k = r % R
@@ -85,12 +86,14 @@ class _Rounds:
                 main.wait_event(self.consumed[k])
             self._sample(r)
             self.ready[k].record()
-            with torch.cuda.stream(self.side):
-                self.side.wait_event(self.ready[k])
-                self._deliver(r, stream=self.side)
+            side = self.sides[r % nsides]  # consecutive deliveries may overlap
+            with torch.cuda.stream(side):
+                side.wait_event(self.ready[k])
+                self._deliver(r, stream=side)
                 self.consumed[k].record()
             self._update(r)
-        main.wait_stream(self.side)
+        for side in self.sides[:nsides]:
+            main.wait_stream(side)
 
     def results(self):
         self.edp.edp_sync(self.m.ring.ctx)
@@ -101,7 +104,8 @@ class _Rounds:
         return per_round, (leaves, lv, pending, qmax)
 
 
-def test_overlapped_rounds_equal_serial_rounds(edp_lib, orc):
+@pytest.mark.parametrize("nsides", [1, 2])
+def test_overlapped_rounds_equal_serial_rounds(edp_lib, orc, nsides):
     edp = edp_lib
     frames, action, reward, done = fx.dqn_transitions(30, N_INGEST, F)
     q = orc.priorities_from_td(fx.td_errors(30, N_INGEST), ALPHA, EPS)
@@ -110,11 +114,11 @@ def test_overlapped_rounds_equal_serial_rounds(edp_lib, orc):
         run.warm()
     torch.cuda.synchronize()
     runs[0].serial()
-    runs[1].overlapped()
+    runs[1].overlapped(nsides)
     g = torch.cuda.CUDAGraph()
     torch.cuda.synchronize()
     with torch.cuda.graph(g, capture_error_mode="thread_local"):
-        runs[2].overlapped()
+        runs[2].overlapped(nsides)
     g.replay()
     ref_rounds, ref_tree = runs[0].results()
     # the rounds did change the tree and sampled more than one index set

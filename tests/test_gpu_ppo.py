@@ -158,3 +158,56 @@ def test_hwc_chw_channels(edp_lib, orc, C):
     dummy = np.zeros(cap, np.float32)
     ref, _, _ = orc.deliver_ppo(o_ring, cap, cap + 13, H, W, C, ref_idx, dummy, dummy)
     assert np.array_equal(bits(out), ref)
+
+
+def test_ppo_iteration_in_one_call(edp_lib, orc):
+    """The whole iteration delivered by one call (granularity g_del = 1),
+    with GAE on a second stream beside the shuffle: mini-batch m is rows
+    [4096 m, 4096 (m + 1)) of the output and equals, bit for bit, what the
+    m-th per-mini-batch call delivers; strided rows equal the oracle."""
+    edp = edp_lib
+    T, E, H, W, C = 128, 256, 64, 64, 3
+    n, M = T * E, 8
+    mb = n // M
+    obs, r, v, d = fx.ppo_rollout(3, T, E)
+    ring = _ppo_ring(edp, n)
+    edp.edp_ingest(ring.ctx, cuda(obs), n)
+    dr, dv, dd = cuda(r), cuda(v), cuda(d)
+    adv = torch.empty((T, E), device="cuda")
+    ret = torch.empty((T, E), device="cuda")
+    nrm = torch.empty((T, E), device="cuda")
+    idx = torch.empty(n, dtype=torch.int64, device="cuda")
+    side = torch.cuda.Stream()
+    fork, gae_done = torch.cuda.Event(), torch.cuda.Event()
+    torch.cuda.synchronize()
+    fork.record()
+    with torch.cuda.stream(side):
+        side.wait_event(fork)
+        edp.edp_gae(ring.ctx, dr, dv, dd, T, E, G, LAM, adv, ret, nrm, stream=side)
+        gae_done.record()
+    edp.edp_sample(ring.ctx, edp.EDP_SAMPLE_PERMUTE, n, 3, 1, idx)
+    torch.cuda.current_stream().wait_event(gae_done)
+    out = torch.full((n, C, H, W), float("nan"), dtype=torch.bfloat16, device="cuda")
+    a_all = torch.full((n,), float("nan"), device="cuda")
+    r_all = torch.full((n,), float("nan"), device="cuda")
+    nrm_flat, ret_flat = nrm.view(-1), ret.view(-1)
+    edp.edp_deliver(ring.ctx, idx, n, edp.make_batch(
+        out, gather=[(nrm_flat, a_all), (ret_flat, r_all)]))
+    edp.edp_sync(ring.ctx)
+    perm = orc.permutation(n, 3, 1)
+    assert np.array_equal(to_np(idx), perm)
+    ra, rr = orc.gae(r, v, d, G, LAM)
+    rn, _, _ = orc.normalize(ra.ravel())
+    assert np.abs(to_np(nrm).ravel() - rn).max() <= 1e-5
+    assert np.array_equal(bits(a_all), bits(nrm_flat)[perm])
+    assert np.array_equal(bits(r_all), bits(ret_flat)[perm])
+    full = bits(out)
+    for m in (0, 3, M - 1):
+        o = torch.empty((mb, C, H, W), dtype=torch.bfloat16, device="cuda")
+        edp.edp_deliver(ring.ctx, idx[m * mb:(m + 1) * mb], mb, edp.make_batch(o))
+        edp.edp_sync(ring.ctx)
+        assert np.array_equal(bits(o), full[m * mb:(m + 1) * mb])
+    s = np.arange(0, n, 61)
+    ref, _, _ = orc.deliver_ppo(obs, n, n, H, W, C, perm[s], rn.astype(np.float32),
+                                rr.ravel().astype(np.float32))
+    assert np.array_equal(full[s], ref)
