@@ -1110,7 +1110,7 @@ def run_edp(args):
 
     use_graph = not args.no_graph
     others = []
-    for name, fn, desc in scheds[1:]:
+    for name, fn, desc in ([] if args.no_other_schedules else scheds[1:]):
         ms_o, _ = timed(fn)
         others.append({"schedule": name, "value": job_gbs(wl.round_bytes, K, world, ms_o),
                        "ms_per_step": ms_o / K, "description": desc})
@@ -1203,6 +1203,8 @@ def main():
     ap.add_argument("--capacity", type=int, default=0,
                     help="override the ring capacity (profiling small cases)")
     ap.add_argument("--no-graph", action="store_true")
+    ap.add_argument("--no-other-schedules", action="store_true",
+                    help="time only the main schedule")
     ap.add_argument("--schedule", default="",
                     help="the workload's schedule timed as the main number "
                          "(default: its first); the others are reported too")

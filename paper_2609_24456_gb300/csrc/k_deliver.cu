@@ -32,6 +32,13 @@ constexpr int kWarps = kThreads / 32;
 // loads in flight per lane (8 x 8 bytes) in the normalising delivery
 constexpr int kNormUnroll = 8;
 
+// unrolled rows per warp iteration and iterations per warp (chunk span) of
+// each kernel; CTA slots per SM the frame-stack delivery leaves free
+constexpr int kStackUnroll = 4, kStackIters = 3, kStackHeadroom = 2;
+constexpr int kStackMinBlocks = 6;  // __launch_bounds__: at most 40 registers
+constexpr int kHwcUnroll = 2, kHwcIters = 2;
+constexpr int kNormIters = 3;
+
 struct Common {
   const int64_t *idx;
   uint32_t B;
@@ -242,9 +249,9 @@ __device__ __forceinline__ void stack_span(const Common &c, const StackArgs &a,
 }
 
 template <int UN>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kThreads, kStackMinBlocks)
 k_deliver_stack(Common c, StackArgs a) {
-  __shared__ uint32_t s_chunk;
+  __shared__ uint32_t s_chunk[2];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const uint64_t pol = policy_stream();
   pdl_wait();
@@ -256,14 +263,22 @@ k_deliver_stack(Common c, StackArgs a) {
     if (f < total) stack_span<UN>(c, a, f, min(total, f + a.span), lane, pol);
     return;
   }
-  for (;;) {
-    if (threadIdx.x == 0) s_chunk = atomicAdd(&c.work[0], 1u);
-    __syncthreads();
-    const uint64_t f0 = (uint64_t)s_chunk * per_chunk;
-    __syncthreads();  // s_chunk is rewritten by the next grab
+  // Thread 0 grabs the next chunk while the CTA works on the current one
+  // and publishes it in the other half of s_chunk before the one barrier
+  // per chunk; the half it overwrites was read before the previous barrier.
+  if (threadIdx.x == 0) s_chunk[0] = atomicAdd(&c.work[0], 1u);
+  __syncthreads();
+  uint32_t cur = s_chunk[0];
+  for (int p = 1;; p ^= 1) {
+    const uint64_t f0 = (uint64_t)cur * per_chunk;
     if (f0 >= total) break;  // uniform across the CTA
+    uint32_t nxt = 0;
+    if (threadIdx.x == 0) nxt = atomicAdd(&c.work[0], 1u);
     const uint64_t f = f0 + (uint64_t)warp * a.span;
     if (f < total) stack_span<UN>(c, a, f, min(total, f + a.span), lane, pol);
+    if (threadIdx.x == 0) s_chunk[p] = nxt;
+    __syncthreads();
+    cur = s_chunk[p];
   }
   // every CTA has made its last grab: the last to retire resets the pair
   if (threadIdx.x == 0 && atomicAdd(&c.work[1], 1u) == gridDim.x - 1) {
@@ -462,12 +477,6 @@ unsigned grid_for(Kern kern, uint64_t units, uint64_t per_iter, int iters, int s
   }
   return (unsigned)(blocks ? blocks : 1);
 }
-
-// unrolled rows per warp iteration and iterations per warp (chunk span) of
-// each kernel; CTA slots per SM the frame-stack delivery leaves free
-constexpr int kStackUnroll = 4, kStackIters = 3, kStackHeadroom = 2;
-constexpr int kHwcUnroll = 2, kHwcIters = 2;
-constexpr int kNormIters = 3;
 
 }  // namespace
 
