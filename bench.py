@@ -807,7 +807,7 @@ class MmReplay(Workload):
         self.demote_bytes = ingest * 2 * (self.F + 4 * self.L)
         self.round_bytes = self.deliver_bytes + batch * 8 + self.ingest_bytes + \
             (self.demote_bytes if self.tiered else 0)
-        self.launches_per_round = 2 + (5 if ingest else 0)
+        self.launches_per_round = 2 + (3 if ingest else 0)  # + swap obs, swap tokens, metadata
 
     def config(self):
         c = {"workload": self.name, "capacity": self.cap, "batch": self.B,

@@ -424,28 +424,43 @@ edp_status edp_ingest(edp_ctx *ctx, const edp_fields *src, uint64_t n,
   const uint64_t keep_h = Tn < ctx->cap_h ? Tn : ctx->cap_h;
   const uint64_t keep = Tn < ctx->cap ? Tn : ctx->cap;
   uint64_t new_hbm_lo = T;
+  bool swapped = false;
   if (ctx->cap_c) {
     const uint64_t in_hbm = T < ctx->cap_h ? T : ctx->cap_h;
     uint64_t lo = T - in_hbm;
     if (lo < Tn - keep) lo = Tn - keep;  // evicted outright
     const uint64_t hi = (Tn - keep_h) < T ? (Tn - keep_h) : T;
-    if (hi > lo) e = launch_demote(ctx, lo, hi - lo, s);
     // new ids [max(T, Tn - keep), Tn - keep_h) -> host tier directly
     const uint64_t dlo = T > Tn - keep ? T : Tn - keep;
     const uint64_t dhi = Tn - keep_h;
-    if (e == cudaSuccess && dhi > dlo)
-      e = launch_copy_rows_to_host(ctx, f.obs, f.tokens, dlo - T, dlo, dhi - dlo, s);
-    if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_ingest(host tier)");
     if (new_hbm_lo < Tn - keep_h) new_hbm_lo = Tn - keep_h;
+    // steady state: every new id takes the HBM slot of the id it demotes
+    // (id L leaves, id L + cap_h arrives) -> one fused pass, both link
+    // directions at once
+    swapped = hi > lo && dhi <= dlo && hi - lo == Tn - new_hbm_lo &&
+              lo + ctx->cap_h == new_hbm_lo;
+    if (swapped) {
+      const uint64_t skip = new_hbm_lo - T;
+      e = launch_swap(ctx, lo, f.obs + skip * ctx->obs_bytes,
+                      f.tokens ? f.tokens + skip * (ctx->tok_bytes / 4) : nullptr,
+                      hi - lo, s);
+    } else {
+      if (hi > lo) e = launch_demote(ctx, lo, hi - lo, s);
+      if (e == cudaSuccess && dhi > dlo)
+        e = launch_copy_rows_to_host(ctx, f.obs, f.tokens, dlo - T, dlo, dhi - dlo, s);
+    }
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_ingest(host tier)");
   }
   const uint64_t skip = new_hbm_lo - T, nh = Tn - new_hbm_lo;
-  e = launch_copy_rows(ctx->st.obs, ctx->cap_h, new_hbm_lo % ctx->cap_h,
-                       f.obs + skip * ctx->obs_bytes, nh, ctx->obs_bytes, s);
-  if (e == cudaSuccess && ctx->tok_bytes)
-    e = launch_copy_rows((uint8_t *)ctx->st.tokens, ctx->cap_h,
-                         new_hbm_lo % ctx->cap_h,
-                         (const uint8_t *)f.tokens + skip * ctx->tok_bytes, nh,
-                         ctx->tok_bytes, s);
+  if (!swapped) {
+    e = launch_copy_rows(ctx->st.obs, ctx->cap_h, new_hbm_lo % ctx->cap_h,
+                         f.obs + skip * ctx->obs_bytes, nh, ctx->obs_bytes, s);
+    if (e == cudaSuccess && ctx->tok_bytes)
+      e = launch_copy_rows((uint8_t *)ctx->st.tokens, ctx->cap_h,
+                           new_hbm_lo % ctx->cap_h,
+                           (const uint8_t *)f.tokens + skip * ctx->tok_bytes, nh,
+                           ctx->tok_bytes, s);
+  }
   if (e == cudaSuccess) e = launch_ingest_meta(ctx, &f, n, q, s);
   if (e == cudaSuccess && ctx->depth) {
     uint64_t first = ctx->total % ctx->cap, count = n;

@@ -300,6 +300,12 @@ cudaError_t launch_ingest_meta(edp_ctx *ctx, const edp_fields *src, uint64_t n,
                                const uint32_t *q, cudaStream_t s);
 cudaError_t launch_demote(edp_ctx *ctx, uint64_t first_id, uint64_t n,
                           cudaStream_t s);
+// Demotion and insertion fused, for the steady state of a full two-tier
+// ring: ids first_id + j leave HBM slot (first_id + j) mod cap_h for host
+// slot (first_id + j) mod cap_c while source rows j of the ingest (obs,
+// tokens) take their HBM slot.
+cudaError_t launch_swap(edp_ctx *ctx, uint64_t first_id, const uint8_t *obs,
+                        const int32_t *tokens, uint64_t n, cudaStream_t s);
 // rows [src_row, src_row + n) of an ingest source -> host-tier slots of ids
 // first_id .. first_id + n - 1
 cudaError_t launch_copy_rows_to_host(edp_ctx *ctx, const uint8_t *obs,

@@ -45,6 +45,58 @@ k_copy_rows(uint8_t *__restrict__ dst, uint64_t dst_cap, uint64_t dst_first,
   }
 }
 
+// Swap rows through HBM: HBM row (first + j) mod hbm_cap moves to host row
+// (first + j) mod host_cap and source row j takes its place.  One thread
+// handles one 16-byte chunk in all three rows, reading the old HBM value
+// before writing the new one, so no other thread's order matters.  The
+// host-link traffic goes both ways at once (source rows in, demoted rows
+// out), which a demotion followed by a copy would serialise.
+__global__ void __launch_bounds__(kCopyThreads)
+k_swap_rows(uint8_t *__restrict__ hbm, uint64_t hbm_cap, uint8_t *__restrict__ host,
+            uint64_t host_cap, const uint8_t *__restrict__ src, uint64_t first,
+            uint64_t n, uint32_t cpr) {
+  const uint64_t row_bytes = (uint64_t)cpr * 16u;
+  for (uint64_t j = blockIdx.y; j < n; j += gridDim.y) {
+    uint4 *h = reinterpret_cast<uint4 *>(hbm + ((first + j) % hbm_cap) * row_bytes);
+    uint4 *c = reinterpret_cast<uint4 *>(host + ((first + j) % host_cap) * row_bytes);
+    const uint4 *s = reinterpret_cast<const uint4 *>(src + j * row_bytes);
+    const uint32_t step = gridDim.x * kCopyThreads * kCopyUnroll;
+    for (uint32_t w0 = blockIdx.x * kCopyThreads * kCopyUnroll + threadIdx.x;
+         w0 < cpr; w0 += step) {
+      uint4 old_[kCopyUnroll], new_[kCopyUnroll];
+#pragma unroll
+      for (int u = 0; u < kCopyUnroll; ++u) {
+        const uint32_t w = w0 + u * kCopyThreads;
+        if (w < cpr) {
+          old_[u] = h[w];
+          new_[u] = s[w];
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < kCopyUnroll; ++u) {
+        const uint32_t w = w0 + u * kCopyThreads;
+        if (w < cpr) {
+          c[w] = old_[u];
+          h[w] = new_[u];
+        }
+      }
+    }
+  }
+}
+
+cudaError_t swap_rows(uint8_t *hbm, uint64_t hbm_cap, uint8_t *host, uint64_t host_cap,
+                      const uint8_t *src, uint64_t first, uint64_t n,
+                      uint64_t row_bytes, cudaStream_t s) {
+  if (!n) return cudaSuccess;
+  const uint32_t cpr = (uint32_t)(row_bytes / 16);
+  uint32_t gx = (cpr + kCopyThreads * kCopyUnroll - 1) / (kCopyThreads * kCopyUnroll);
+  if (gx > 64) gx = 64;
+  const uint32_t gy = n < 65535 ? (uint32_t)n : 65535u;
+  k_swap_rows<<<dim3(gx, gy), kCopyThreads, 0, s>>>(hbm, hbm_cap, host, host_cap, src,
+                                                   first, n, cpr);
+  return cudaGetLastError();
+}
+
 cudaError_t copy_rows(uint8_t *dst, uint64_t dst_cap, uint64_t dst_first,
                       const uint8_t *src, uint64_t src_cap, uint64_t src_first,
                       uint64_t n, uint64_t row_bytes, cudaStream_t s) {
@@ -165,6 +217,16 @@ cudaError_t launch_demote(edp_ctx *c, uint64_t first_id, uint64_t n,
     e = copy_rows((uint8_t *)c->st.host_tokens, c->cap_c, first_id % c->cap_c,
                   (const uint8_t *)c->st.tokens, c->cap_h, first_id % c->cap_h,
                   n, c->tok_bytes, s);
+  return e;
+}
+
+cudaError_t launch_swap(edp_ctx *c, uint64_t first_id, const uint8_t *obs,
+                        const int32_t *tokens, uint64_t n, cudaStream_t s) {
+  cudaError_t e = swap_rows(c->st.obs, c->cap_h, c->st.host_obs, c->cap_c, obs,
+                            first_id, n, c->obs_bytes, s);
+  if (e == cudaSuccess && c->tok_bytes)
+    e = swap_rows((uint8_t *)c->st.tokens, c->cap_h, (uint8_t *)c->st.host_tokens,
+                  c->cap_c, (const uint8_t *)tokens, first_id, n, c->tok_bytes, s);
   return e;
 }
 
