@@ -42,10 +42,13 @@
  *   edp_sample, edp_update_priorities*, edp_priorities_from_td, edp_gae and
  *   other deliveries of the same context, once the sampling that wrote its
  *   `idx` has completed (an event) and while nothing overwrites `idx`, `q`
- *   or the rows it reads (edp_ingest).  edp_gae likewise may overlap
- *   edp_sample (GAE scratch and shuffle scratch are separate).  Every other
- *   pair of calls on one context shares the priority tree or the context's
- *   scratch and must be ordered.
+ *   or the rows it reads (edp_ingest).  A large frame-stack delivery takes
+ *   one of 32 work counters of its context, round robin in issue order (for
+ *   a captured graph, the order at capture): deliveries that run at the
+ *   same time must have been issued fewer than 32 deliveries apart.
+ *   edp_gae likewise may overlap edp_sample (GAE scratch and shuffle
+ *   scratch are separate).  Every other pair of calls on one context shares
+ *   the priority tree or the context's scratch and must be ordered.
  * - Errors: argument and state errors are returned synchronously and leave
  *   the context unchanged.  A CUDA launch error returns EDP_ERR_CUDA.
  *   Data-dependent faults found on the device (an index out of range, an

@@ -1,0 +1,71 @@
+"""The work-counter path of the frame-stack delivery.
+
+A batch with more work chunks than the delivery's persistent grid holds is
+handed out chunk by chunk from a per-launch counter (32 counter pairs per
+context, used round robin and reset by each launch's last CTA).  Here a
+batch of 1,024 stacks (about 2,900 chunks) is delivered many times: from two
+streams at once, so two launches with different counter pairs run
+concurrently, and more than 32 times in a row inside a CUDA graph, so every
+pair is reused.  Every delivery must equal the first bit for bit, and the
+first must equal the oracle on a strided sample of rows.
+"""
+import numpy as np
+import pytest
+import torch
+
+from gpu_util import MirroredDqn, bits, dqn_outputs, fx, to_np
+
+pytestmark = pytest.mark.gpu
+
+B, CAP, N_INGEST = 1024, 3000, 2900
+
+
+def test_concurrent_and_repeated_counter_deliveries(edp_lib, orc):
+    edp = edp_lib
+    frames, action, reward, done = fx.dqn_transitions(40, N_INGEST, done_p=0.05)
+    m = MirroredDqn(CAP)
+    m.ingest(orc, frames, action, reward, done)
+    idx = torch.empty(B, dtype=torch.int64, device="cuda")
+    edp.edp_sample(m.ring.ctx, edp.EDP_SAMPLE_UNIFORM, B, 41, 0, idx)
+    outs = [dqn_outputs(B, m.K, m.F) for _ in range(4)]
+    batches = [edp.make_batch(*o) for o in outs]
+    streams = [torch.cuda.Stream(), torch.cuda.Stream()]
+    torch.cuda.synchronize()
+    # two concurrent launches per stream pair, twice
+    start = torch.cuda.Event()
+    start.record()
+    for i, b in enumerate(batches):
+        st = streams[i % 2]
+        st.wait_event(start)
+        edp.edp_deliver(m.ring.ctx, idx, B, b, stream=st)
+    torch.cuda.synchronize()
+    edp.edp_sync(m.ring.ctx)
+    ref = [bits(t) if t.is_floating_point() else to_np(t) for t in outs[0]]
+    for o in outs[1:]:
+        for x, y in zip(ref, o):
+            assert np.array_equal(x, bits(y) if y.is_floating_point() else to_np(y))
+    # the first delivery against the oracle on every 7th row
+    sel = np.arange(0, B, 7)
+    ref_idx = to_np(idx)
+    r_obs, r_nxt, r_act, r_rew, r_dn = orc.deliver_dqn(
+        m.frames, m.done, m.action, m.reward, m.cap, m.total, m.K, ref_idx[sel])
+    assert np.array_equal(ref[0][sel].reshape(r_obs.shape), r_obs.view(np.uint32))
+    assert np.array_equal(ref[1][sel].reshape(r_nxt.shape), r_nxt.view(np.uint32))
+    assert np.array_equal(ref[2][sel], r_act)
+    assert np.array_equal(ref[3][sel], r_rew.view(np.uint32))
+    assert np.array_equal(ref[4][sel], r_dn)
+    # 40 launches in one graph (every counter pair used at least once more),
+    # alternating between two output sets; the last two must equal ref
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, capture_error_mode="thread_local"):
+        for i in range(40):
+            edp.edp_deliver(m.ring.ctx, idx, B, batches[2 + i % 2])
+    for o in outs[2:]:
+        for t in o:
+            t.fill_(7)
+    g.replay()
+    torch.cuda.synchronize()
+    edp.edp_sync(m.ring.ctx)
+    for o in outs[2:]:
+        for x, y in zip(ref, o):
+            assert np.array_equal(x, bits(y) if y.is_floating_point() else to_np(y))
