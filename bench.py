@@ -685,19 +685,25 @@ class PpoIteration(Workload):
         for m in range(self.M):
             self._mb(m, r)
 
-    def _deliver_all(self):
-        b = self.edp.make_batch(self.out_all,
-                                gather=[(self.nrm.view(-1), self.a_all),
-                                        (self.ret.view(-1), self.r_all)])
-        self.edp.edp_deliver(self.ring.ctx, self.idx, self.n, b)
+    def _deliver_all(self, parts=1):
+        """The iteration's deliveries in `parts` calls (granularity
+        g_del = 1 / parts); call p fills rows [p n / parts, (p+1) n / parts)
+        of the output."""
+        m = self.n // parts
+        for p in range(parts):
+            sl = slice(p * m, (p + 1) * m)
+            b = self.edp.make_batch(self.out_all[sl],
+                                    gather=[(self.nrm.view(-1), self.a_all[sl]),
+                                            (self.ret.view(-1), self.r_all[sl])])
+            self.edp.edp_deliver(self.ring.ctx, self.idx[sl], m, b)
 
-    def round_batched(self, r):
+    def round_parts(self, r, parts):
         """GAE on a side stream beside the shuffle (the two are independent:
-        GAE reads the rollout scalars, the shuffle only its keys), then one
-        delivery call for the whole iteration: the delivery granularity
-        g_del = 1 of Sec. 4.2 instead of one call per mini-batch.  Mini-batch
-        m is rows [4096 m, 4096 (m + 1)) of the output, equal to what the
-        m-th per-mini-batch call delivers."""
+        GAE reads the rollout scalars, the shuffle only its keys), then the
+        iteration's delivery in `parts` calls: delivery granularity
+        g_del = 1 / parts (Sec. 4.2).  With parts = 1 a single call delivers
+        all mini-batches; mini-batch m is rows [4096 m, 4096 (m + 1)) of the
+        output, equal to what the m-th per-mini-batch call delivers."""
         import torch
         main = torch.cuda.current_stream()
         self.fork.record()  # the side stream starts after prior work
@@ -710,12 +716,21 @@ class PpoIteration(Workload):
         self.edp.edp_sample(self.ring.ctx, self.edp.EDP_SAMPLE_PERMUTE, self.n,
                             self.seed, r, self.idx)
         main.wait_event(self.gae_done)
-        self._deliver_all()
+        self._deliver_all(parts)
+
+    def round_batched(self, r):
+        self.round_parts(r, 1)
 
     def schedules(self):
+        """The delivery-granularity sweep of Sec. 6.1 on this iteration:
+        g_del = 1 (main), 1/2, 1/4 and 1/8 with GAE beside the shuffle, and
+        the plain one-stream iteration with one call per mini-batch."""
+        sweep = [("g=1/%d" % k, (lambda r, k=k: self.round_parts(r, k)),
+                  "GAE on a side stream beside the shuffle; %d delivery calls of "
+                  "%d samples (g_del = 1/%d)" % (k, self.n // k, k)) for k in (2, 4, 8)]
         return [("batched", self.round_batched,
                  "GAE on a side stream beside the shuffle; one delivery call "
-                 "for all 8 mini-batches (g_del = 1)"),
+                 "for all 8 mini-batches (g_del = 1)")] + sweep + [
                 ("per-minibatch", self.round,
                  "GAE, shuffle, 8 mini-batch deliveries of 4,096, one stream "
                  "(g_del = 1/8)")]
