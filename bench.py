@@ -276,6 +276,18 @@ class Workload:
         torch.cuda.synchronize()
         return e0.elapsed_time(e1) * 1e3 / n
 
+    def time_calls(self, fn, n, mk, stream):
+        """Average device time (us) of fn() run n times back to back from a
+        CUDA graph (two eager calls first)."""
+        import torch
+        run = self._graph_or_eager(lambda: [fn() for _ in range(n)], True)
+        e0, e1 = mk(), mk()
+        e0.record(stream)
+        run()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) * 1e3 / n
+
     def time_latency(self, n, mk, stream):
         """Sample -> batch latency (us) of n steps, events around each."""
         import torch
@@ -420,6 +432,26 @@ class PerReplay(Workload):
     def deliver_once(self, r):
         o = self.outs[r % self.R]
         self.edp.edp_deliver(self.ring.ctx, o["idx"], self.B, o["batch"])
+
+    def extra(self, device, mk, stream, deliver_us):
+        """Ingestion (row a1) on this ring, timed after everything else: 4,096
+        new transitions per call from device staging -- frames, metadata
+        and their PER leaves at the running maximum priority (the deferred
+        newest leaf included) with the tree above them refreshed."""
+        import torch
+        from paper_2609_24456_gb300 import fixtures as fx
+        n = 4096
+        st = torch.empty((n, self.F), dtype=torch.uint8, device=device)
+        fx.content_fill_torch(self.seed, self.cap, st)
+        _, action, reward, done = fx.dqn_transitions(self.seed + 1, n, with_frames=False)
+        a, rw, d = dev(action, device), dev(reward, device), dev(done, device)
+        us = self.time_calls(lambda: self.edp.edp_ingest(
+            self.ring.ctx, st, n, action=a, reward=rw, done=d), 50, mk, stream)
+        nbytes = n * (2 * self.F + 2 * 9) + n * 4
+        return {"ingest": {"rows": n, "us": us, "GBs": nbytes / (us / 1e6) / 1e9,
+                           "bytes_per_call": nbytes,
+                           "what": "frames read + written, action/reward/done read + "
+                                   "written, PER leaves written; tree refresh"}}
 
     def latency_step(self, r, ev_end):
         o = self.outs[r % self.R]
@@ -737,6 +769,18 @@ class PpoIteration(Workload):
 
     def deliver_once(self, r):
         self._deliver_all()
+
+    def extra(self, device, mk, stream, deliver_us):
+        """Rollout ingestion (row a1), reported beside the iteration as the
+        workload asks: the 32,768 observations of a rollout copied from the
+        actors' device buffer into the ring (402.7 MB read + 402.7 MB
+        written)."""
+        us = self.time_calls(lambda: self.edp.edp_ingest(self.ring.ctx, self.d_obs, self.n),
+                             50, mk, stream)
+        nbytes = 2 * self.n * self.F
+        return {"ingest": {"rows": self.n, "us": us, "GBs": nbytes / (us / 1e6) / 1e9,
+                           "bytes_per_call": nbytes,
+                           "what": "rollout observations device -> ring"}}
 
     def latency_step(self, r, ev_end):
         self._gae()
