@@ -641,8 +641,8 @@ class PpoIteration(Workload):
     dtype = "u8->bf16,f64"
     T, E, H, W, C, M = 128, 256, 64, 64, 3, 8
 
-    def __init__(self, seed=1236):
-        self.seed = seed
+    def __init__(self, seed=1236, sched=True):
+        self.seed, self.sched = seed, sched
         self.n = self.T * self.E
         self.mb = self.n // self.M
         F = self.H * self.W * self.C
@@ -778,9 +778,153 @@ class PpoIteration(Workload):
         us = self.time_calls(lambda: self.edp.edp_ingest(self.ring.ctx, self.d_obs, self.n),
                              50, mk, stream)
         nbytes = 2 * self.n * self.F
-        return {"ingest": {"rows": self.n, "us": us, "GBs": nbytes / (us / 1e6) / 1e9,
-                           "bytes_per_call": nbytes,
-                           "what": "rollout observations device -> ring"}}
+        out = {"ingest": {"rows": self.n, "us": us, "GBs": nbytes / (us / 1e6) / 1e9,
+                          "bytes_per_call": nbytes,
+                          "what": "rollout observations device -> ring"}}
+        if self.sched:
+            out["sched"] = self.sched_experiment(device, mk, stream)
+        return out
+
+    # -- latency-aware scheduling, measured (Sec. 6; the auto-versus-manual
+    # comparison of Sec. 7, reproduced with synthetic data) ----------------
+    def _learn(self, m):
+        """Stand-in learner update on mini-batch m: one bf16 GEMM over its
+        observations (4,096 x 12,288 @ 12,288 x 512, cuBLAS), about the cost
+        of a small policy network's forward and backward pass."""
+        import torch
+        x = self.out_all[m * self.mb:(m + 1) * self.mb].view(self.mb, -1)
+        torch.matmul(x, self.w_learn, out=self.y_learn)
+
+    def _iteration(self, r, parts, overlap):
+        """Ingest the rollout, GAE beside the shuffle, then the delivery in
+        `parts` calls and the learner on every mini-batch: inline (deliver
+        part c, learn its mini-batches, next part), or overlapped (the parts
+        delivered on a side stream back to back, the learner on part c once
+        its delivery has finished: mini-batch pipelining)."""
+        import torch
+        main = torch.cuda.current_stream()
+        self.edp.edp_ingest(self.ring.ctx, self.d_obs, self.n)
+        self.fork.record()
+        with torch.cuda.stream(self.side):
+            self.side.wait_event(self.fork)
+            self.edp.edp_gae(self.ring.ctx, self.r, self.v, self.d, self.T, self.E,
+                             0.99, 0.95, self.adv, self.ret, self.nrm, stream=self.side)
+            self.gae_done.record()
+        self.edp.edp_sample(self.ring.ctx, self.edp.EDP_SAMPLE_PERMUTE, self.n,
+                            self.seed, r, self.idx)
+        main.wait_event(self.gae_done)
+        m_per = self.M // parts
+        rows = self.n // parts
+
+        def deliver(c, st=None):
+            sl = slice(c * rows, (c + 1) * rows)
+            b = self.edp.make_batch(self.out_all[sl],
+                                    gather=[(self.nrm.view(-1), self.a_all[sl]),
+                                            (self.ret.view(-1), self.r_all[sl])])
+            self.edp.edp_deliver(self.ring.ctx, self.idx[sl], rows, b, stream=st)
+
+        if not overlap:
+            for c in range(parts):
+                deliver(c)
+                for m in range(c * m_per, (c + 1) * m_per):
+                    self._learn(m)
+            return
+        self.fork.record()
+        with torch.cuda.stream(self.side):
+            self.side.wait_event(self.fork)
+            for c in range(parts):
+                deliver(c, self.side)
+                self.part_done[c].record()
+        for c in range(parts):
+            main.wait_event(self.part_done[c])
+            for m in range(c * m_per, (c + 1) * m_per):
+                self._learn(m)
+        main.wait_stream(self.side)
+
+    def sched_experiment(self, device, mk, stream, reps=20):
+        """Profile the operator costs once, let edp_sched_choose pick the
+        delivery timing and granularity (Eq. 2), and time every feasible
+        configuration to see whether the pick is the fastest.  On-policy
+        candidates: g_del = k/8 for k | 8.  Overlap means pipelining within
+        the iteration, so it needs g_del < 1; g_del = 1 runs inline only."""
+        import torch
+        self.w_learn = torch.randn(self.F, 512, device=device).to(torch.bfloat16) * 0.01
+        self.y_learn = torch.empty(self.mb, 512, device=device, dtype=torch.bfloat16)
+        self.part_done = [torch.cuda.Event() for _ in range(self.M)]
+        G = self.edp.edp_sched_granularities(True, self.M)
+        # profiled costs (us): learner update of one iteration, one delivery
+        # invocation at each g, the ingestion side (ingest + GAE beside the
+        # shuffle), and one cross-stream hand-off
+        t_update = self.time_calls(lambda: [self._learn(m) for m in range(self.M)],
+                                   reps, mk, stream)
+        t_del = []
+        for g in G:
+            rows = int(round(g * self.n))
+            sl = slice(0, rows)
+            b = self.edp.make_batch(self.out_all[sl],
+                                    gather=[(self.nrm.view(-1), self.a_all[sl]),
+                                            (self.ret.view(-1), self.r_all[sl])])
+            t_del.append(self.time_calls(
+                lambda: self.edp.edp_deliver(self.ring.ctx, self.idx[sl], rows, b),
+                reps, mk, stream))
+
+        def ing_side():
+            self.edp.edp_ingest(self.ring.ctx, self.d_obs, self.n)
+            self.fork.record()
+            with torch.cuda.stream(self.side):
+                self.side.wait_event(self.fork)
+                self.edp.edp_gae(self.ring.ctx, self.r, self.v, self.d, self.T, self.E,
+                                 0.99, 0.95, self.adv, self.ret, self.nrm,
+                                 stream=self.side)
+                self.gae_done.record()
+            self.edp.edp_sample(self.ring.ctx, self.edp.EDP_SAMPLE_PERMUTE, self.n,
+                                self.seed, 0, self.idx)
+            torch.cuda.current_stream().wait_event(self.gae_done)
+        t_ing = self.time_calls(ing_side, reps, mk, stream)
+
+        def handoff():
+            self.fork.record()
+            with torch.cuda.stream(self.side):
+                self.side.wait_event(self.fork)
+                self.y_learn[:1, :1].zero_()
+                self.gae_done.record()
+            torch.cuda.current_stream().wait_event(self.gae_done)
+        t_sync = self.time_calls(handoff, reps, mk, stream)
+        nd = len(G)
+        feasible = [(o, j) for o in (0, 1) for j in range(nd) if not (o and G[j] >= 1)]
+
+        def pick(c_del):
+            _, scores = self.edp.edp_sched_choose(0.0, t_update, 0.0, t_sync, [1.0], [t_ing],
+                                                  G, t_del, all_scores=True,
+                                                  contention_del=c_del)
+            pred = {(o, j): scores[o * nd + j] for (o, j) in feasible}  # o_ing = 0
+            return min(feasible, key=lambda k: (pred[k], k)), pred
+
+        measured = {(o, j): self.time_calls(
+            lambda: self._iteration(0, int(round(1 / G[j])), o), reps, mk, stream)
+            for (o, j) in feasible}
+        fastest = min(measured, key=measured.get)
+        paper_pick, paper_pred = pick(0.0)
+        # one probe pair calibrates the contention: inline and overlapped at
+        # the finest granularity; the share of the model's hidden time that
+        # the overlap actually saved
+        j0 = 0
+        tbar = t_del[j0] / G[j0]
+        hide0 = (1.0 - G[j0]) * min(t_update, tbar)
+        saved = measured[(0, j0)] - measured[(1, j0)] + t_sync
+        c_del = min(1.0, max(0.0, 1.0 - saved / hide0)) if hide0 > 0 else 1.0
+        cal_pick, cal_pred = pick(c_del)
+        fmt = lambda k: {"g_del": G[k[1]], "overlap_del": k[0]}
+        return {"costs_us": {"t_update": t_update, "t_ing": t_ing, "t_sync_del": t_sync,
+                             "t_del": dict(zip(["%g" % g for g in G], t_del))},
+                "configs": [dict(fmt(k), measured_us=measured[k],
+                                 predicted_us=paper_pred[k],
+                                 predicted_calibrated_us=cal_pred[k]) for k in feasible],
+                "fastest": fmt(fastest),
+                "paper_model": dict(fmt(paper_pick),
+                                    over_fastest=measured[paper_pick] / measured[fastest]),
+                "calibrated": dict(fmt(cal_pick), contention_del=c_del,
+                                   over_fastest=measured[cal_pick] / measured[fastest])}
 
     def latency_step(self, r, ev_end):
         self._gae()

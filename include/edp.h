@@ -322,6 +322,70 @@ EDP_API edp_status edp_get_info(const edp_ctx *ctx, edp_info *out);
 EDP_API edp_status edp_probe_host_read(const void *host_src, uint64_t bytes,
                                uint64_t *d_fold, edp_stream stream);
 
+/* ---------------------------------------------------------------------------
+ * Latency-aware scheduling (Sec. 6): choose when ingestion and delivery run
+ * (timing: inline, or overlapped with rollout / learner update) and how much
+ * each invocation processes (granularity g: g >= 1 batches g rollout units /
+ * training batches, 0 < g < 1 pipelines a fraction of one), from profiled
+ * costs, by the iteration-latency model of Sec. 6.2 and Appendix D and the
+ * enumeration of Eq. 2 (Sec. 6.3):
+ *
+ *   Tbar(g)    = T(g) / g                       (per-unit cost)
+ *   gamma(g)   = 1 if g >= 1, else 1 - g
+ *   hide_ing   = (1 - c_ing) gamma(g_ing) min(T_rollout, Tbar_ing(g_ing))
+ *   hide_del   = (1 - c_del) gamma(g_del) min(T_update,  Tbar_del(g_del))
+ *   T_ing_path = T_rollout + Tbar_ing(g_ing) + o_ing (T_sync_ing - hide_ing)
+ *   T_del_path = T_update  + Tbar_del(g_del) + o_del (T_sync_del - hide_del)
+ *   T_iter     = T_ing_path + T_del_path,  minimised over o_ing, o_del in
+ *                {0, 1} and the candidate granularities.
+ *
+ * c_ing, c_del are not in the paper, which assumes the hidden part of an
+ * operator costs its neighbour nothing; they are 0 there (the default of a
+ * zeroed struct).  On one GPU the delivery and the learner update contend
+ * for the same SMs and HBM, so only part of the overlap hides: a caller
+ * that measured it passes the contention c in [0, 1].
+ *
+ * Host-only: no GPU work, no context.  Times in any one unit.
+ * ------------------------------------------------------------------------- */
+typedef struct {
+  double t_rollout;      /* one actor rollout */
+  double t_update;       /* one learner update */
+  double t_sync_ing;     /* synchronisation added by overlapping ingestion */
+  double t_sync_del;     /* ... by overlapping delivery */
+  uint32_t n_ing, n_del; /* number of candidate granularities (>= 1 each) */
+  const double *g_ing;   /* [n_ing] candidate g_ing, each > 0 */
+  const double *t_ing;   /* [n_ing] T_ing(g): one invocation's wall time */
+  const double *g_del;   /* [n_del] candidate g_del, each > 0 */
+  const double *t_del;   /* [n_del] T_del(g) */
+  double contention_ing; /* c_ing in [0, 1]: share of the hidden time lost */
+  double contention_del; /* c_del in [0, 1] */
+} edp_sched_costs;
+
+typedef struct {
+  uint32_t overlap_ing, overlap_del; /* timing flags, 0 or 1 */
+  uint32_t i_ing, i_del;             /* indices of the chosen granularities */
+  double g_ing, g_del;
+  double t_ing_path, t_del_path, t_iter;
+} edp_sched_choice;
+
+/* Score every candidate (o_ing, o_del, i_ing, i_del) and write the one with
+ * the lowest T_iter to *best; ties keep the first in the order o_ing,
+ * o_del, i_ing, i_del, each ascending (so inline timing and the earlier
+ * candidate win a tie).  t_iter_all (may be NULL) receives every score,
+ * [2][2][n_ing][n_del] in that order.  EDP_ERR_INVALID for a NULL argument,
+ * a zero count, a non-positive or non-finite g, a negative or non-finite
+ * time, or a contention outside [0, 1]. */
+EDP_API edp_status edp_sched_choose(const edp_sched_costs *costs,
+                                    edp_sched_choice *best, double *t_iter_all);
+
+/* Candidate granularities derived from the RL configuration (Sec. 6.3):
+ * off-policy (on_policy = 0): 1, 2, 4, ... up to `m` batches per invocation;
+ * on-policy: k / m for every divisor k of m, m = mini-batches per rollout
+ * unit, ascending.  Writes at most `cap` values to g and returns how many
+ * there are (call with cap = 0 to size g); 0 if m == 0. */
+EDP_API uint32_t edp_sched_granularities(uint32_t on_policy, uint32_t m, double *g,
+                                         uint32_t cap);
+
 /* ABI version compiled into the library (EDP_ABI_VERSION). */
 EDP_API int edp_abi_version(void);
 

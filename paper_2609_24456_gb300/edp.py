@@ -66,6 +66,23 @@ class edp_info(C.Structure):
                 ("max_q", C.c_void_p)]
 
 
+class edp_sched_costs(C.Structure):
+    _fields_ = [("t_rollout", C.c_double), ("t_update", C.c_double),
+                ("t_sync_ing", C.c_double), ("t_sync_del", C.c_double),
+                ("n_ing", C.c_uint32), ("n_del", C.c_uint32),
+                ("g_ing", C.POINTER(C.c_double)), ("t_ing", C.POINTER(C.c_double)),
+                ("g_del", C.POINTER(C.c_double)), ("t_del", C.POINTER(C.c_double)),
+                ("contention_ing", C.c_double), ("contention_del", C.c_double)]
+
+
+class edp_sched_choice(C.Structure):
+    _fields_ = [("overlap_ing", C.c_uint32), ("overlap_del", C.c_uint32),
+                ("i_ing", C.c_uint32), ("i_del", C.c_uint32),
+                ("g_ing", C.c_double), ("g_del", C.c_double),
+                ("t_ing_path", C.c_double), ("t_del_path", C.c_double),
+                ("t_iter", C.c_double)]
+
+
 # exported symbols and their signatures (restype, argtypes)
 _VP, _U32, _U64, _D = C.c_void_p, C.c_uint32, C.c_uint64, C.c_double
 SIGNATURES = {
@@ -86,6 +103,9 @@ SIGNATURES = {
     "edp_get_info": (C.c_int, [_VP, C.POINTER(edp_info)]),
     "edp_probe_host_read": (C.c_int, [_VP, _U64, _VP, _VP]),
     "edp_abi_version": (C.c_int, []),
+    "edp_sched_choose": (C.c_int, [C.POINTER(edp_sched_costs),
+                                   C.POINTER(edp_sched_choice), _VP]),
+    "edp_sched_granularities": (_U32, [_U32, _U32, _VP, _U32]),
 }
 
 _lib = None
@@ -313,3 +333,34 @@ class Ring:
             self.close()
         except Exception:
             pass
+
+
+def _dvec(xs):
+    return (C.c_double * len(xs))(*[float(x) for x in xs])
+
+
+def edp_sched_choose(t_rollout, t_update, t_sync_ing, t_sync_del, g_ing, t_ing,
+                     g_del, t_del, all_scores=False, contention_ing=0.0,
+                     contention_del=0.0):
+    """Latency-minimising timing and granularity (host only).  Returns the
+    edp_sched_choice, and with all_scores the [2][2][n_ing][n_del] list of
+    every candidate's T_iter."""
+    gi, ti, gd, td = _dvec(g_ing), _dvec(t_ing), _dvec(g_del), _dvec(t_del)
+    c = edp_sched_costs(t_rollout, t_update, t_sync_ing, t_sync_del, len(g_ing),
+                        len(g_del), gi, ti, gd, td, contention_ing, contention_del)
+    out = edp_sched_choice()
+    n = 4 * len(g_ing) * len(g_del)
+    buf = (C.c_double * n)() if all_scores else None
+    st = lib().edp_sched_choose(C.byref(c), C.byref(out),
+                                C.cast(buf, C.c_void_p) if buf is not None else None)
+    if st != EDP_OK:
+        raise EdpError(st, "edp_sched_choose: invalid costs")
+    return (out, list(buf)) if all_scores else out
+
+
+def edp_sched_granularities(on_policy, m):
+    """Candidate granularities for an off- or on-policy configuration."""
+    n = lib().edp_sched_granularities(int(bool(on_policy)), m, None, 0)
+    buf = (C.c_double * max(n, 1))()
+    lib().edp_sched_granularities(int(bool(on_policy)), m, C.cast(buf, C.c_void_p), n)
+    return list(buf)[:n]

@@ -44,7 +44,8 @@ def test_struct_layouts_match_binding(tmp_path):
     from paper_2609_24456_gb300 import edp
     structs = {"edp_config": edp.edp_config, "edp_storage": edp.edp_storage,
                "edp_fields": edp.edp_fields, "edp_batch": edp.edp_batch,
-               "edp_info": edp.edp_info}
+               "edp_info": edp.edp_info, "edp_sched_costs": edp.edp_sched_costs,
+               "edp_sched_choice": edp.edp_sched_choice}
     lines = ['#include <stdio.h>', '#include <stddef.h>', '#include "edp.h"',
              "int main(void) {"]
     for sname, cls in structs.items():
