@@ -1120,11 +1120,13 @@ class MmReplay(Workload):
             self.h_out[k].copy_(o[k], non_blocking=True)
 
     def extra(self, device, mk, stream, deliver_us):
-        """Two-tier only: host-link bandwidth measured in this run (zero-copy
-        read kernel and a pinned H2D copy) and the host-tier share of the
-        delivery's reads against it."""
+        """Two-tier: host-link bandwidth measured in this run (zero-copy read
+        kernel and a pinned H2D copy) and the host-tier share of the
+        delivery's reads against it.  Single tier: the placement experiment
+        (bandwidth table, placement map, and the model checked against
+        measured transfers at this workload's sample size)."""
         if not self.tiered:
-            return {}
+            return {"placement": self.placement_experiment(device, mk, stream, deliver_us)}
         import torch
         from paper_2609_24456_gb300 import edp
         nbytes = 4 << 30
@@ -1155,7 +1157,133 @@ class MmReplay(Workload):
                               "frac_of_link": achieved / link,
                               "host_bytes_per_delivery": host_bytes}}
 
-    def cpu_setup(self, host_rows=16384):
+    def placement_experiment(self, device, mk, stream, deliver_us, rows=16384):
+        """Bandwidth-aware placement on this node (Sec. 5; the placement
+        sweep of Sec. 7, reproduced with synthetic data): profile the
+        effective bandwidths once (edp_place_profile), build the candidate
+        placements for CPU actors and a learner on this GPU, and let the
+        library solve Eq. 1 over per-sample sizes (the placement map) at the
+        paper's sweep capacity of 10^6.  Then, at this workload's sample
+        (150,528-byte image + 2,048 bytes of tokens), time both legs of each
+        placement with the mechanism its bandwidths stand for -- CPU actors
+        copying into host memory, or the GPU reading page-locked staging;
+        the learner's batch gathered on the CPU and copied (pageable),
+        delivered by the kernel from page-locked memory in place (pinned),
+        or from HBM -- and compare the ranking."""
+        import numpy as np
+        import torch
+        from paper_2609_24456_gb300 import edp
+        from paper_2609_24456_gb300 import fixtures as fx
+        bw = edp.edp_place_profile(device.index or 0, 1 << 30)
+        x = self.F + 4 * self.L
+        ring_bytes = self.cap * x
+        mem_gpu = bw["hbm_free"] + ring_bytes - 8e9  # this ring's HBM is the buffer's
+        avail = 0.0
+        with open("/proc/meminfo") as f:
+            for line in f:
+                if line.startswith("MemAvailable:"):
+                    avail = float(line.split()[1]) * 1024
+        mem_host = 0.8 * avail
+        def best_of(fn, k=3):
+            t = []
+            for _ in range(k):
+                torch.cuda.synchronize()
+                t0 = time.perf_counter()
+                fn()
+                torch.cuda.synchronize()
+                t.append(time.perf_counter() - t0)
+            return min(t)
+
+        n_in, B = 4096, self.B
+        rng = np.random.default_rng(self.seed)
+        stage = torch.empty((n_in, x), dtype=torch.uint8, pin_memory=True)
+        stage.numpy()[:] = rng.integers(0, 256, size=(n_in, x), dtype=np.uint8)
+        sel = np.sort(rng.integers(0, rows, size=B))
+        meas = {}
+        # host pageable: actors memcpy into the ring; the learner's batch is
+        # gathered on the CPU into page-locked staging and copied in
+        page = np.empty((rows, x), dtype=np.uint8)
+        page[:] = 1
+        t_in = best_of(lambda: np.copyto(page[:n_in], stage.numpy())) / n_in
+        pin_b = torch.empty((B, x), dtype=torch.uint8, pin_memory=True)
+        dev_b = torch.empty((B, x), dtype=torch.uint8, device=device)
+
+        def gather_copy():
+            np.take(page, sel, axis=0, out=pin_b.numpy())
+            dev_b.copy_(pin_b, non_blocking=True)
+        t_gc = best_of(gather_copy)
+        meas["host_pageable"] = t_in + t_gc / B
+        del page
+        # the pageable path's out-leg bandwidth is that of its mechanism, a
+        # CPU gather then a pageable copy, measured here at this row size
+        bw_gather_copy = B * x / t_gc
+        names = ["host_pageable", "host_pinned", "gpu", "gpu+host"]
+        opts = [dict(kind=edp.EDP_PLACE_HOST_PAGEABLE, bw_in=bw["host_copy"],
+                     bw_out=bw_gather_copy, mem=mem_host),
+                dict(kind=edp.EDP_PLACE_HOST_PINNED, bw_in=bw["host_copy"],
+                     bw_out=bw["zero_copy_read"], mem=mem_host),
+                dict(kind=edp.EDP_PLACE_GPU, bw_in=bw["h2d_pinned"], bw_out=bw["hbm_copy"],
+                     mem=mem_gpu),
+                dict(kind=edp.EDP_PLACE_GPU_HOST, bw_in=bw["h2d_pinned"],
+                     bw_out=bw["hbm_copy"], mem=mem_gpu, bw_out2=bw["zero_copy_read"],
+                     mem2=mem_host)]
+        xs = [int(512 * 2 ** (k / 2)) for k in range(25)]  # 512 B .. 2 MiB, half octaves
+        pmap = edp.edp_place_map(opts, 1e6, xs)
+        best, t_pred = edp.edp_place_choose(opts, self.cap, x)
+
+
+        # host pinned: actors memcpy into page-locked memory; the kernel
+        # delivers from it in place (a ring whose HBM tier holds one entry)
+        cfg = edp.make_config(rows, (self.C, self.H, self.W), edp.EDP_XFORM_CHW_NORM_BF16,
+                              hbm_capacity=1, tokens=self.L, norm_mean=MEAN3,
+                              norm_std=STD3, device=device.index or 0)
+        pr = edp.Ring(cfg, action=False, reward=False, done=False)
+        obs = torch.empty((n_in, self.F), dtype=torch.uint8, device=device)
+        tok = torch.empty((n_in, self.L), dtype=torch.int32, device=device)
+        for lo in range(0, rows, n_in):
+            fx.content_fill_torch(self.seed, lo, obs)
+            fx.token_fill_torch(self.seed, lo, tok)
+            edp.edp_ingest(pr.ctx, obs, n_in, tokens=tok)
+        hobs = pr.host_obs.numpy()
+        t_in = best_of(lambda: np.copyto(hobs[:n_in], stage.numpy()[:, :self.F])) / n_in
+        idx = torch.empty(B, dtype=torch.int64, device=device)
+        out = self.outs[0]
+        batch = edp.make_batch(out["obs"], tokens=out["tok"])
+        edp.edp_sample(pr.ctx, edp.EDP_SAMPLE_UNIFORM, B, self.seed, 0, idx)
+        t_out = self.time_calls(lambda: edp.edp_deliver(pr.ctx, idx, B, batch), 20, mk,
+                                stream) * 1e-6
+        meas["host_pinned"] = t_in + t_out / B
+        pr.close()
+        del pr, hobs
+        # GPU: the ingest kernel reads page-locked staging into HBM; the
+        # delivery kernel gathers from HBM (its time measured above)
+        st_obs = torch.empty((n_in, self.F), dtype=torch.uint8, pin_memory=True)
+        st_tok = torch.empty((n_in, self.L), dtype=torch.int32, pin_memory=True)
+        st_rew = torch.zeros(n_in, dtype=torch.float32, pin_memory=True)
+        st_obs.numpy()[:] = stage.numpy()[:, :self.F]
+        st_tok.numpy()[:] = 7
+        t_in = self.time_calls(lambda: edp.edp_ingest(self.ring.ctx, st_obs, n_in,
+                                                      tokens=st_tok, reward=st_rew),
+                               10, mk, stream) * 1e-6 / n_in
+        meas["gpu"] = t_in + deliver_us * 1e-6 / B
+        # the two-tier placement holds this buffer in HBM alone (h = 1): its
+        # transfers are the GPU placement's
+        meas["gpu+host"] = meas["gpu"]
+        fastest = min(meas, key=meas.get)
+        return {"bandwidth_GBs": dict({k: v / 1e9 for k, v in bw.items() if k != "hbm_free"},
+                                      host_gather_copy=bw_gather_copy / 1e9),
+                "mem_GB": {"gpu": mem_gpu / 1e9, "host": mem_host / 1e9},
+                "map_c_buf_1e6": [{"x_bytes": xx, "placement": names[c] if c < 4 else None}
+                                  for xx, c in zip(xs, pmap)],
+                "at_this_sample": {
+                    "x_bytes": x, "c_buf": self.cap,
+                    "predicted_us_per_sample": {n: t * 1e6 for n, t in zip(names, t_pred)},
+                    "measured_us_per_sample": {n: t * 1e6 for n, t in meas.items()},
+                    "chosen": names[best], "fastest_measured": fastest,
+                    "measured_ranking": sorted(meas, key=meas.get),
+                    "predicted_ranking": [names[i] for i in sorted(range(4),
+                                                                   key=lambda i: (t_pred[i], i))]}}
+
         import numpy as np
         import oracle as orc
         from paper_2609_24456_gb300 import fixtures as fx

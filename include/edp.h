@@ -327,7 +327,7 @@ EDP_API edp_status edp_probe_host_read(const void *host_src, uint64_t bytes,
  * (timing: inline, or overlapped with rollout / learner update) and how much
  * each invocation processes (granularity g: g >= 1 batches g rollout units /
  * training batches, 0 < g < 1 pipelines a fraction of one), from profiled
- * costs, by the iteration-latency model of Sec. 6.2 and Appendix D and the
+ * costs, by the iteration-latency model of Sec. 6.2 and Appendix E and the
  * enumeration of Eq. 2 (Sec. 6.3):
  *
  *   Tbar(g)    = T(g) / g                       (per-unit cost)
@@ -385,6 +385,80 @@ EDP_API edp_status edp_sched_choose(const edp_sched_costs *costs,
  * there are (call with cap = 0 to size g); 0 if m == 0. */
 EDP_API uint32_t edp_sched_granularities(uint32_t on_policy, uint32_t m, double *g,
                                          uint32_t cap);
+
+/* ---------------------------------------------------------------------------
+ * Bandwidth-aware placement (Sec. 5): the per-sample transfer latency of a
+ * placement p (Sec. 5.1)
+ *
+ *   T(p, x) = x / BW(actor -> p) + x / BW(p -> learner GPU)
+ *
+ * and the feasible minimum of Eq. 1, found by the linear scan of Alg. 1:
+ * p* = argmin T(p, x) subject to C_buf x <= Mem(p); the first option wins a
+ * tie.  A placement may have two tiers (the paper's mixture of local and
+ * remote reads, here fast and slow memory of one node): the newest
+ * transitions fill tier 1, so with uniform sampling a share
+ * h = min(1, Mem1 / (C_buf x)) of the reads comes from tier 1 and
+ *
+ *   x / BW(p -> GPU) = x (h / bw_out + (1 - h) / bw_out2),
+ *
+ * feasible when C_buf x <= Mem1 + Mem2.  Bandwidths in bytes/s, sizes in
+ * bytes, times in seconds.  Host-only: no GPU work, no context.
+ * ------------------------------------------------------------------------- */
+typedef enum {
+  EDP_PLACE_HOST_PAGEABLE = 0, /* CPU pageable memory (staged copies) */
+  EDP_PLACE_HOST_PINNED = 1,   /* CPU page-locked memory, zero-copy reads */
+  EDP_PLACE_GPU = 2,           /* HBM of the learner's GPU */
+  EDP_PLACE_GPU_HOST = 3       /* newest in HBM, older in page-locked memory */
+} edp_place_kind;
+
+typedef struct {
+  uint32_t kind;      /* edp_place_kind; not used by the arithmetic */
+  uint32_t tiers;     /* 1 or 2 */
+  double bw_in;       /* effective bandwidth actor -> placement, > 0 */
+  double bw_out;      /* tier 1 -> learner GPU, > 0 */
+  double mem;         /* capacity of tier 1, >= 0 */
+  double bw_out2;     /* tier 2 -> learner GPU (> 0 when tiers == 2) */
+  double mem2;        /* capacity of tier 2 (tiers == 2) */
+} edp_place_option;
+
+/* Alg. 1 over opts[0..n): *best = index of the chosen placement, or n when
+ * none is feasible (status EDP_ERR_EMPTY).  t_all (may be NULL) receives
+ * T(p, x) for every option, +infinity for infeasible ones.
+ * EDP_ERR_INVALID for NULL opts/best, n == 0, c_buf or x not finite and
+ * > 0, or an option with a non-positive or non-finite bandwidth, a
+ * negative capacity, or tiers not 1 or 2. */
+EDP_API edp_status edp_place_choose(const edp_place_option *opts, uint32_t n,
+                                    double c_buf, double x, uint32_t *best,
+                                    double *t_all);
+
+/* The placement map of Appendix D: the choice of edp_place_choose for each
+ * per-sample size x[0..nx) (n where none is feasible), computed once so
+ * that a change of x at run time is a lookup.  Errors as edp_place_choose;
+ * an infeasible size is not an error here. */
+EDP_API edp_status edp_place_map(const edp_place_option *opts, uint32_t n,
+                                 double c_buf, const double *x, uint32_t nx,
+                                 uint32_t *choice);
+
+/* Effective bandwidths of this node's paths (Sec. 5.1: measured by
+ * microbenchmarks on the deployment stack), in bytes moved per second;
+ * each is the best of three timed transfers of `bytes`. */
+typedef struct {
+  double hbm_copy;       /* device -> device copy (each byte read and written) */
+  double h2d_pinned;     /* cudaMemcpy, page-locked host -> device */
+  double d2h_pinned;     /* cudaMemcpy, device -> page-locked host */
+  double h2d_pageable;   /* cudaMemcpy, pageable host -> device */
+  double zero_copy_read; /* a kernel reading page-locked host memory in place */
+  double host_copy;      /* one CPU thread, memcpy pageable -> page-locked */
+  double hbm_free;       /* free device memory (bytes) before the buffers below */
+} edp_place_bw;
+
+/* Measure edp_place_bw on `device` with buffers of `bytes` (a multiple of
+ * 16, >= 1 MiB): allocates 2 x bytes of device memory, `bytes` of
+ * page-locked and `bytes` of pageable host memory for the duration of the
+ * call and frees them.  EDP_ERR_INVALID for bad arguments, EDP_ERR_OOM when
+ * an allocation fails, EDP_ERR_CUDA for other CUDA errors.  Synchronises
+ * the device. */
+EDP_API edp_status edp_place_profile(int device, uint64_t bytes, edp_place_bw *out);
 
 /* ABI version compiled into the library (EDP_ABI_VERSION). */
 EDP_API int edp_abi_version(void);

@@ -2,7 +2,7 @@
 only: the tests and the benchmark's CPU leg may use it, the library never).
 
 Sec. 6.2 models one RL iteration as the exposed ingestion path plus the
-exposed delivery path; Appendix D gives the hidden terms; Eq. 2 (Sec. 6.3)
+exposed delivery path; Appendix E gives the hidden terms; Eq. 2 (Sec. 6.3)
 picks the timing flags and granularities that minimise the sum by scoring
 every candidate.  Plain Python floats, the formulas in the paper's order.
 """
@@ -14,12 +14,12 @@ def per_unit(t_of_g, g):
 
 
 def gamma(g):
-    """Overlapable share (Appendix D): 1 for g >= 1, 1 - g for 0 < g < 1."""
+    """Overlapable share (Appendix E): 1 for g >= 1, 1 - g for 0 < g < 1."""
     return 1.0 if g >= 1 else 1.0 - g
 
 
 def hide(t_neighbour, g, t_of_g, contention=0.0):
-    """hide = gamma(g) * min(T_neighbour, Tbar(g)) (Appendix D), where the
+    """hide = gamma(g) * min(T_neighbour, Tbar(g)) (Appendix E), where the
     neighbour is the rollout for ingestion and the update for delivery,
     scaled by (1 - contention) -- a factor the paper does not have (it is 0
     there): the share of the overlap lost when operator and neighbour share

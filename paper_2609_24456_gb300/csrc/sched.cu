@@ -1,5 +1,5 @@
 // sched.cu -- latency-aware scheduling of ingestion and delivery (Sec. 6):
-// the iteration-latency model (Sec. 6.2, Appendix D) and the cost-based
+// the iteration-latency model (Sec. 6.2, Appendix E) and the cost-based
 // choice of timing and granularity (Eq. 2, Sec. 6.3).  Host code only; the
 // formulas are stated in edp.h.
 #include <cmath>

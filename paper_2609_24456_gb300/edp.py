@@ -83,6 +83,22 @@ class edp_sched_choice(C.Structure):
                 ("t_iter", C.c_double)]
 
 
+EDP_PLACE_HOST_PAGEABLE, EDP_PLACE_HOST_PINNED, EDP_PLACE_GPU, EDP_PLACE_GPU_HOST = range(4)
+
+
+class edp_place_option(C.Structure):
+    _fields_ = [("kind", C.c_uint32), ("tiers", C.c_uint32), ("bw_in", C.c_double),
+                ("bw_out", C.c_double), ("mem", C.c_double), ("bw_out2", C.c_double),
+                ("mem2", C.c_double)]
+
+
+class edp_place_bw(C.Structure):
+    _fields_ = [("hbm_copy", C.c_double), ("h2d_pinned", C.c_double),
+                ("d2h_pinned", C.c_double), ("h2d_pageable", C.c_double),
+                ("zero_copy_read", C.c_double), ("host_copy", C.c_double),
+                ("hbm_free", C.c_double)]
+
+
 # exported symbols and their signatures (restype, argtypes)
 _VP, _U32, _U64, _D = C.c_void_p, C.c_uint32, C.c_uint64, C.c_double
 SIGNATURES = {
@@ -106,6 +122,10 @@ SIGNATURES = {
     "edp_sched_choose": (C.c_int, [C.POINTER(edp_sched_costs),
                                    C.POINTER(edp_sched_choice), _VP]),
     "edp_sched_granularities": (_U32, [_U32, _U32, _VP, _U32]),
+    "edp_place_choose": (C.c_int, [C.POINTER(edp_place_option), _U32, _D, _D,
+                                   C.POINTER(C.c_uint32), _VP]),
+    "edp_place_map": (C.c_int, [C.POINTER(edp_place_option), _U32, _D, _VP, _U32, _VP]),
+    "edp_place_profile": (C.c_int, [C.c_int, _U64, C.POINTER(edp_place_bw)]),
 }
 
 _lib = None
@@ -364,3 +384,48 @@ def edp_sched_granularities(on_policy, m):
     buf = (C.c_double * max(n, 1))()
     lib().edp_sched_granularities(int(bool(on_policy)), m, C.cast(buf, C.c_void_p), n)
     return list(buf)[:n]
+
+
+def _options(opts):
+    """opts: sequence of dicts with kind, bw_in, bw_out, mem and, for two
+    tiers, bw_out2 and mem2."""
+    arr = (edp_place_option * len(opts))()
+    for a, o in zip(arr, opts):
+        two = "bw_out2" in o
+        a.kind, a.tiers = o.get("kind", 0), 2 if two else 1
+        a.bw_in, a.bw_out, a.mem = o["bw_in"], o["bw_out"], o["mem"]
+        a.bw_out2, a.mem2 = (o["bw_out2"], o["mem2"]) if two else (0.0, 0.0)
+    return arr
+
+
+def edp_place_choose(opts, c_buf, x):
+    """(index of the chosen placement or len(opts) if none fits, [T(p, x)])."""
+    arr = _options(opts)
+    best = C.c_uint32()
+    t = (C.c_double * len(opts))()
+    st = lib().edp_place_choose(arr, len(opts), float(c_buf), float(x), C.byref(best),
+                                C.cast(t, C.c_void_p))
+    if st not in (EDP_OK, EDP_ERR_EMPTY):
+        raise EdpError(st, "edp_place_choose: invalid options")
+    return best.value, list(t)
+
+
+def edp_place_map(opts, c_buf, xs):
+    """The placement chosen for every per-sample size in xs."""
+    arr = _options(opts)
+    xv = _dvec(xs)
+    out = (C.c_uint32 * max(len(xs), 1))()
+    st = lib().edp_place_map(arr, len(opts), float(c_buf), C.cast(xv, C.c_void_p),
+                             len(xs), C.cast(out, C.c_void_p))
+    if st != EDP_OK:
+        raise EdpError(st, "edp_place_map: invalid options")
+    return list(out)[:len(xs)]
+
+
+def edp_place_profile(device=0, nbytes=1 << 30):
+    """Effective bandwidths of this node's paths (bytes/s) as a dict."""
+    out = edp_place_bw()
+    st = lib().edp_place_profile(int(device), int(nbytes), C.byref(out))
+    if st != EDP_OK:
+        raise EdpError(st, "edp_place_profile failed (status %d)" % st)
+    return {f: getattr(out, f) for f, _ in edp_place_bw._fields_}

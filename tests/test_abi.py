@@ -45,7 +45,9 @@ def test_struct_layouts_match_binding(tmp_path):
     structs = {"edp_config": edp.edp_config, "edp_storage": edp.edp_storage,
                "edp_fields": edp.edp_fields, "edp_batch": edp.edp_batch,
                "edp_info": edp.edp_info, "edp_sched_costs": edp.edp_sched_costs,
-               "edp_sched_choice": edp.edp_sched_choice}
+               "edp_sched_choice": edp.edp_sched_choice,
+               "edp_place_option": edp.edp_place_option,
+               "edp_place_bw": edp.edp_place_bw}
     lines = ['#include <stdio.h>', '#include <stddef.h>', '#include "edp.h"',
              "int main(void) {"]
     for sname, cls in structs.items():

@@ -1,4 +1,4 @@
-"""Pins of the scheduling model (Sec. 6.2-6.3, Eq. 2, Appendix D) against
+"""Pins of the scheduling model (Sec. 6.2-6.3, Eq. 2, Appendix E) against
 values worked out by hand from the formulas, and against properties that
 any correct enumeration has."""
 import itertools
