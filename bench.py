@@ -1270,7 +1270,34 @@ class MmReplay(Workload):
         # transfers are the GPU placement's
         meas["gpu+host"] = meas["gpu"]
         fastest = min(meas, key=meas.get)
-        return {"bandwidth_GBs": dict({k: v / 1e9 for k, v in bw.items() if k != "hbm_free"},
+        # online migration (Alg. 2): this buffer from the GPU placement to
+        # GPU + host (half of it in HBM), one edp_migrate call, against the
+        # makespan of its transfers run side by side (Appendix D, with the
+        # flows fixed by the layout: the newer half HBM -> HBM, the older
+        # half HBM -> page-locked memory)
+        cfg2 = edp.make_config(self.cap, (self.C, self.H, self.W),
+                               edp.EDP_XFORM_CHW_NORM_BF16, hbm_capacity=self.cap // 2,
+                               tokens=self.L, norm_mean=MEAN3, norm_std=STD3,
+                               device=device.index or 0)
+        r2 = edp.Ring(cfg2, action=False, done=False)
+        torch.cuda.synchronize()
+        e0, e1 = mk(), mk()
+        e0.record(stream)
+        edp.edp_migrate(self.ring.ctx, r2.ctx)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        edp.edp_sync(r2.ctx)
+        mig_s = e0.elapsed_time(e1) / 1e3
+        n_h = self.cap // 2
+        f_hbm, f_host = n_h * x, (self.cap - n_h) * x
+        pred_s = max(f_hbm / bw["hbm_copy"], f_host / bw["d2h_pinned"])
+        r2.close()
+        del r2
+        migration = {"from": "gpu", "to": "gpu+host (half in HBM)",
+                     "bytes_to_hbm": f_hbm, "bytes_to_host": f_host,
+                     "measured_ms": mig_s * 1e3, "predicted_makespan_ms": pred_s * 1e3}
+        return {"migration": migration,
+                "bandwidth_GBs": dict({k: v / 1e9 for k, v in bw.items() if k != "hbm_free"},
                                       host_gather_copy=bw_gather_copy / 1e9),
                 "mem_GB": {"gpu": mem_gpu / 1e9, "host": mem_host / 1e9},
                 "map_c_buf_1e6": [{"x_bytes": xx, "placement": names[c] if c < 4 else None}

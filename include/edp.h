@@ -312,6 +312,23 @@ EDP_API edp_status edp_sync(edp_ctx *ctx, edp_stream stream);
  * call on the context. */
 EDP_API const char *edp_last_error(const edp_ctx *ctx);
 
+/* Online placement migration (Sec. 5.3, Alg. 2): move the experience state
+ * of `src` into `dst`, a context created empty with the new placement --
+ * another hbm_capacity (GPU only <-> GPU + host tier) or another capacity
+ * -- and the same transform, observation shape, frame_stack, next_obs,
+ * tokens, prioritized flag, metadata arrays and device.  dst receives the
+ * newest n = min(size, dst capacity) transitions, oldest first, as if they
+ * had been its first n insertions (its total becomes n, so slots change:
+ * indices sampled from src do not apply to dst): payload rows go from
+ * their tier in src to their tier in dst (HBM or page-locked host, every
+ * direction in one launch, Appendix D), action / reward / done and
+ * priority leaves along, and the deferred and maximum priorities; dst's
+ * tree is rebuilt.  src is left unchanged.  The two must not share storage, and
+ * nothing may write src or use dst on another stream until `stream` has
+ * passed this call.  EDP_ERR_STATE when dst is not empty or the layouts
+ * differ. */
+EDP_API edp_status edp_migrate(const edp_ctx *src, edp_ctx *dst, edp_stream stream);
+
 /* Fill *out with the context's cursors and tree layout. */
 EDP_API edp_status edp_get_info(const edp_ctx *ctx, edp_info *out);
 

@@ -357,6 +357,37 @@ edp_status edp_destroy(edp_ctx *ctx) {
   return EDP_OK;
 }
 
+edp_status edp_migrate(const edp_ctx *src, edp_ctx *dst, edp_stream stream) {
+  if (!src || !dst || src == dst) return EDP_ERR_INVALID;
+  if (dst->total != 0)
+    return fail(dst, EDP_ERR_STATE, "edp_migrate: the destination must be empty");
+  const edp_config &a = src->cfg, &b = dst->cfg;
+  if (a.transform != b.transform || a.obs_c != b.obs_c || a.obs_h != b.obs_h ||
+      a.obs_w != b.obs_w || a.frame_stack != b.frame_stack || a.next_obs != b.next_obs ||
+      a.tokens != b.tokens || (a.prioritized != 0) != (b.prioritized != 0) ||
+      a.device != b.device)
+    return fail(dst, EDP_ERR_STATE,
+                "edp_migrate: source and destination differ in layout or device");
+  if ((src->st.action != nullptr) != (dst->st.action != nullptr) ||
+      (src->st.reward != nullptr) != (dst->st.reward != nullptr) ||
+      (src->st.done != nullptr) != (dst->st.done != nullptr))
+    return fail(dst, EDP_ERR_STATE, "edp_migrate: metadata arrays differ");
+  cudaSetDevice(b.device);
+  cudaStream_t s = (cudaStream_t)stream;
+  const uint64_t size = ring_size(src);
+  const uint64_t n = size < dst->cap ? size : dst->cap;
+  cudaError_t e = launch_migrate(src, dst, src->total - n, n, s);
+  if (e == cudaSuccess && dst->depth) {
+    // deferred and running-maximum priorities travel with the leaves
+    e = cudaMemcpyAsync(&dst->ctrl->pending_q, &src->ctrl->pending_q, 2 * sizeof(uint32_t),
+                        cudaMemcpyDeviceToDevice, s);
+    if (e == cudaSuccess) e = launch_tree_build_all(dst, s);
+  }
+  if (e != cudaSuccess) return cuda_fail(dst, e, "edp_migrate");
+  dst->total = n;
+  return EDP_OK;
+}
+
 edp_status edp_get_info(const edp_ctx *ctx, edp_info *o) {
   if (!ctx || !o) return EDP_ERR_INVALID;
   memset(o, 0, sizeof *o);

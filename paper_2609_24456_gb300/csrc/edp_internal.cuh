@@ -306,6 +306,10 @@ cudaError_t launch_demote(edp_ctx *ctx, uint64_t first_id, uint64_t n,
 // tokens) take their HBM slot.
 cudaError_t launch_swap(edp_ctx *ctx, uint64_t first_id, const uint8_t *obs,
                         const int32_t *tokens, uint64_t n, cudaStream_t s);
+// payload, metadata and leaves of src ids [L0, L0 + n) into dst's placement
+// as dst ids 0 .. n-1 (dst then has n insertions)
+cudaError_t launch_migrate(const edp_ctx *src, edp_ctx *dst, uint64_t L0, uint64_t n,
+                           cudaStream_t s);
 // rows [src_row, src_row + n) of an ingest source -> host-tier slots of ids
 // first_id .. first_id + n - 1
 cudaError_t launch_copy_rows_to_host(edp_ctx *ctx, const uint8_t *obs,

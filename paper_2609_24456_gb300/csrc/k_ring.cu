@@ -230,6 +230,102 @@ cudaError_t launch_swap(edp_ctx *c, uint64_t first_id, const uint8_t *obs,
   return e;
 }
 
+// ---- migration between placements (Sec. 5.3, Alg. 2) ---------------------
+// Where the payload row of logical id L lives in a ring with `total`
+// insertions: the newest min(total, cap_h) ids in HBM at L mod cap_h, older
+// ones in the host tier at L mod cap_c.
+struct TierView {
+  uint8_t *hbm;
+  uint8_t *host;
+  uint64_t cap_h, cap_c, total, row;
+};
+
+__device__ __forceinline__ uint8_t *tier_row(const TierView &v, uint64_t L) {
+  const uint64_t in_hbm = v.total < v.cap_h ? v.total : v.cap_h;
+  if (L >= v.total - in_hbm) return v.hbm + (L % v.cap_h) * v.row;
+  return v.host + (L % v.cap_c) * v.row;
+}
+
+// Rows of source ids [L0, L0 + n), renumbered 0 .. n-1 in dst, from their
+// place in src to their place in dst; every direction (HBM or host to HBM
+// or host) runs in the same launch.
+__global__ void __launch_bounds__(kCopyThreads)
+k_migrate_rows(TierView src, TierView dst, uint64_t L0, uint64_t n) {
+  const uint32_t cpr = (uint32_t)(src.row / 16);
+  for (uint64_t j = blockIdx.y; j < n; j += gridDim.y) {
+    const uint4 *s = reinterpret_cast<const uint4 *>(tier_row(src, L0 + j));
+    uint4 *d = reinterpret_cast<uint4 *>(tier_row(dst, j));
+    const uint32_t step = gridDim.x * kCopyThreads * kCopyUnroll;
+    for (uint32_t w0 = blockIdx.x * kCopyThreads * kCopyUnroll + threadIdx.x; w0 < cpr;
+         w0 += step) {
+      uint4 v[kCopyUnroll];
+#pragma unroll
+      for (int u = 0; u < kCopyUnroll; ++u) {
+        const uint32_t w = w0 + u * kCopyThreads;
+        if (w < cpr) v[u] = s[w];
+      }
+#pragma unroll
+      for (int u = 0; u < kCopyUnroll; ++u) {
+        const uint32_t w = w0 + u * kCopyThreads;
+        if (w < cpr) d[w] = v[u];
+      }
+    }
+  }
+}
+
+// Metadata and priority leaves of source ids [L0, L0 + n): slot
+// (L0 + j) mod cap_s in src, j mod cap_d in dst.
+__global__ void k_migrate_meta(const int32_t *sa, const float *sr, const uint8_t *sd,
+                               const uint32_t *sl, uint64_t cap_s, int32_t *da, float *dr,
+                               uint8_t *dd, uint32_t *dl, uint64_t cap_d, uint64_t L0,
+                               uint64_t n) {
+  for (uint64_t j = blockIdx.x * (uint64_t)blockDim.x + threadIdx.x; j < n;
+       j += (uint64_t)gridDim.x * blockDim.x) {
+    const uint64_t ms = (L0 + j) % cap_s, md = j % cap_d;
+    if (da) da[md] = sa ? sa[ms] : 0;
+    if (dr) dr[md] = sr ? sr[ms] : 0.f;
+    if (dd) dd[md] = sd ? sd[ms] : (uint8_t)0;
+    if (dl) dl[md] = sl ? sl[ms] : 0u;
+  }
+}
+
+cudaError_t migrate_payload(const TierView &s, const TierView &d, uint64_t L0, uint64_t n,
+                            cudaStream_t st) {
+  if (!n) return cudaSuccess;
+  const uint32_t cpr = (uint32_t)(s.row / 16);
+  uint32_t gx = (cpr + kCopyThreads * kCopyUnroll - 1) / (kCopyThreads * kCopyUnroll);
+  if (gx > 64) gx = 64;
+  const uint32_t gy = n < 65535 ? (uint32_t)n : 65535u;
+  k_migrate_rows<<<dim3(gx, gy), kCopyThreads, 0, st>>>(s, d, L0, n);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_migrate(const edp_ctx *src, edp_ctx *dst, uint64_t L0, uint64_t n,
+                           cudaStream_t st) {
+  TierView s{src->st.obs, src->st.host_obs, src->cap_h, src->cap_c ? src->cap_c : 1,
+             src->total, src->obs_bytes};
+  TierView d{dst->st.obs, dst->st.host_obs, dst->cap_h, dst->cap_c ? dst->cap_c : 1, n,
+             dst->obs_bytes};
+  cudaError_t e = migrate_payload(s, d, L0, n, st);
+  if (e == cudaSuccess && src->tok_bytes) {
+    s.hbm = (uint8_t *)src->st.tokens;
+    s.host = (uint8_t *)src->st.host_tokens;
+    s.row = src->tok_bytes;
+    d.hbm = (uint8_t *)dst->st.tokens;
+    d.host = (uint8_t *)dst->st.host_tokens;
+    d.row = dst->tok_bytes;
+    e = migrate_payload(s, d, L0, n, st);
+  }
+  if (e != cudaSuccess || !n) return e;
+  const int threads = 256;
+  uint64_t blocks = (n + threads - 1) / threads;
+  if (blocks > 4096) blocks = 4096;
+  k_migrate_meta<<<(unsigned)blocks, threads, 0, st>>>(
+      src->st.action, src->st.reward, src->st.done, src->leaves, src->cap, dst->st.action,
+      dst->st.reward, dst->st.done, dst->leaves, dst->cap, L0, n);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_copy_rows_to_host(edp_ctx *c, const uint8_t *obs,
                                      const int32_t *tokens, uint64_t src_row,
                                      uint64_t first_id, uint64_t n,

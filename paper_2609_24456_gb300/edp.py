@@ -126,6 +126,7 @@ SIGNATURES = {
                                    C.POINTER(C.c_uint32), _VP]),
     "edp_place_map": (C.c_int, [C.POINTER(edp_place_option), _U32, _D, _VP, _U32, _VP]),
     "edp_place_profile": (C.c_int, [C.c_int, _U64, C.POINTER(edp_place_bw)]),
+    "edp_migrate": (C.c_int, [_VP, _VP, _VP]),
 }
 
 _lib = None
@@ -429,3 +430,9 @@ def edp_place_profile(device=0, nbytes=1 << 30):
     if st != EDP_OK:
         raise EdpError(st, "edp_place_profile failed (status %d)" % st)
     return {f: getattr(out, f) for f, _ in edp_place_bw._fields_}
+
+
+def edp_migrate(src_ctx, dst_ctx, stream=None):
+    """Move src's experience state into the empty context dst (new placement)."""
+    return _check(dst_ctx, lib().edp_migrate(src_ctx, dst_ctx, stream_handle(stream)),
+                  "edp_migrate")
