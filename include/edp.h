@@ -304,6 +304,44 @@ EDP_API edp_status edp_gae(edp_ctx *ctx, const float *r, const float *v,
                    double lambda, float *adv, float *ret, float *adv_norm,
                    edp_stream stream);
 
+/* ---------------------------------------------------------------------------
+ * LLM post-training (Appendix A, Table "Verl map"): advantage computation is
+ * part of ingestion; the hand-off of variable-length sequences is delivery
+ * (Sec. 2.2 names padding / packing of variable-length sequences among the
+ * delivery operators).  Any context of the GPU serves for error reporting;
+ * its ring is not used.
+ * ------------------------------------------------------------------------- */
+
+/* Group-relative advantages (GRPO, Shao et al. 2024): responses to one prompt
+ * form a group, g = [group_off[g], group_off[g+1]); for i in g
+ *   A_i = (r_i - mean_g) / (std_g + eps),
+ * std_g the sample standard deviation (divisor n_g - 1; 0 for n_g = 1).
+ * Computed in fp64, stored fp32; A_i = 0 where std_g + eps = 0.  r, adv:
+ * device float[group_off[n_groups]]; group_off: device uint64[n_groups + 1],
+ * non-decreasing, group_off[0] = 0.  A group of equal rewards gets A = 0. */
+EDP_API edp_status edp_grpo_advantage(edp_ctx *ctx, const float *r,
+                                      const uint64_t *group_off, uint32_t n_groups,
+                                      float eps, float *adv, edp_stream stream);
+
+/* Packed delivery of variable-length sequences (the "varlen" layout):
+ * sequence s of tokens (device int32) is [seq_off[s], seq_off[s+1]),
+ * seq_off device uint64[n_seq + 1] non-decreasing.  For the batch
+ * idx[0..batch) (device int64, any order, repeats allowed):
+ *   out_off[k]  = sum_{j<k} len(idx[j])              (uint64[batch + 1])
+ *   out_tokens[out_off[k] + t] = tokens[seq_off[idx[k]] + t]
+ *   out_value[out_off[k] + t]  = seq_value[idx[k]]   (optional: a per-
+ *                       sequence value, e.g. its advantage, on every token)
+ * out_cap: elements available in out_tokens / out_value.  An index outside
+ * [0, n_seq) delivers an empty sequence; output beyond out_cap is not
+ * written; both set a device flag that edp_sync reports (EDP_ERR_INVALID;
+ * for an overflow the message gives the size needed).  batch <= 2^20. */
+EDP_API edp_status edp_pack_deliver(edp_ctx *ctx, const int32_t *tokens,
+                                    const uint64_t *seq_off, uint64_t n_seq,
+                                    const int64_t *idx, uint32_t batch,
+                                    const float *seq_value, int32_t *out_tokens,
+                                    uint64_t *out_off, float *out_value, uint64_t out_cap,
+                                    edp_stream stream);
+
 /* Wait for `stream`, then report (and clear) asynchronous CUDA errors and
  * device-side flags recorded since the previous edp_sync. */
 EDP_API edp_status edp_sync(edp_ctx *ctx, edp_stream stream);

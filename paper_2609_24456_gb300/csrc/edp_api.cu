@@ -669,6 +669,48 @@ edp_status edp_gae(edp_ctx *ctx, const float *r, const float *v,
   return EDP_OK;
 }
 
+edp_status edp_grpo_advantage(edp_ctx *ctx, const float *r, const uint64_t *group_off,
+                              uint32_t n_groups, float eps, float *adv, edp_stream stream) {
+  if (!ctx) return EDP_ERR_INVALID;
+  if (!r || !group_off || !adv || n_groups == 0)
+    return fail(ctx, EDP_ERR_INVALID, "edp_grpo_advantage: NULL array or no group");
+  if (!(eps >= 0.f) || !std::isfinite(eps))
+    return fail(ctx, EDP_ERR_INVALID, "edp_grpo_advantage: eps must be finite and >= 0");
+  const void *p;
+  const void *ptrs[] = {r, group_off, adv};
+  for (const void *o : ptrs)
+    if (!device_view(ctx, o, &p, false))
+      return fail(ctx, EDP_ERR_INVALID, "edp_grpo_advantage: arrays must be device memory");
+  cudaSetDevice(ctx->cfg.device);
+  cudaError_t e = launch_grpo(ctx, r, group_off, n_groups, eps, adv, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_grpo_advantage");
+  return EDP_OK;
+}
+
+edp_status edp_pack_deliver(edp_ctx *ctx, const int32_t *tokens, const uint64_t *seq_off,
+                            uint64_t n_seq, const int64_t *idx, uint32_t batch,
+                            const float *seq_value, int32_t *out_tokens,
+                            uint64_t *out_off, float *out_value, uint64_t out_cap,
+                            edp_stream stream) {
+  if (!ctx) return EDP_ERR_INVALID;
+  if (!tokens || !seq_off || !idx || !out_tokens || !out_off)
+    return fail(ctx, EDP_ERR_INVALID, "edp_pack_deliver: NULL array");
+  if (n_seq == 0 || batch == 0 || batch > (1u << 20))
+    return fail(ctx, EDP_ERR_INVALID, "edp_pack_deliver: need n_seq > 0, 0 < batch <= 2^20");
+  if ((seq_value == nullptr) != (out_value == nullptr))
+    return fail(ctx, EDP_ERR_INVALID, "edp_pack_deliver: seq_value and out_value go together");
+  const void *p;
+  const void *ptrs[] = {tokens, seq_off, idx, seq_value, out_tokens, out_off, out_value};
+  for (const void *o : ptrs)
+    if (o && !device_view(ctx, o, &p, false))
+      return fail(ctx, EDP_ERR_INVALID, "edp_pack_deliver: arrays must be device memory");
+  cudaSetDevice(ctx->cfg.device);
+  cudaError_t e = launch_pack(ctx, tokens, seq_off, n_seq, idx, batch, seq_value, out_tokens,
+                              out_off, out_value, out_cap, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_pack_deliver");
+  return EDP_OK;
+}
+
 edp_status edp_sync(edp_ctx *ctx, edp_stream stream) {
   if (!ctx) return EDP_ERR_INVALID;
   cudaSetDevice(ctx->cfg.device);
@@ -689,6 +731,10 @@ edp_status edp_sync(edp_ctx *ctx, edp_stream stream) {
     return fail(ctx, EDP_ERR_EMPTY, "device: total priority was 0 (flags 0x%x)", h.err);
   if (h.err & DEVERR_TREE)
     return fail(ctx, EDP_ERR_STATE, "device: inconsistent priority tree (flags 0x%x)", h.err);
+  if (h.err & DEVERR_OVERFLOW)
+    return fail(ctx, EDP_ERR_INVALID,
+                "device: packed output exceeds its capacity (needed %llu, flags 0x%x)", bi,
+                h.err);
   return fail(ctx, EDP_ERR_INVALID,
               "device: index out of range (first offender %llu, flags 0x%x)", bi, h.err);
 }

@@ -19,6 +19,7 @@ enum : uint32_t {
   DEVERR_EMPTY = 2u,    // total priority 0 at sampling time
   DEVERR_TIMEOUT = 4u,  // a bounded device-side wait expired (no kernel waits now)
   DEVERR_TREE = 8u,     // a tree descent found no child holding its target
+  DEVERR_OVERFLOW = 16u,  // packed output larger than its buffer (clipped)
 };
 
 // Small device-resident control block (one per context).
@@ -316,6 +317,13 @@ cudaError_t launch_copy_rows_to_host(edp_ctx *ctx, const uint8_t *obs,
                                      const int32_t *tokens, uint64_t src_row,
                                      uint64_t first_id, uint64_t n,
                                      cudaStream_t s);
+// LLM post-training: group-relative advantages and packed delivery
+cudaError_t launch_grpo(edp_ctx *ctx, const float *r, const uint64_t *goff, uint32_t ng,
+                        float eps, float *adv, cudaStream_t s);
+cudaError_t launch_pack(edp_ctx *ctx, const int32_t *tokens, const uint64_t *soff,
+                        uint64_t nseq, const int64_t *idx, uint32_t B, const float *sv,
+                        int32_t *otok, uint64_t *ooff, float *osv, uint64_t cap,
+                        cudaStream_t s);
 cudaError_t launch_tree_refresh(edp_ctx *ctx, uint64_t first_leaf,
                                 uint64_t count, cudaStream_t s);
 cudaError_t launch_tree_build_all(edp_ctx *ctx, cudaStream_t s);

@@ -127,6 +127,9 @@ SIGNATURES = {
     "edp_place_map": (C.c_int, [C.POINTER(edp_place_option), _U32, _D, _VP, _U32, _VP]),
     "edp_place_profile": (C.c_int, [C.c_int, _U64, C.POINTER(edp_place_bw)]),
     "edp_migrate": (C.c_int, [_VP, _VP, _VP]),
+    "edp_grpo_advantage": (C.c_int, [_VP, _VP, _VP, _U32, C.c_float, _VP, _VP]),
+    "edp_pack_deliver": (C.c_int, [_VP, _VP, _VP, _U64, _VP, _U32, _VP, _VP, _VP, _VP,
+                                   _U64, _VP]),
 }
 
 _lib = None
@@ -436,3 +439,17 @@ def edp_migrate(src_ctx, dst_ctx, stream=None):
     """Move src's experience state into the empty context dst (new placement)."""
     return _check(dst_ctx, lib().edp_migrate(src_ctx, dst_ctx, stream_handle(stream)),
                   "edp_migrate")
+
+
+def edp_grpo_advantage(ctx, r, group_off, n_groups, eps, adv, stream=None):
+    return _check(ctx, lib().edp_grpo_advantage(ctx, ptr(r), ptr(group_off), n_groups,
+                                                float(eps), ptr(adv), stream_handle(stream)),
+                  "edp_grpo_advantage")
+
+
+def edp_pack_deliver(ctx, tokens, seq_off, n_seq, idx, batch, out_tokens, out_off,
+                     out_cap, seq_value=None, out_value=None, stream=None):
+    return _check(ctx, lib().edp_pack_deliver(
+        ctx, ptr(tokens), ptr(seq_off), n_seq, ptr(idx), batch, ptr(seq_value),
+        ptr(out_tokens), ptr(out_off), ptr(out_value), out_cap, stream_handle(stream)),
+        "edp_pack_deliver")

@@ -25,6 +25,7 @@ _C_MIX1, _C_MIX2 = 0x7FEB352D, 0x2C1B3C6D
 
 # streams of the numpy generators
 S_FRAMES, S_ACTION, S_REWARD, S_DONE, S_TD, S_OBS, S_VALUE, S_TOKENS = range(8)
+S_LLM_LEN, S_LLM_TOK, S_LLM_REWARD = range(8, 11)
 
 
 def rng(seed: int, stream: int) -> np.random.Generator:
@@ -144,3 +145,25 @@ def token_fill_torch(seed: int, first_id: int, out, vocab: int = 32000):
     u = out.to(torch.int64) & M32
     out.copy_((u % vocab).to(torch.int32))
     return out
+
+
+# --- LLM post-training batch (GRPO) -------------------------------------------
+def llm_rollout(seed: int, n_prompts: int, group: int, lmin: int = 128,
+                lmax: int = 4096, vocab: int = 152064, binary_frac: float = 0.5):
+    """A GRPO batch: n_prompts groups of `group` responses with lengths
+    U[lmin, lmax] tokens, token ids U[0, vocab) (int32, packed, with uint64
+    offsets), and one reward per response: for a share binary_frac of the
+    groups 0/1 correctness ~ Bernoulli(0.4) (math RL; some groups constant),
+    for the others N(0, 1).  Returns tokens, seq_off, rewards, group_off."""
+    n = n_prompts * group
+    lens = rng(seed, S_LLM_LEN).integers(lmin, lmax + 1, size=n).astype(np.uint64)
+    seq_off = np.zeros(n + 1, np.uint64)
+    np.cumsum(lens, out=seq_off[1:])
+    tokens = rng(seed, S_LLM_TOK).integers(0, vocab, size=int(seq_off[-1]),
+                                           dtype=np.int32)
+    g = rng(seed, S_LLM_REWARD)
+    binary = g.random(n_prompts) < binary_frac
+    r = np.where(np.repeat(binary, group), (g.random(n) < 0.4).astype(np.float32),
+                 g.standard_normal(n).astype(np.float32)).astype(np.float32)
+    group_off = (np.arange(n_prompts + 1, dtype=np.uint64) * np.uint64(group))
+    return tokens, seq_off, r, group_off

@@ -1,0 +1,131 @@
+"""GPU parity of the LLM post-training operators through the C ABI:
+group-relative advantages within 1 ulp of the fp64 oracle (rounded once to
+fp32), packed delivery of variable-length sequences bit-exact (tokens,
+offsets, per-token values), including groups of one, constant groups,
+repeated and invalid indices and an output buffer that is too small, at
+small sizes and at a 512-prompt x 16-response batch."""
+import numpy as np
+import pytest
+import torch
+
+from gpu_util import bits, cuda, fx, to_np
+
+pytestmark = pytest.mark.gpu
+
+
+def _ctx(edp):
+    cfg = edp.make_config(64, (1, 16, 16), edp.EDP_XFORM_CHW_NORM_BF16)
+    return edp.Ring(cfg, action=False, reward=False, done=False)
+
+
+def _ulps(a, b):
+    a = a.view(np.int32).astype(np.int64)
+    b = b.view(np.int32).astype(np.int64)
+    return np.abs(a - b)
+
+
+def _grpo_check(edp, ring, r, goff, eps):
+    d_r, d_off = cuda(r), cuda(goff)
+    adv = torch.full((len(r),), float("nan"), device="cuda")
+    edp.edp_grpo_advantage(ring.ctx, d_r, d_off, len(goff) - 1, eps, adv)
+    edp.edp_sync(ring.ctx)
+    from oracle import llm
+    ref = llm.grpo_advantage(r, goff, eps)
+    got = to_np(adv)
+    assert _ulps(got, ref).max() <= 1
+    return got, ref
+
+
+def test_grpo_edge_groups(edp_lib):
+    edp = edp_lib
+    ring = _ctx(edp)
+    r = np.array([1, 2, 3, 5, 5, 5, 7, 0, 1, 4], np.float32)
+    goff = np.array([0, 3, 6, 7, 9, 9, 10], np.uint64)  # includes an empty group
+    got, _ = _grpo_check(edp, ring, r, goff, 0.0)
+    assert list(got[:7]) == [-1.0, 0.0, 1.0, 0.0, 0.0, 0.0, 0.0]
+    assert got[9] == 0.0  # a group of one
+    _grpo_check(edp, ring, r, goff, 1e-6)
+
+
+@pytest.mark.parametrize("group", [1, 2, 7, 16, 33, 1000])
+def test_grpo_random(edp_lib, group):
+    edp = edp_lib
+    ring = _ctx(edp)
+    _, _, r, goff = fx.llm_rollout(group, 300, group, lmin=1, lmax=2)
+    _grpo_check(edp, ring, r, goff, 1e-6)
+
+
+def _pack_check(edp, ring, tokens, seq_off, idx, value, cap=None):
+    from oracle import llm
+    ref, ref_off, ref_v = llm.pack(tokens, seq_off, idx, value)
+    cap = len(ref) if cap is None else cap
+    B = len(idx)
+    out = torch.full((max(cap, 1),), -7, dtype=torch.int32, device="cuda")
+    ov = torch.full((max(cap, 1),), float("nan"), device="cuda")
+    ooff = torch.full((B + 1,), -1, dtype=torch.int64, device="cuda")
+    d_tok, d_off, d_idx, d_v = cuda(tokens), cuda(seq_off), cuda(np.asarray(idx, np.int64)), \
+        cuda(value)
+    edp.edp_pack_deliver(ring.ctx, d_tok, d_off, len(seq_off) - 1, d_idx, B, out, ooff, cap,
+                         seq_value=d_v, out_value=ov)
+    return ref, ref_off, ref_v, out, ooff, ov
+
+
+def test_pack_small_ragged(edp_lib):
+    edp = edp_lib
+    ring = _ctx(edp)
+    tokens, seq_off, r, _ = fx.llm_rollout(4, 10, 4, lmin=0, lmax=700)  # empty ones too
+    rng = np.random.default_rng(5)
+    for B in [1, 3, 40, 1500]:
+        idx = rng.integers(0, 40, size=B)
+        ref, ref_off, ref_v, out, ooff, ov = _pack_check(edp, ring, tokens, seq_off, idx, r)
+        edp.edp_sync(ring.ctx)
+        n = len(ref)
+        assert np.array_equal(to_np(ooff).view(np.uint64), ref_off)
+        assert np.array_equal(to_np(out)[:n], ref)
+        assert np.array_equal(bits(ov)[:n], ref_v.view(np.uint32))
+
+
+def test_pack_invalid_index_and_overflow(edp_lib):
+    edp = edp_lib
+    ring = _ctx(edp)
+    tokens, seq_off, r, _ = fx.llm_rollout(6, 4, 2, lmin=5, lmax=50)
+    idx = [3, -1, 8, 2]  # -1 and 8 are outside the 8 sequences
+    ref, ref_off, ref_v, out, ooff, ov = _pack_check(edp, ring, tokens, seq_off, idx, r)
+    with pytest.raises(edp.EdpError) as e:
+        edp.edp_sync(ring.ctx)
+    assert e.value.status == edp.EDP_ERR_INVALID
+    n = len(ref)
+    assert np.array_equal(to_np(ooff).view(np.uint64), ref_off)
+    assert np.array_equal(to_np(out)[:n], ref)
+    # output buffer too small: the first `cap` elements are written, the
+    # rest are not, and the error names the size needed
+    idx = [0, 1, 2, 3, 4, 5]
+    from oracle import llm
+    full, full_off, full_v = llm.pack(tokens, seq_off, idx, r)
+    cap = len(full) - 17
+    ref, ref_off, ref_v, out, ooff, ov = _pack_check(edp, ring, tokens, seq_off, idx, r, cap)
+    with pytest.raises(edp.EdpError) as e:
+        edp.edp_sync(ring.ctx)
+    assert str(len(full)) in str(e.value)
+    assert np.array_equal(to_np(ooff).view(np.uint64), full_off)
+    assert np.array_equal(to_np(out)[:cap], full[:cap])
+    assert np.array_equal(bits(ov)[:cap], full_v[:cap].view(np.uint32))
+    edp.edp_sync(ring.ctx)  # the flag was cleared
+
+
+def test_grpo_batch_full_size(edp_lib):
+    """512 prompts x 16 responses of 128..4,096 tokens (about 17 M tokens):
+    advantages, then the whole batch delivered in a shuffled order with
+    every token carrying its response's advantage."""
+    edp = edp_lib
+    ring = _ctx(edp)
+    tokens, seq_off, r, goff = fx.llm_rollout(7, 512, 16)
+    n = len(r)
+    adv_got, adv_ref = _grpo_check(edp, ring, r, goff, 1e-6)
+    perm = np.random.default_rng(8).permutation(n)
+    ref, ref_off, ref_v, out, ooff, ov = _pack_check(edp, ring, tokens, seq_off, perm,
+                                                     adv_got)
+    edp.edp_sync(ring.ctx)
+    assert np.array_equal(to_np(ooff).view(np.uint64), ref_off)
+    assert np.array_equal(to_np(out), ref)
+    assert np.array_equal(bits(ov), ref_v.view(np.uint32))
