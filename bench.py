@@ -1339,11 +1339,143 @@ class MmReplay(Workload):
                        idx % self.hrows, MEAN3, STD3)
 
 
+class LlmBatch(Workload):
+    """GRPO post-training batch (synthetic stand-in for a DAPO-Math-style
+    rollout): 512 prompts x 16 responses of U[128, 4,096] tokens (~17.3 M
+    int32 tokens), rewards 0/1 for half the groups and N(0, 1) for the rest.
+    Step = group-relative advantages (ingestion) + the whole batch delivered
+    in a shuffled order as packed tokens with output offsets and every token
+    carrying its response's advantage (delivery)."""
+    name = "grpo-batch-512x16-128..4096tok"
+    kernel = "k_pack_gather"
+    dtype = "i32,f32 (f64 group sums)"
+    P, G = 512, 16
+
+    def __init__(self, seed=1238, perms=8):
+        self.seed, self.n_perm = seed, perms
+        from paper_2609_24456_gb300 import fixtures as fx
+        self.h_tok, self.h_off, self.h_r, self.h_goff = fx.llm_rollout(seed, self.P, self.G)
+        self.n = len(self.h_r)
+        self.T = int(self.h_off[-1])
+        n, T = self.n, self.T
+        grpo = 4 * n + 8 * (self.P + 1) + 4 * n
+        # per sequence: idx 8, offsets 16, out offset 8, value 4; per token:
+        # read 4, write 4 + 4
+        self.deliver_bytes = n * (8 + 16 + 8 + 4) + 12 * T
+        self.round_bytes = grpo + self.deliver_bytes
+        self.launches_per_round = 1 + 3
+
+    def config(self):
+        return {"workload": self.name, "prompts": self.P, "responses_per_prompt": self.G,
+                "tokens": self.T, "lengths": "U[128, 4096]",
+                "l2": "token array 69 MB in, 138 MB out per step, rotating over 2 output sets"}
+
+    def setup(self, device):
+        import numpy as np
+        import torch
+        from paper_2609_24456_gb300 import edp
+        self.edp = edp
+        cfg = edp.make_config(64, (1, 16, 16), edp.EDP_XFORM_CHW_NORM_BF16,
+                              device=device.index or 0)
+        self.ring = edp.Ring(cfg, action=False, reward=False, done=False)
+        self.tok = dev(self.h_tok, device)
+        self.off = dev(self.h_off.view(np.int64), device)
+        self.r = dev(self.h_r, device)
+        self.goff = dev(self.h_goff.view(np.int64), device)
+        self.adv = torch.empty(self.n, device=device)
+        rng = np.random.default_rng(self.seed)
+        self.h_perms = [rng.permutation(self.n).astype(np.int64) for _ in range(self.n_perm)]
+        self.perms = [dev(p, device) for p in self.h_perms]
+        self.outs = [(torch.empty(self.T, dtype=torch.int32, device=device),
+                      torch.empty(self.T, device=device),
+                      torch.empty(self.n + 1, dtype=torch.int64, device=device),
+                      torch.empty(8 * (self.n // 8 + 1), dtype=torch.int64, device=device))
+                     for _ in range(2)]
+        # tokens of each eighth of each permutation (mini-batch deliveries)
+        lens = np.diff(self.h_off.astype(np.int64))
+        self.part_tokens = [lens[p].reshape(8, -1).sum(axis=1) for p in self.h_perms]
+
+    def _grpo(self):
+        self.edp.edp_grpo_advantage(self.ring.ctx, self.r, self.goff, self.P, 1e-6, self.adv)
+
+    def _pack(self, r, parts=1):
+        """One packed delivery of the permuted batch, or `parts` (8) of its
+        mini-batches, each with its own offsets, one after the other in the
+        output."""
+        ot, ov, oo, oparts = self.outs[r % 2]
+        k = r % self.n_perm
+        if parts == 1:
+            self.edp.edp_pack_deliver(self.ring.ctx, self.tok, self.off, self.n,
+                                      self.perms[k], self.n, ot, oo, self.T,
+                                      seq_value=self.adv, out_value=ov)
+            return
+        m, done = self.n // parts, 0
+        for p in range(parts):
+            nt = int(self.part_tokens[k][p])
+            self.edp.edp_pack_deliver(self.ring.ctx, self.tok, self.off, self.n,
+                                      self.perms[k][p * m:(p + 1) * m], m,
+                                      ot[done:done + nt], oparts[p * (m + 1):(p + 1) * (m + 1)],
+                                      nt, seq_value=self.adv, out_value=ov[done:done + nt])
+            done += nt
+
+    def round(self, r):
+        self._grpo()
+        self._pack(r)
+
+    def round_parts(self, r):
+        self._grpo()
+        self._pack(r, 8)
+
+    def schedules(self):
+        return [("batched", self.round, "advantages, then one packed delivery of all "
+                 "8,192 responses (g_del = 1)"),
+                ("per-minibatch", self.round_parts, "advantages, then 8 packed deliveries "
+                 "of 1,024 responses (g_del = 1/8)")]
+
+    def deliver_once(self, r):
+        self._pack(r)
+
+    def latency_step(self, r, ev_end):
+        self._grpo()
+        self._pack(r)
+        ev_end.record()
+
+    def e2e_setup(self, device):
+        import torch
+        self.h_in = torch.from_numpy(self.h_r.copy()).pin_memory()
+        self.h_idx = [torch.from_numpy(p).pin_memory() for p in self.h_perms]
+        self.h_tok_out = torch.empty(self.T, dtype=torch.int32, pin_memory=True)
+        self.h_v_out = torch.empty(self.T, dtype=torch.float32, pin_memory=True)
+        self.h_o_out = torch.empty(self.n + 1, dtype=torch.int64, pin_memory=True)
+        self.h2d = 4 * self.n + 8 * self.n
+        self.d2h = 8 * self.T + 8 * (self.n + 1)
+
+    def e2e_round(self, r):
+        self.r.copy_(self.h_in, non_blocking=True)
+        self.perms[r % self.n_perm].copy_(self.h_idx[r % self.n_perm], non_blocking=True)
+        self.round(r)
+        ot, ov, oo, _ = self.outs[r % 2]
+        self.h_tok_out.copy_(ot, non_blocking=True)
+        self.h_v_out.copy_(ov, non_blocking=True)
+        self.h_o_out.copy_(oo, non_blocking=True)
+
+    def cpu_setup(self):
+        from oracle import llm
+        self.llm = llm
+        self.cpu_sample = "whole steps of this workload (GRPO advantages of 8,192 rewards, " \
+                          "packing of ~17.3 M tokens)"
+
+    def cpu_round(self, r):
+        adv = self.llm.grpo_advantage(self.h_r, self.h_goff, 1e-6)
+        self.llm.pack(self.h_tok, self.h_off, self.h_perms[r % self.n_perm], adv)
+
+
 WORKLOADS = {
     "per1m": PerReplay,
     "dqn10k": DqnTiny,
     "ppo": PpoIteration,
     "mm200k": MmReplay,
+    "grpo": LlmBatch,
     # two-tier: 800,000 transitions (the 1.6M of the full configuration scaled
     # to the GPU box's host memory), newest half in HBM, 4,096 ingested per step
     "tiered": lambda **kw: MmReplay(capacity=kw.get("capacity") or 800_000,

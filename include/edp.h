@@ -27,9 +27,10 @@
  *   when NULL) and released by edp_destroy.  libedp never frees caller memory.
  *   Scratch is allocated at a call's first use and grown (after a device
  *   synchronisation) when a later call needs more: edp_update_priorities_td
- *   (4 bytes per pair), the PERMUTE sampling mode and edp_gae with
- *   normalisation.  Before capturing calls into a CUDA graph, make each of
- *   them once at its largest size, outside the capture.
+ *   (4 bytes per pair), the PERMUTE sampling mode, edp_gae with
+ *   normalisation and edp_pack_deliver (16 bytes per batch entry).  Before
+ *   capturing calls into a CUDA graph, make each of them once at its
+ *   largest size, outside the capture.
  * - Asynchrony: every call validates its arguments on the host, enqueues its
  *   kernels on `stream` and returns without synchronising.  Results are
  *   valid once the stream has reached that point.  Host-side cursors
@@ -47,7 +48,7 @@
  *   a captured graph, the order at capture): deliveries that run at the
  *   same time must have been issued fewer than 32 deliveries apart.
  *   edp_gae likewise may overlap edp_sample (GAE scratch and shuffle
- *   scratch are separate).  Every other pair of calls on one context shares
+ *   scratch are separate); edp_gae and edp_pack_deliver share scratch.  Every other pair of calls on one context shares
  *   the priority tree or the context's scratch and must be ordered.
  * - Errors: argument and state errors are returned synchronously and leave
  *   the context unchanged.  A CUDA launch error returns EDP_ERR_CUDA.

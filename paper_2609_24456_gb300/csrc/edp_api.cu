@@ -707,6 +707,8 @@ edp_status edp_pack_deliver(edp_ctx *ctx, const int32_t *tokens, const uint64_t 
   cudaSetDevice(ctx->cfg.device);
   cudaError_t e = launch_pack(ctx, tokens, seq_off, n_seq, idx, batch, seq_value, out_tokens,
                               out_off, out_value, out_cap, (cudaStream_t)stream);
+  if (e == cudaErrorMemoryAllocation)
+    return fail(ctx, EDP_ERR_OOM, "edp_pack_deliver: scratch allocation failed");
   if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_pack_deliver");
   return EDP_OK;
 }
