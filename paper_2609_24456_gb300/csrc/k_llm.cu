@@ -4,10 +4,10 @@
 // with a per-sequence value broadcast to their tokens.
 //
 // Advantages: one warp per group; fp64 sums of r and of (r - mean)^2 (two
-// passes), one rounding to fp32 per output.  Packing: the batch's sequence
-// lengths with each entry's source start and value (one thread each, into
-// the context's scratch), a one-CTA scan of the lengths into the output
-// offsets, then one CTA per sequence copies its tokens (4-byte loads and stores: neither the source
+// passes), one rounding to fp32 per output.  Packing: each batch entry's
+// source start, length and value (one thread each, into the context's
+// scratch) with per-CTA length sums turned into prefixes by the last CTA,
+// then one CTA per sequence forms its output offset and copies its tokens (4-byte loads and stores: neither the source
 // nor the destination offset is aligned to more than a token) and writes
 // the value beside each token.  Both copy kernels are HBM-bound.
 #include "edp_internal.cuh"
@@ -18,8 +18,6 @@ namespace {
 constexpr unsigned kFull = 0xffffffffu;
 constexpr int kGrpoThreads = 256;
 constexpr int kGrpoWarps = kGrpoThreads / 32;
-constexpr int kScanThreads = 1024;
-constexpr int kScanPer = 8;
 constexpr int kPackThreads = 256;
 constexpr int kPackUnroll = 8;
 
@@ -57,118 +55,132 @@ k_grpo(const float *__restrict__ r, const uint64_t *__restrict__ goff, uint32_t 
 }
 
 // What the copy of batch entry k needs, resolved once: where its tokens
-// start and the value its tokens carry.
+// start, how many there are, and the value they carry.
 struct PackEntry {
   uint64_t src;
   float value;
-  uint32_t pad;
+  uint32_t len;
 };
 
-// Lengths of the batch's sequences, one thread per entry: out_off[k + 1] =
-// len(idx[k]) (0 and a flag for an index out of range); out_off[0] = 0; and
-// entry k's source start and value.
+__device__ __forceinline__ uint64_t block_sum(uint64_t v, uint64_t *red) {
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+#pragma unroll
+  for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
+  __syncthreads();  // red may still be read by a previous call
+  if (lane == 0) red[wid] = v;
+  __syncthreads();
+  uint64_t t = 0;
+#pragma unroll
+  for (int w = 0; w < kPackThreads / 32; ++w) t += red[w];
+  return t;
+}
+
+// One thread per batch entry: its entry (0 tokens and a flag for an index
+// out of range); per CTA the sum of its 256 lengths.  The last CTA to finish
+// (a ticket on the launch's work counter) turns those sums into exclusive
+// prefixes, writes out_off[batch] = the total and resets the counter.
 __global__ void __launch_bounds__(kPackThreads)
 k_pack_lengths(const uint64_t *__restrict__ soff, uint64_t nseq,
                const int64_t *__restrict__ idx, uint32_t B, const float *__restrict__ sv,
-               uint64_t *__restrict__ ooff, PackEntry *__restrict__ ent, Ctrl *ctrl) {
+               PackEntry *__restrict__ ent, uint64_t *__restrict__ part,
+               uint64_t *__restrict__ pre, uint64_t *__restrict__ ooff, uint64_t cap,
+               uint32_t *work, Ctrl *ctrl) {
+  __shared__ uint64_t red[kPackThreads / 32];
+  __shared__ uint32_t ticket;
   pdl_wait();
   pdl_launch();
   const uint64_t k = (uint64_t)blockIdx.x * kPackThreads + threadIdx.x;
-  if (k == 0) ooff[0] = 0;
-  if (k >= B) return;
-  const int64_t s = idx[k];
-  uint64_t len = 0, a = 0;
-  float value = 0.f;
-  if (s >= 0 && (uint64_t)s < nseq) {
-    a = soff[s];
-    const uint64_t b = soff[s + 1];
-    len = b > a ? b - a : 0;
-    if (sv) value = sv[s];
-  } else {
-    flag(ctrl, DEVERR_INDEX, (unsigned long long)s);
+  uint64_t len = 0;
+  if (k < B) {
+    const int64_t s = idx[k];
+    uint64_t a = 0;
+    float value = 0.f;
+    if (s >= 0 && (uint64_t)s < nseq) {
+      a = soff[s];
+      const uint64_t b = soff[s + 1];
+      len = b > a ? b - a : 0;
+      if (sv) value = sv[s];
+    } else {
+      flag(ctrl, DEVERR_INDEX, (unsigned long long)s);
+    }
+    ent[k] = PackEntry{a, value, (uint32_t)len};
   }
-  ooff[k + 1] = len;
-  ent[k] = PackEntry{a, value, 0u};
-}
-
-// In-place inclusive scan of out_off[1 .. B] in one CTA, in tiles of
-// kScanThreads x kScanPer entries (each thread's entries loaded together):
-// out_off[k] becomes the sum of the first k lengths.
-__global__ void __launch_bounds__(kScanThreads)
-k_pack_scan(uint32_t B, uint64_t *__restrict__ ooff, uint64_t cap, Ctrl *ctrl) {
-  __shared__ uint64_t wsum[kScanThreads / 32];
-  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-  pdl_wait();
-  pdl_launch();
-  uint64_t *len = ooff + 1;
+  const uint64_t sum = block_sum(len, red);
+  if (threadIdx.x == 0) {
+    part[blockIdx.x] = sum;
+    __threadfence();
+    ticket = atomicAdd(&work[0], 1u);
+  }
+  __syncthreads();
+  if (ticket != gridDim.x - 1) return;
+  __threadfence();
+  // the last CTA: exclusive prefix of the per-CTA sums, kPackThreads at a time
   uint64_t carry = 0;
-  for (uint64_t base = 0; base < B; base += (uint64_t)kScanThreads * kScanPer) {
-    const uint64_t k0 = base + (uint64_t)threadIdx.x * kScanPer;
-    uint64_t v[kScanPer];
-#pragma unroll
-    for (int u = 0; u < kScanPer; ++u) v[u] = k0 + u < B ? len[k0 + u] : 0;
-    uint64_t mine = 0;
-#pragma unroll
-    for (int u = 0; u < kScanPer; ++u) mine += v[u];
-    uint64_t incl = mine;
+  for (uint32_t base = 0; base < gridDim.x; base += kPackThreads) {
+    const uint32_t i = base + threadIdx.x;
+    const uint64_t v = i < gridDim.x ? __ldcg(&part[i]) : 0;
+    uint64_t incl = v;
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
       const uint64_t t = __shfl_up_sync(kFull, incl, o);
       if (lane >= o) incl += t;
     }
-    if (lane == 31) wsum[wid] = incl;
     __syncthreads();
-    if (wid == 0) {
-      uint64_t w = wsum[lane];
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const uint64_t t = __shfl_up_sync(kFull, w, o);
-        if (lane >= o) w += t;
-      }
-      wsum[lane] = w;  // inclusive prefix over warps
-    }
+    if (lane == 31) red[wid] = incl;
     __syncthreads();
-    uint64_t run = carry + incl - mine + (wid ? wsum[wid - 1] : 0);
+    uint64_t before = carry;
+    for (int w = 0; w < wid; ++w) before += red[w];
+    if (i < gridDim.x) pre[i] = before + incl - v;
+    uint64_t tile = 0;
 #pragma unroll
-    for (int u = 0; u < kScanPer; ++u) {
-      run += v[u];
-      if (k0 + u < B) len[k0 + u] = run;
-    }
-    carry += wsum[31];
-    __syncthreads();  // wsum is rewritten by the next tile
+    for (int w = 0; w < kPackThreads / 32; ++w) tile += red[w];
+    carry += tile;
   }
-  if (threadIdx.x == 0 && carry > cap) flag(ctrl, DEVERR_OVERFLOW, (unsigned long long)carry);
+  if (threadIdx.x == 0) {
+    ooff[B] = carry;
+    if (carry > cap) flag(ctrl, DEVERR_OVERFLOW, (unsigned long long)carry);
+    work[0] = 0u;  // every CTA has taken its ticket
+  }
 }
 
-// One CTA per sequence: one round trip for the entry and its offsets, then
-// a thread keeps kPackUnroll loads in flight (2,048 tokens per CTA pass).
+// One CTA per sequence: its output offset is the prefix of its 256-entry
+// chunk plus the lengths before it in the chunk (one round trip and a block
+// sum), then a thread keeps kPackUnroll loads in flight (2,048 tokens per
+// CTA pass).
 __global__ void __launch_bounds__(kPackThreads)
 k_pack_gather(const int32_t *__restrict__ tokens, const PackEntry *__restrict__ ent,
-              uint32_t B, int32_t *__restrict__ otok, const uint64_t *__restrict__ ooff,
-              float *__restrict__ osv, uint64_t cap) {
+              const uint64_t *__restrict__ pre, uint32_t B, int32_t *__restrict__ otok,
+              uint64_t *__restrict__ ooff, float *__restrict__ osv, uint64_t cap) {
+  __shared__ uint64_t red[kPackThreads / 32];
   const uint64_t pol = policy_stream();
   pdl_wait();
   pdl_launch();
   for (uint32_t k = blockIdx.x; k < B; k += gridDim.x) {
+    const uint32_t c0 = k / kPackThreads * kPackThreads;
+    const uint32_t j = c0 + threadIdx.x;
+    uint64_t v = j < k ? ent[j].len : 0;
+    if (threadIdx.x == 0) v += pre[k / kPackThreads];
     const PackEntry e = ent[k];
-    const uint64_t dst = ooff[k], end = ooff[k + 1];
-    if (end <= dst || dst >= cap) continue;
-    const uint64_t n = min(end - dst, cap - dst);
+    const uint64_t dst = block_sum(v, red);
+    if (threadIdx.x == 0) ooff[k] = dst;
+    if (e.len == 0 || dst >= cap) continue;
+    const uint64_t n = min((uint64_t)e.len, cap - dst);
     const int32_t *src = tokens + e.src;
     int32_t *out = otok + dst;
     for (uint64_t t0 = threadIdx.x; t0 < n; t0 += kPackThreads * kPackUnroll) {
-      int32_t v[kPackUnroll];
+      int32_t w[kPackUnroll];
 #pragma unroll
       for (int u = 0; u < kPackUnroll; ++u) {
         const uint64_t t = t0 + u * kPackThreads;
-        v[u] = t < n ? (int32_t)ld_stream(reinterpret_cast<const uint32_t *>(src + t), pol)
+        w[u] = t < n ? (int32_t)ld_stream(reinterpret_cast<const uint32_t *>(src + t), pol)
                      : 0;
       }
 #pragma unroll
       for (int u = 0; u < kPackUnroll; ++u) {
         const uint64_t t = t0 + u * kPackThreads;
         if (t < n) {
-          out[t] = v[u];
+          out[t] = w[u];
           if (osv) osv[dst + t] = e.value;
         }
       }
@@ -190,16 +202,20 @@ cudaError_t launch_pack(edp_ctx *c, const int32_t *tokens, const uint64_t *soff,
                         uint64_t nseq, const int64_t *idx, uint32_t B, const float *sv,
                         int32_t *otok, uint64_t *ooff, float *osv, uint64_t cap,
                         cudaStream_t s) {
-  PackEntry *ent = (PackEntry *)ctx_scratch(c, (size_t)B * sizeof(PackEntry));
-  if (!ent) return cudaErrorMemoryAllocation;
-  cudaError_t e = launch_pdl(k_pack_lengths, dim3((B + kPackThreads - 1) / kPackThreads),
-                             dim3(kPackThreads), s, soff, nseq, idx, B, sv, ooff, ent, c->ctrl);
-  if (e == cudaSuccess)
-    e = launch_pdl(k_pack_scan, dim3(1), dim3(kScanThreads), s, B, ooff, cap, c->ctrl);
+  const uint32_t G = (B + kPackThreads - 1) / kPackThreads;
+  const size_t ent_bytes = ((size_t)B * sizeof(PackEntry) + 255) & ~(size_t)255;
+  uint8_t *scr = (uint8_t *)ctx_scratch(c, ent_bytes + 2 * (size_t)G * sizeof(uint64_t));
+  if (!scr) return cudaErrorMemoryAllocation;
+  PackEntry *ent = (PackEntry *)scr;
+  uint64_t *part = (uint64_t *)(scr + ent_bytes);
+  uint64_t *pre = part + G;
+  uint32_t *work = c->ctrl->work + 2 * (c->work_seq++ % kWorkSlots);
+  cudaError_t e = launch_pdl(k_pack_lengths, dim3(G), dim3(kPackThreads), s, soff, nseq, idx,
+                             B, sv, ent, part, pre, ooff, cap, work, c->ctrl);
   if (e != cudaSuccess) return e;
   const unsigned grid = B < 65535u * 16u ? B : 65535u * 16u;
   return launch_pdl(k_pack_gather, dim3(grid), dim3(kPackThreads), s, tokens,
-                    (const PackEntry *)ent, B, otok, (const uint64_t *)ooff, osv, cap);
+                    (const PackEntry *)ent, (const uint64_t *)pre, B, otok, ooff, osv, cap);
 }
 
 }  // namespace edp
