@@ -579,12 +579,21 @@ class DqnTiny(Workload):
                             self.seed, r, o["idx"])
         self.edp.edp_deliver(self.ring.ctx, o["idx"], self.B, o["batch"])
 
+    def round_fused(self, r):
+        o = self.outs[r % self.R]
+        self.edp.edp_sample_deliver(self.ring.ctx, self.B, self.seed, r, o["idx"], o["batch"])
+
+    def schedules(self):
+        return [("fused", self.round_fused, "uniform draw inside the delivery kernel "
+                 "(edp_sample_deliver), one launch per batch"),
+                ("sample+deliver", self.round, "edp_sample then edp_deliver, one stream")]
+
     def deliver_once(self, r):
         o = self.outs[r % self.R]
         self.edp.edp_deliver(self.ring.ctx, o["idx"], self.B, o["batch"])
 
     def latency_step(self, r, ev_end):
-        self.round(r)
+        self.round_fused(r)
         ev_end.record()
 
     def e2e_setup(self, device):
@@ -1087,11 +1096,32 @@ class MmReplay(Workload):
             lambda st: self.edp.edp_deliver(self.ring.ctx, o["idx"], self.B, o["batch"],
                                             stream=st))
 
+    def round_fused(self, r):
+        """Fused sample -> deliver calls alternating between two side
+        streams: output set k is always written from side stream k, so
+        stream order protects its reuse; consecutive batches overlap."""
+        import torch
+        k = r % 2
+        o = self.outs[k]
+        side = self.sides[k]
+        if not self.side_used:
+            self.fork_ev = torch.cuda.Event()
+            self.fork_ev.record()
+            for st in self.sides:
+                st.wait_event(self.fork_ev)
+        self.side_used = True
+        with torch.cuda.stream(side):
+            self.edp.edp_sample_deliver(self.ring.ctx, self.B, self.seed, r, o["idx"],
+                                        o["batch"], stream=side)
+
     def schedules(self):
         one = ("one stream", self.round, "sample -> deliver, one stream")
         if self.ingest:
             return [one]
-        return [("overlapped", self.round_overlap,
+        return [("fused overlapped", self.round_fused,
+                 "uniform draw inside the delivery kernel (edp_sample_deliver), "
+                 "calls alternating between two side streams"),
+                ("overlapped", self.round_overlap,
                  "delivery on side streams, overlapping sampling r+1"), one]
 
     def deliver_once(self, r):
@@ -1100,9 +1130,7 @@ class MmReplay(Workload):
 
     def latency_step(self, r, ev_end):
         o = self.outs[r % 2]
-        self.edp.edp_sample(self.ring.ctx, self.edp.EDP_SAMPLE_UNIFORM, self.B,
-                            self.seed, r, o["idx"])
-        self.edp.edp_deliver(self.ring.ctx, o["idx"], self.B, o["batch"])
+        self.edp.edp_sample_deliver(self.ring.ctx, self.B, self.seed, r, o["idx"], o["batch"])
         ev_end.record()
 
     def e2e_setup(self, device):

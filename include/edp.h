@@ -235,7 +235,8 @@ EDP_API edp_status edp_destroy(edp_ctx *ctx);
 EDP_API edp_status edp_ingest(edp_ctx *ctx, const edp_fields *src, uint64_t n,
                       const uint32_t *q, edp_stream stream);
 
-/* Sampling (Sec. 2.2 delivery "select").  Writes idx (device int64 [batch])
+/* Sampling (Sec. 2.2: choosing which stored transitions a batch holds).
+ * Writes idx (device int64 [batch])
  * and, for PRIORITIZED, q (device uint32 [batch], may be NULL) = the sampled
  * leaves.  Errors: EDP_ERR_EMPTY when no transition is sampleable;
  * EDP_ERR_STATE for PRIORITIZED without a tree; EDP_ERR_INVALID when
@@ -244,12 +245,23 @@ EDP_API edp_status edp_sample(edp_ctx *ctx, edp_sample_mode mode, uint32_t batch
                       uint64_t seed, uint64_t round, int64_t *idx,
                       uint32_t *q, edp_stream stream);
 
-/* Delivery (Sec. 2.2 "materializes the selected transitions and performs
- * batch/layout transformations"): fused gather + transform + collate (+ IS
+/* Delivery (Sec. 2.2: the chosen transitions are materialised in the
+ * learner's batch layout): fused gather + transform + collate (+ IS
  * weights) of the `batch` slots in idx (device int64).  A slot outside the
  * sampleable range is reported by edp_sync and its outputs are zeroed. */
 EDP_API edp_status edp_deliver(edp_ctx *ctx, const int64_t *idx, uint32_t batch,
                        const edp_batch *out, edp_stream stream);
+
+/* Fused uniform sample -> deliver: the UNIFORM draw of edp_sample (same seed,
+ * round, indices) made inside the delivery kernel, one launch instead of
+ * two.  idx (device int64 [batch]) receives the drawn slots; out as for
+ * edp_deliver, without q / isw (uniform draws carry no priorities:
+ * EDP_ERR_INVALID).  EDP_ERR_EMPTY when no transition is sampleable; other
+ * errors as edp_deliver.  Prioritized sampling keeps its own kernel, whose
+ * tree descents every delivery warp would otherwise repeat. */
+EDP_API edp_status edp_sample_deliver(edp_ctx *ctx, uint32_t batch, uint64_t seed,
+                                      uint64_t round, int64_t *idx, const edp_batch *out,
+                                      edp_stream stream);
 
 /* Priority callback (Appendix C, Invariant 2; PER).  Sets the priority of
  * each (idx[p], q[p]); for a repeated slot the last pair wins.  Pairs whose

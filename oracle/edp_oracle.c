@@ -202,7 +202,7 @@ ORC_API void orc_priorities_from_td(const float *td, uint64_t n, double alpha,
 }
 
 /* ------------------------------------------------------------------------ */
-/* Samplers (Sec. 2.2: delivery "samples from a persistent replay dataset"). */
+/* Samplers (Sec. 2.2: off-policy delivery draws from the stored replay data). */
 /* ------------------------------------------------------------------------ */
 
 /* Uniform with replacement over the first n_valid logical offsets:
@@ -327,8 +327,8 @@ ORC_API uint16_t orc_norm_bf16(uint8_t b, float mean, float stdv) {
 }
 
 /* ------------------------------------------------------------------------ */
-/* Frame-stack delivery (Sec. 2.2: delivery "materializes the selected       */
-/* transitions and performs concatenation and reshaping"; frame stacking of  */
+/* Frame-stack delivery (Sec. 2.2: delivery materialises the chosen          */
+/* transitions, concatenating and reshaping them; frame stacking of          */
 /* Mnih et al., Nature 2015).  Readings:                                     */
 /*  - obs(i) = [f(i-K+1), ..., f(i)] over logical predecessors; f(j) is an   */
 /*    all-zero frame when j precedes the oldest stored transition or when    */

@@ -550,9 +550,9 @@ edp_status edp_sample(edp_ctx *ctx, edp_sample_mode mode, uint32_t batch,
   return EDP_OK;
 }
 
-edp_status edp_deliver(edp_ctx *ctx, const int64_t *idx, uint32_t batch,
-                       const edp_batch *out, edp_stream stream) {
-  if (!ctx) return EDP_ERR_INVALID;
+// Argument checks shared by edp_deliver and edp_sample_deliver.
+static edp_status deliver_checks(edp_ctx *ctx, const int64_t *idx, uint32_t batch,
+                                 const edp_batch *out) {
   if (!idx || !out || !out->obs)
     return fail(ctx, EDP_ERR_INVALID, "edp_deliver: idx/out/out->obs is NULL");
   if (batch == 0) return fail(ctx, EDP_ERR_INVALID, "edp_deliver: batch == 0");
@@ -585,9 +585,34 @@ edp_status edp_deliver(edp_ctx *ctx, const int64_t *idx, uint32_t batch,
   if (!aligned16(out->obs) || (out->next_obs && !aligned16(out->next_obs)) ||
       (out->tokens && !aligned16(out->tokens)))
     return fail(ctx, EDP_ERR_INVALID, "edp_deliver: obs/next_obs/tokens 16-B aligned");
+  return EDP_OK;
+}
+
+edp_status edp_deliver(edp_ctx *ctx, const int64_t *idx, uint32_t batch,
+                       const edp_batch *out, edp_stream stream) {
+  if (!ctx) return EDP_ERR_INVALID;
+  const edp_status st = deliver_checks(ctx, idx, batch, out);
+  if (st != EDP_OK) return st;
   cudaSetDevice(ctx->cfg.device);
   cudaError_t e = launch_deliver(ctx, idx, batch, out, (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_deliver");
+  return EDP_OK;
+}
+
+edp_status edp_sample_deliver(edp_ctx *ctx, uint32_t batch, uint64_t seed, uint64_t round,
+                              int64_t *idx, const edp_batch *out, edp_stream stream) {
+  if (!ctx) return EDP_ERR_INVALID;
+  if (n_valid(ctx) == 0)
+    return fail(ctx, EDP_ERR_EMPTY, "edp_sample_deliver: no sampleable transition");
+  if (out && (out->isw || out->q))
+    return fail(ctx, EDP_ERR_INVALID,
+                "edp_sample_deliver: uniform draws carry no priorities (q/isw must be NULL)");
+  const edp_status st = deliver_checks(ctx, idx, batch, out);
+  if (st != EDP_OK) return st;
+  cudaSetDevice(ctx->cfg.device);
+  DrawUniform d{seed, round, idx};
+  cudaError_t e = launch_deliver(ctx, idx, batch, out, (cudaStream_t)stream, &d);
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_sample_deliver");
   return EDP_OK;
 }
 

@@ -317,6 +317,15 @@ cudaError_t launch_copy_rows_to_host(edp_ctx *ctx, const uint8_t *obs,
                                      const int32_t *tokens, uint64_t src_row,
                                      uint64_t first_id, uint64_t n,
                                      cudaStream_t s);
+// Delivery.  With `draw`, the batch is drawn by the uniform sampler inside
+// the delivery kernel (idx unused; draw->idx_out receives the indices).
+struct DrawUniform {
+  uint64_t seed, round;
+  int64_t *idx_out;
+};
+cudaError_t launch_deliver(edp_ctx *ctx, const int64_t *idx, uint32_t B,
+                           const edp_batch *out, cudaStream_t s,
+                           const DrawUniform *draw = nullptr);
 // LLM post-training: group-relative advantages and packed delivery
 cudaError_t launch_grpo(edp_ctx *ctx, const float *r, const uint64_t *goff, uint32_t ng,
                         float eps, float *adv, cudaStream_t s);
@@ -339,8 +348,6 @@ cudaError_t launch_update(edp_ctx *ctx, const int64_t *idx, const uint32_t *q,
                           cudaStream_t s);
 cudaError_t launch_prio_from_td(const float *td, uint32_t n, double alpha,
                                 double eps, uint32_t *q, cudaStream_t s);
-cudaError_t launch_deliver(edp_ctx *ctx, const int64_t *idx, uint32_t B,
-                           const edp_batch *out, cudaStream_t s);
 cudaError_t launch_gae(edp_ctx *ctx, const float *r, const float *v,
                        const uint8_t *d, uint32_t T, uint32_t E, double gamma,
                        double lambda, float *adv, float *ret, float *adv_norm,

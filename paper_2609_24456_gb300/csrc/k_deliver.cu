@@ -57,12 +57,26 @@ struct Common {
   Ctrl *ctrl;
   uint32_t *work;  // this launch's work counter pair, or null (one chunk per CTA)
   float r1, r2;
+  // fused uniform sampling: idx is then an output, sample k is drawn here
+  int draw;
+  uint64_t seed, round;
+  int64_t *idx_out;
 };
 
 // Resolve slot -> logical offset; false (and a flag) when not sampleable.
 __device__ __forceinline__ bool sample_slot(const Common &c, uint32_t k,
                                             uint64_t *slot, uint64_t *off,
                                             bool report) {
+  if (c.draw) {
+    // the uniform sampler's draw (Philox stream 0), made where it is used;
+    // the warp that delivers the sample's first unit writes its index
+    const uint64_t o = mulhi64(philox_u64(c.seed, k, c.round, 0), c.nvalid);
+    const uint64_t t = c.oldest + o;
+    *slot = t >= c.cap ? t - c.cap : t;
+    *off = o;
+    if (report) c.idx_out[k] = (int64_t)*slot;
+    return true;
+  }
   const int64_t s = c.idx[k];
   if (s < 0 || (uint64_t)s >= c.cap) {
     if (report) flag(c.ctrl, DEVERR_INDEX, (unsigned long long)s);
@@ -481,9 +495,15 @@ unsigned grid_for(Kern kern, uint64_t units, uint64_t per_iter, int iters, int s
 }  // namespace
 
 cudaError_t launch_deliver(edp_ctx *ctx, const int64_t *idx, uint32_t B,
-                           const edp_batch *out, cudaStream_t s) {
+                           const edp_batch *out, cudaStream_t s, const DrawUniform *draw) {
   Common c{};
   c.idx = idx;
+  if (draw) {
+    c.draw = 1;
+    c.seed = draw->seed;
+    c.round = draw->round;
+    c.idx_out = draw->idx_out;
+  }
   c.B = B;
   c.cap = ctx->cap;
   const uint64_t size = ctx->total < ctx->cap ? ctx->total : ctx->cap;

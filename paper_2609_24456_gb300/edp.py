@@ -108,6 +108,7 @@ SIGNATURES = {
     "edp_ingest": (C.c_int, [_VP, C.POINTER(edp_fields), _U64, _VP, _VP]),
     "edp_sample": (C.c_int, [_VP, C.c_int, _U32, _U64, _U64, _VP, _VP, _VP]),
     "edp_deliver": (C.c_int, [_VP, _VP, _U32, C.POINTER(edp_batch), _VP]),
+    "edp_sample_deliver": (C.c_int, [_VP, _U32, _U64, _U64, _VP, C.POINTER(edp_batch), _VP]),
     "edp_update_priorities": (C.c_int, [_VP, _VP, _VP, _U32, _VP]),
     "edp_update_priorities_td": (C.c_int, [_VP, _VP, _VP, _U32, _D, _D, _VP]),
     "edp_update_priorities_td_static": (C.c_int, [_VP, _VP, _VP, _U32, _D, _D, _VP]),
@@ -220,6 +221,12 @@ def make_batch(obs, next_obs=None, action=None, reward=None, done=None,
         b.gather_src[i] = ptr(src)
         b.gather_dst[i] = ptr(dst)
     return b
+
+
+def edp_sample_deliver(ctx, batch, seed, round_, idx, out: edp_batch, stream=None):
+    return _check(ctx, lib().edp_sample_deliver(ctx, batch, seed, round_, ptr(idx),
+                                                C.byref(out), stream_handle(stream)),
+                  "edp_sample_deliver")
 
 
 def edp_deliver(ctx, idx, batch, out: edp_batch, stream=None):
