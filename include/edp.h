@@ -303,9 +303,9 @@ EDP_API edp_status edp_priorities_from_td(edp_ctx *ctx, const float *td, uint32_
                                   double alpha, double eps, uint32_t *q,
                                   edp_stream stream);
 
-/* Generalized advantage estimation (Schulman et al., ICLR'16) -- the
- * "computing returns/advantages" and "normalization" of on-policy ingestion
- * (Sec. 2.2).  Device arrays, time-major: r, d [T][E]; v [T+1][E].
+/* Generalized advantage estimation (Schulman et al., ICLR'16) -- the return
+ * and advantage computation and their normalisation, steps of on-policy
+ * ingestion (Sec. 2.2).  Device arrays, time-major: r, d [T][E]; v [T+1][E].
  *   delta_t = r_t + gamma V_{t+1} (1 - d_t) - V_t
  *   A_t = delta_t + gamma lambda (1 - d_t) A_{t+1},  A_T = 0
  *   ret_t = A_t + V_t

@@ -447,9 +447,9 @@ ORC_API void orc_deliver_mm(const uint8_t *obs_ring, const int32_t *tok_ring,
 }
 
 /* ------------------------------------------------------------------------ */
-/* Generalized advantage estimation (Schulman et al., ICLR'16), the          */
-/* "computing returns/advantages" and "normalization" steps of on-policy     */
-/* ingestion (Sec. 2.2).  Direct-sum definition, fp64:                       */
+/* Generalized advantage estimation (Schulman et al., ICLR'16), the return  */
+/* / advantage and normalisation steps of on-policy ingestion (Sec. 2.2).    */
+/* Direct-sum definition, fp64:                                              */
 /*   delta_t = r_t + gamma V_{t+1} (1 - d_t) - V_t                           */
 /*   A_t = sum_{l >= 0, t+l < T} (gamma lambda)^l prod_{m<l}(1 - d_{t+m})    */
 /*         delta_{t+l}                                                       */

@@ -1,6 +1,6 @@
 // k_gae.cu -- generalized advantage estimation with global advantage
-// normalisation (Schulman et al., ICLR'16; the "computing returns/advantages"
-// and "normalization" steps of on-policy ingestion, Sec. 2.2).
+// normalisation (Schulman et al., ICLR'16; the return / advantage and
+// normalisation steps of on-policy ingestion, Sec. 2.2).
 //
 //   delta_t = r_t + gamma V_{t+1} (1 - d_t) - V_t
 //   A_t = delta_t + c_t A_{t+1},  c_t = gamma lambda (1 - d_t),  A_T = 0
