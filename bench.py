@@ -225,6 +225,7 @@ class Workload:
         self.ready = [torch.cuda.Event() for _ in range(sets)]
         self.consumed = [torch.cuda.Event() for _ in range(sets)]
         self.in_flight = set()  # output sets whose delivery is not yet joined
+        self.side_used = False
 
     def _overlapped(self, k, sample, deliver, after=None):
         """One round with its delivery on a side stream: sample() on the
