@@ -69,3 +69,29 @@ def test_concurrent_and_repeated_counter_deliveries(edp_lib, orc):
     for o in outs[2:]:
         for x, y in zip(ref, o):
             assert np.array_equal(x, bits(y) if y.is_floating_point() else to_np(y))
+
+
+@pytest.mark.parametrize("B", [37, 1024])
+def test_outputs_16_byte_aligned_only(edp_lib, orc, B):
+    """Outputs 16 bytes past a 32-byte boundary (the alignment the ABI
+    requires, and no more) give the same batches as aligned ones, on the
+    one-chunk-per-CTA and the counter paths."""
+    edp = edp_lib
+    frames, action, reward, done = fx.dqn_transitions(42, N_INGEST, done_p=0.05)
+    m = MirroredDqn(CAP)
+    m.ingest(orc, frames, action, reward, done)
+    idx = torch.empty(B, dtype=torch.int64, device="cuda")
+    edp.edp_sample(m.ring.ctx, edp.EDP_SAMPLE_UNIFORM, B, 43, 0, idx)
+    n = B * 4 * m.F
+    aligned = dqn_outputs(B, m.K, m.F)
+    # each output 16 bytes past a fresh (256-byte aligned) allocation
+    obs = torch.full((n + 4,), float("nan"), device="cuda")[4:].view(B, 4, m.F)
+    nxt = torch.full((n + 4,), float("nan"), device="cuda")[4:].view(B, 4, m.F)
+    assert obs.data_ptr() % 32 == 16 and nxt.data_ptr() % 32 == 16
+    odd = (obs, nxt) + tuple(torch.empty_like(t) for t in aligned[2:])
+    edp.edp_deliver(m.ring.ctx, idx, B, edp.make_batch(*aligned))
+    edp.edp_deliver(m.ring.ctx, idx, B, edp.make_batch(*odd))
+    edp.edp_sync(m.ring.ctx)
+    for x, y in zip(aligned, odd):
+        assert np.array_equal(bits(x) if x.is_floating_point() else to_np(x),
+                              bits(y) if y.is_floating_point() else to_np(y))
