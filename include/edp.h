@@ -380,6 +380,23 @@ EDP_API const char *edp_last_error(const edp_ctx *ctx);
  * differ. */
 EDP_API edp_status edp_migrate(const edp_ctx *src, edp_ctx *dst, edp_stream stream);
 
+/* Checkpoint / resume (no counterpart in the paper, which keeps no
+ * fault tolerance; an experience buffer worth hours of rollouts is worth
+ * saving).  edp_save waits for `stream`, then writes the context's
+ * retained transitions in logical order -- payload rows from both tiers,
+ * action / reward / done, priority leaves, the deferred and maximum
+ * priorities -- with a header describing the layout, to the file `path`.
+ * edp_load reads such a file into an empty context of the same layout
+ * (transform, observation shape, frame_stack, next_obs, tokens,
+ * prioritized flag, metadata arrays); capacity and tier split may differ:
+ * the newest min(saved, capacity) transitions become its first insertions,
+ * placed by its own tier map, and its tree is rebuilt on `stream`.  Both
+ * stage the data through 64 MiB of host memory and synchronise.
+ * EDP_ERR_INVALID for an unreadable, foreign or truncated file (the context
+ * is left empty), EDP_ERR_STATE for a non-empty context or another layout. */
+EDP_API edp_status edp_save(edp_ctx *ctx, const char *path, edp_stream stream);
+EDP_API edp_status edp_load(edp_ctx *ctx, const char *path, edp_stream stream);
+
 /* Fill *out with the context's cursors and tree layout. */
 EDP_API edp_status edp_get_info(const edp_ctx *ctx, edp_info *out);
 

@@ -1,9 +1,11 @@
 // edp_api.cu -- the C ABI of libedp: argument validation, host-side cursors
 // of the logical ring, and kernel dispatch.  Every step of the data path
 // runs in the kernels of the other translation units.
+#include <algorithm>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <new>
 
@@ -385,6 +387,206 @@ edp_status edp_migrate(const edp_ctx *src, edp_ctx *dst, edp_stream stream) {
   }
   if (e != cudaSuccess) return cuda_fail(dst, e, "edp_migrate");
   dst->total = n;
+  return EDP_OK;
+}
+
+}  // extern "C"
+
+// ---- checkpoint / resume ------------------------------------------------
+namespace {
+
+struct CkptHeader {
+  char magic[8];
+  uint32_t version, transform, obs_c, obs_h, obs_w, frame_stack, next_obs, tokens;
+  uint32_t prioritized, has_action, has_reward, has_done, pending_q, max_q, pad;
+  uint64_t n, obs_bytes, tok_bytes;
+};
+static_assert(sizeof(CkptHeader) == 96, "checkpoint header layout");
+constexpr char kMagic[8] = {'E', 'D', 'P', 'C', 'K', 'P', 'T', '1'};
+constexpr size_t kStage = 64u << 20;  // bytes staged per transfer
+
+// Where the payload row of logical id L lives (the tier map): the newest
+// min(total, cap_h) ids in HBM at L mod cap_h, older ones in the host tier.
+uint8_t *row_of(const edp_ctx *c, uint8_t *hbm, uint8_t *host, uint64_t row, uint64_t L) {
+  const uint64_t in_hbm = c->total < c->cap_h ? c->total : c->cap_h;
+  if (L >= c->total - in_hbm) return hbm + (L % c->cap_h) * row;
+  return host + (L % (c->cap_c ? c->cap_c : 1)) * row;
+}
+
+// Visit ids [L0, L0 + n) in order as runs of consecutive rows of one array:
+// fn(first id, count, pointer to the first row).
+template <typename F>
+void payload_runs(const edp_ctx *c, uint8_t *hbm, uint8_t *host, uint64_t row, uint64_t L0,
+                  uint64_t n, F fn) {
+  uint64_t j = 0;
+  while (j < n) {
+    uint8_t *p = row_of(c, hbm, host, row, L0 + j);
+    uint64_t k = 1;
+    while (j + k < n && row_of(c, hbm, host, row, L0 + j + k) == p + k * row) ++k;
+    fn(j, k, p);
+    j += k;
+  }
+}
+
+// The same for an array indexed by slot L mod cap.
+template <typename F>
+void slot_runs(uint64_t cap, uint64_t L0, uint64_t n, F fn) {
+  uint64_t j = 0;
+  while (j < n) {
+    const uint64_t s = (L0 + j) % cap;
+    const uint64_t k = std::min<uint64_t>(n - j, cap - s);
+    fn(j, k, s);
+    j += k;
+  }
+}
+
+bool same_layout(const edp_ctx *c, const CkptHeader &h) {
+  const edp_config &g = c->cfg;
+  return h.transform == g.transform && h.obs_c == g.obs_c && h.obs_h == g.obs_h &&
+         h.obs_w == g.obs_w && h.frame_stack == g.frame_stack && h.next_obs == g.next_obs &&
+         h.tokens == g.tokens && h.prioritized == (g.prioritized != 0) &&
+         h.has_action == (c->st.action != nullptr) && h.has_reward == (c->st.reward != nullptr) &&
+         h.has_done == (c->st.done != nullptr);
+}
+
+}  // namespace
+
+extern "C" {
+
+edp_status edp_save(edp_ctx *ctx, const char *path, edp_stream stream) {
+  if (!ctx) return EDP_ERR_INVALID;
+  if (!path) return fail(ctx, EDP_ERR_INVALID, "edp_save: path is NULL");
+  cudaSetDevice(ctx->cfg.device);
+  cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_save");
+  CkptHeader h{};
+  std::memcpy(h.magic, kMagic, 8);
+  h.version = 1;
+  const edp_config &g = ctx->cfg;
+  h.transform = g.transform; h.obs_c = g.obs_c; h.obs_h = g.obs_h; h.obs_w = g.obs_w;
+  h.frame_stack = g.frame_stack; h.next_obs = g.next_obs; h.tokens = g.tokens;
+  h.prioritized = g.prioritized != 0;
+  h.has_action = ctx->st.action != nullptr;
+  h.has_reward = ctx->st.reward != nullptr;
+  h.has_done = ctx->st.done != nullptr;
+  h.n = ring_size(ctx);
+  h.obs_bytes = ctx->obs_bytes;
+  h.tok_bytes = ctx->tok_bytes;
+  if (ctx->depth) {
+    uint32_t pm[2];
+    e = cudaMemcpy(pm, &ctx->ctrl->pending_q, sizeof pm, cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_save");
+    h.pending_q = pm[0];
+    h.max_q = pm[1];
+  }
+  FILE *f = std::fopen(path, "wb");
+  if (!f) return fail(ctx, EDP_ERR_INVALID, "edp_save: cannot open %s", path);
+  uint8_t *stage = (uint8_t *)std::malloc(kStage);
+  const bool staged = stage != nullptr;
+  bool ok = staged && std::fwrite(&h, sizeof h, 1, f) == 1;
+  const uint64_t L0 = ctx->total - h.n;
+  // copy `bytes` from (device or host) src to the file through the stage
+  auto put = [&](const void *src, uint64_t bytes) {
+    for (uint64_t o = 0; ok && o < bytes; o += kStage) {
+      const size_t b = (size_t)std::min<uint64_t>(kStage, bytes - o);
+      ok = cudaMemcpy(stage, (const uint8_t *)src + o, b, cudaMemcpyDefault) == cudaSuccess &&
+           std::fwrite(stage, 1, b, f) == b;
+    }
+  };
+  auto payload = [&](uint8_t *hbm, uint8_t *host, uint64_t row) {
+    payload_runs(ctx, hbm, host, row, L0, h.n,
+                 [&](uint64_t, uint64_t k, uint8_t *p) { put(p, k * row); });
+  };
+  payload(ctx->st.obs, ctx->st.host_obs, ctx->obs_bytes);
+  if (ctx->tok_bytes)
+    payload((uint8_t *)ctx->st.tokens, (uint8_t *)ctx->st.host_tokens, ctx->tok_bytes);
+  auto meta = [&](const void *base, size_t elem) {
+    if (!base) return;
+    slot_runs(ctx->cap, L0, h.n, [&](uint64_t, uint64_t k, uint64_t sl) {
+      put((const uint8_t *)base + sl * elem, k * elem);
+    });
+  };
+  meta(ctx->st.action, 4);
+  meta(ctx->st.reward, 4);
+  meta(ctx->st.done, 1);
+  meta(ctx->leaves, 4);
+  std::free(stage);
+  ok = (std::fclose(f) == 0) && ok;
+  if (!ok) {
+    cudaGetLastError();
+    return fail(ctx, staged ? EDP_ERR_INVALID : EDP_ERR_OOM, "edp_save: writing %s failed",
+                path);
+  }
+  return EDP_OK;
+}
+
+edp_status edp_load(edp_ctx *ctx, const char *path, edp_stream stream) {
+  if (!ctx) return EDP_ERR_INVALID;
+  if (!path) return fail(ctx, EDP_ERR_INVALID, "edp_load: path is NULL");
+  if (ctx->total != 0) return fail(ctx, EDP_ERR_STATE, "edp_load: the context must be empty");
+  FILE *f = std::fopen(path, "rb");
+  if (!f) return fail(ctx, EDP_ERR_INVALID, "edp_load: cannot open %s", path);
+  CkptHeader h{};
+  if (std::fread(&h, sizeof h, 1, f) != 1 || std::memcmp(h.magic, kMagic, 8) != 0 ||
+      h.version != 1) {
+    std::fclose(f);
+    return fail(ctx, EDP_ERR_INVALID, "edp_load: %s is not a checkpoint of this format", path);
+  }
+  if (!same_layout(ctx, h) || h.obs_bytes != ctx->obs_bytes || h.tok_bytes != ctx->tok_bytes) {
+    std::fclose(f);
+    return fail(ctx, EDP_ERR_STATE, "edp_load: the checkpoint's layout differs from the context's");
+  }
+  cudaSetDevice(ctx->cfg.device);
+  const uint64_t n = h.n < ctx->cap ? h.n : ctx->cap;  // the newest n are kept
+  const uint64_t skip = h.n - n;
+  uint8_t *stage = (uint8_t *)std::malloc(kStage);
+  const bool staged = stage != nullptr;
+  bool ok = staged;
+  // the context's cursors as they will be: n insertions, ids 0 .. n-1
+  ctx->total = n;
+  auto get = [&](void *dst, uint64_t bytes) {
+    for (uint64_t o = 0; ok && o < bytes; o += kStage) {
+      const size_t b = (size_t)std::min<uint64_t>(kStage, bytes - o);
+      ok = std::fread(stage, 1, b, f) == b &&
+           cudaMemcpy((uint8_t *)dst + o, stage, b, cudaMemcpyDefault) == cudaSuccess;
+    }
+  };
+  auto seek = [&](uint64_t bytes) {
+    if (ok && bytes) ok = std::fseek(f, (long)bytes, SEEK_CUR) == 0;
+  };
+  auto payload = [&](uint8_t *hbm, uint8_t *host, uint64_t row) {
+    seek(skip * row);
+    payload_runs(ctx, hbm, host, row, 0, n,
+                 [&](uint64_t, uint64_t k, uint8_t *p) { get(p, k * row); });
+  };
+  payload(ctx->st.obs, ctx->st.host_obs, ctx->obs_bytes);
+  if (ctx->tok_bytes)
+    payload((uint8_t *)ctx->st.tokens, (uint8_t *)ctx->st.host_tokens, ctx->tok_bytes);
+  auto meta = [&](void *base, size_t elem, bool present) {
+    if (!present) return;
+    seek(skip * elem);
+    slot_runs(ctx->cap, 0, n, [&](uint64_t, uint64_t k, uint64_t sl) {
+      get((uint8_t *)base + sl * elem, k * elem);
+    });
+  };
+  meta(ctx->st.action, 4, h.has_action);
+  meta(ctx->st.reward, 4, h.has_reward);
+  meta(ctx->st.done, 1, h.has_done);
+  meta(ctx->leaves, 4, h.prioritized);
+  std::free(stage);
+  std::fclose(f);
+  cudaError_t e = cudaSuccess;
+  if (ok && ctx->depth) {
+    const uint32_t pm[2] = {h.pending_q, h.max_q};
+    e = cudaMemcpy(&ctx->ctrl->pending_q, pm, sizeof pm, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = launch_tree_build_all(ctx, (cudaStream_t)stream);
+  }
+  if (!ok || e != cudaSuccess) {
+    ctx->total = 0;
+    cudaGetLastError();
+    return fail(ctx, staged ? EDP_ERR_INVALID : EDP_ERR_OOM,
+                "edp_load: reading %s failed (truncated file?)", path);
+  }
   return EDP_OK;
 }
 

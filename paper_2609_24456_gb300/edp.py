@@ -128,6 +128,8 @@ SIGNATURES = {
     "edp_place_map": (C.c_int, [C.POINTER(edp_place_option), _U32, _D, _VP, _U32, _VP]),
     "edp_place_profile": (C.c_int, [C.c_int, _U64, C.POINTER(edp_place_bw)]),
     "edp_migrate": (C.c_int, [_VP, _VP, _VP]),
+    "edp_save": (C.c_int, [_VP, C.c_char_p, _VP]),
+    "edp_load": (C.c_int, [_VP, C.c_char_p, _VP]),
     "edp_grpo_advantage": (C.c_int, [_VP, _VP, _VP, _U32, C.c_float, _VP, _VP]),
     "edp_pack_deliver": (C.c_int, [_VP, _VP, _VP, _U64, _VP, _U32, _VP, _VP, _VP, _VP,
                                    _U64, _VP]),
@@ -460,3 +462,15 @@ def edp_pack_deliver(ctx, tokens, seq_off, n_seq, idx, batch, out_tokens, out_of
         ctx, ptr(tokens), ptr(seq_off), n_seq, ptr(idx), batch, ptr(seq_value),
         ptr(out_tokens), ptr(out_off), ptr(out_value), out_cap, stream_handle(stream)),
         "edp_pack_deliver")
+
+
+def edp_save(ctx, path, stream=None):
+    """Write the context's retained experience to the file `path`."""
+    return _check(ctx, lib().edp_save(ctx, os.fsencode(path), stream_handle(stream)),
+                  "edp_save")
+
+
+def edp_load(ctx, path, stream=None):
+    """Read a checkpoint written by edp_save into the empty context."""
+    return _check(ctx, lib().edp_load(ctx, os.fsencode(path), stream_handle(stream)),
+                  "edp_load")
