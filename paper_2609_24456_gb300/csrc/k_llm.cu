@@ -3,23 +3,30 @@
 // ingestion, and the packed delivery of variable-length token sequences
 // with a per-sequence value broadcast to their tokens.
 //
-// Advantages: one warp per group; fp64 sums of r and of (r - mean)^2 (two
-// passes), one rounding to fp32 per output.  Packing: each batch entry's
-// source start, length and value (one thread each, into the context's
-// scratch) with per-CTA length sums turned into prefixes by the last CTA,
-// then one CTA per sequence forms its output offset and copies its tokens (4-byte loads and stores: neither the source
-// nor the destination offset is aligned to more than a token) and writes
-// the value beside each token.  Both copy kernels are HBM-bound.
+// Advantages: one warp per group, two warps per CTA so the groups spread
+// over every SM (the fp64 pipe is narrow; eight warps on one SM queue on
+// it); fp64 sums of r and of (r - mean)^2 (two passes), one rounding to fp32
+// per output.  Packing: each batch entry's source start, length and value
+// (one thread each, into the context's scratch) with a length sum per
+// 256-entry chunk; then one CTA per sequence forms its output offset -- the
+// chunk sums before its chunk plus the lengths before it in the chunk -- and
+// copies its tokens (4-byte loads and stores: neither the source nor the
+// destination offset is aligned to more than a token), writing the value
+// beside each token.  Up to kDirectChunks chunks the gather CTAs add the
+// chunk sums themselves; beyond that the last lengths CTA turns them into
+// prefixes once.  The gather is HBM-bound.
 #include "edp_internal.cuh"
 
 namespace edp {
 namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
-constexpr int kGrpoThreads = 256;
+constexpr int kGrpoThreads = 64;
 constexpr int kGrpoWarps = kGrpoThreads / 32;
 constexpr int kPackThreads = 256;
 constexpr int kPackUnroll = 8;
+constexpr uint32_t kDirectChunks = 256;  // chunk sums a gather CTA adds itself
+static_assert(kDirectChunks <= kPackThreads, "a gather CTA adds one chunk sum per thread");
 
 __device__ __forceinline__ double warp_sum(double v) {
 #pragma unroll
@@ -76,15 +83,15 @@ __device__ __forceinline__ uint64_t block_sum(uint64_t v, uint64_t *red) {
 }
 
 // One thread per batch entry: its entry (0 tokens and a flag for an index
-// out of range); per CTA the sum of its 256 lengths.  The last CTA to finish
-// (a ticket on the launch's work counter) turns those sums into exclusive
-// prefixes, writes out_off[batch] = the total and resets the counter.
+// out of range); per CTA the sum of its 256 lengths.  With `pre` (more than
+// kDirectChunks chunks) the last CTA to finish (a ticket on the launch's
+// work counter) turns those sums into exclusive prefixes and resets the
+// counter.
 __global__ void __launch_bounds__(kPackThreads)
 k_pack_lengths(const uint64_t *__restrict__ soff, uint64_t nseq,
                const int64_t *__restrict__ idx, uint32_t B, const float *__restrict__ sv,
                PackEntry *__restrict__ ent, uint64_t *__restrict__ part,
-               uint64_t *__restrict__ pre, uint64_t *__restrict__ ooff, uint64_t cap,
-               uint32_t *work, Ctrl *ctrl) {
+               uint64_t *__restrict__ pre, uint32_t *work, Ctrl *ctrl) {
   __shared__ uint64_t red[kPackThreads / 32];
   __shared__ uint32_t ticket;
   pdl_wait();
@@ -106,6 +113,10 @@ k_pack_lengths(const uint64_t *__restrict__ soff, uint64_t nseq,
     ent[k] = PackEntry{a, value, (uint32_t)len};
   }
   const uint64_t sum = block_sum(len, red);
+  if (!pre) {
+    if (threadIdx.x == 0) part[blockIdx.x] = sum;
+    return;
+  }
   if (threadIdx.x == 0) {
     part[blockIdx.x] = sum;
     __threadfence();
@@ -137,33 +148,41 @@ k_pack_lengths(const uint64_t *__restrict__ soff, uint64_t nseq,
     for (int w = 0; w < kPackThreads / 32; ++w) tile += red[w];
     carry += tile;
   }
-  if (threadIdx.x == 0) {
-    ooff[B] = carry;
-    if (carry > cap) flag(ctrl, DEVERR_OVERFLOW, (unsigned long long)carry);
-    work[0] = 0u;  // every CTA has taken its ticket
-  }
+  if (threadIdx.x == 0) work[0] = 0u;  // every CTA has taken its ticket
 }
 
 // One CTA per sequence: its output offset is the prefix of its 256-entry
-// chunk plus the lengths before it in the chunk (one round trip and a block
-// sum), then a thread keeps kPackUnroll loads in flight (2,048 tokens per
-// CTA pass).
-__global__ void __launch_bounds__(kPackThreads)
+// chunk (from `pre`, or the chunk sums before it) plus the lengths before it
+// in the chunk (one round trip and a block sum), then a thread keeps
+// kPackUnroll loads in flight (2,048 tokens per CTA pass).  The CTA of the
+// last entry writes out_off[batch] = the total and flags an overflow.
+__global__ void __launch_bounds__(kPackThreads, 8)  // 32 registers: 8 CTAs per SM
 k_pack_gather(const int32_t *__restrict__ tokens, const PackEntry *__restrict__ ent,
-              const uint64_t *__restrict__ pre, uint32_t B, int32_t *__restrict__ otok,
-              uint64_t *__restrict__ ooff, float *__restrict__ osv, uint64_t cap) {
+              const uint64_t *__restrict__ part, const uint64_t *__restrict__ pre, uint32_t B,
+              int32_t *__restrict__ otok, uint64_t *__restrict__ ooff,
+              float *__restrict__ osv, uint64_t cap, Ctrl *ctrl) {
   __shared__ uint64_t red[kPackThreads / 32];
   const uint64_t pol = policy_stream();
   pdl_wait();
   pdl_launch();
   for (uint32_t k = blockIdx.x; k < B; k += gridDim.x) {
-    const uint32_t c0 = k / kPackThreads * kPackThreads;
-    const uint32_t j = c0 + threadIdx.x;
+    const uint32_t c = k / kPackThreads;
+    const uint32_t j = c * kPackThreads + threadIdx.x;
     uint64_t v = j < k ? ent[j].len : 0;
-    if (threadIdx.x == 0) v += pre[k / kPackThreads];
+    if (pre) {
+      if (threadIdx.x == 0) v += pre[c];
+    } else if (threadIdx.x < c) {
+      v += part[threadIdx.x];  // c <= kDirectChunks = the block size
+    }
     const PackEntry e = ent[k];
     const uint64_t dst = block_sum(v, red);
-    if (threadIdx.x == 0) ooff[k] = dst;
+    if (threadIdx.x == 0) {
+      ooff[k] = dst;
+      if (k == B - 1) {
+        ooff[B] = dst + e.len;
+        if (dst + e.len > cap) flag(ctrl, DEVERR_OVERFLOW, (unsigned long long)(dst + e.len));
+      }
+    }
     if (e.len == 0 || dst >= cap) continue;
     const uint64_t n = min((uint64_t)e.len, cap - dst);
     const int32_t *src = tokens + e.src;
@@ -194,8 +213,11 @@ cudaError_t launch_grpo(edp_ctx *c, const float *r, const uint64_t *goff, uint32
                         float eps, float *adv, cudaStream_t s) {
   uint64_t blocks = (ng + kGrpoWarps - 1) / kGrpoWarps;
   if (blocks > 16ull * c->coop_sms) blocks = 16ull * c->coop_sms;
-  return launch_pdl(k_grpo, dim3((unsigned)blocks), dim3(kGrpoThreads), s, r, goff, ng, eps,
-                    adv);
+  // A plain launch: behind a large grid (the previous step's gather) an
+  // early-launched k_grpo made the whole step slower (62 vs 46 us for the
+  // 512 x 16 batch); its pdl_wait / pdl_launch are then no-ops.
+  k_grpo<<<dim3((unsigned)blocks), dim3(kGrpoThreads), 0, s>>>(r, goff, ng, eps, adv);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_pack(edp_ctx *c, const int32_t *tokens, const uint64_t *soff,
@@ -208,14 +230,15 @@ cudaError_t launch_pack(edp_ctx *c, const int32_t *tokens, const uint64_t *soff,
   if (!scr) return cudaErrorMemoryAllocation;
   PackEntry *ent = (PackEntry *)scr;
   uint64_t *part = (uint64_t *)(scr + ent_bytes);
-  uint64_t *pre = part + G;
+  uint64_t *pre = G > kDirectChunks ? part + G : nullptr;
   uint32_t *work = c->ctrl->work + 2 * (c->work_seq++ % kWorkSlots);
   cudaError_t e = launch_pdl(k_pack_lengths, dim3(G), dim3(kPackThreads), s, soff, nseq, idx,
-                             B, sv, ent, part, pre, ooff, cap, work, c->ctrl);
+                             B, sv, ent, part, pre, work, c->ctrl);
   if (e != cudaSuccess) return e;
   const unsigned grid = B < 65535u * 16u ? B : 65535u * 16u;
   return launch_pdl(k_pack_gather, dim3(grid), dim3(kPackThreads), s, tokens,
-                    (const PackEntry *)ent, (const uint64_t *)pre, B, otok, ooff, osv, cap);
+                    (const PackEntry *)ent, (const uint64_t *)part, (const uint64_t *)pre, B,
+                    otok, ooff, osv, cap, c->ctrl);
 }
 
 }  // namespace edp

@@ -85,6 +85,22 @@ def test_pack_small_ragged(edp_lib):
         assert np.array_equal(bits(ov)[:n], ref_v.view(np.uint32))
 
 
+@pytest.mark.parametrize("B", [65536, 65537, 70000])
+def test_pack_many_chunks(edp_lib, B):
+    """Batches around the size where the chunk prefixes move from the gather
+    CTAs to the lengths pass (256 chunks of 256 entries)."""
+    edp = edp_lib
+    ring = _ctx(edp)
+    tokens, seq_off, r, _ = fx.llm_rollout(9, 500, 2, lmin=0, lmax=9)
+    idx = np.random.default_rng(B).integers(0, 1000, size=B)
+    ref, ref_off, ref_v, out, ooff, ov = _pack_check(edp, ring, tokens, seq_off, idx, r)
+    edp.edp_sync(ring.ctx)
+    n = len(ref)
+    assert np.array_equal(to_np(ooff).view(np.uint64), ref_off)
+    assert np.array_equal(to_np(out)[:n], ref)
+    assert np.array_equal(bits(ov)[:n], ref_v.view(np.uint32))
+
+
 def test_pack_invalid_index_and_overflow(edp_lib):
     edp = edp_lib
     ring = _ctx(edp)
