@@ -71,7 +71,7 @@
 extern "C" {
 #endif
 
-#define EDP_ABI_VERSION 1
+#define EDP_ABI_VERSION 2
 
 /* Symbols of the ABI are exported; everything else in libedp is hidden. */
 #if defined(__GNUC__)
@@ -213,6 +213,13 @@ typedef struct {
   const uint64_t *tree_level[8];/* device; level d has 32^d nodes, d < D */
   const uint32_t *pending_q;    /* device [1]: deferred priority of newest */
   const uint32_t *max_q;        /* device [1]: running maximum priority */
+  /* CHW_NORM_BF16: how the kernel evaluates the per-byte normalisation,
+   * each form checked at creation against the exact chain for all 256 bytes
+   * of every channel: 2 = one FMA, bf16(fma(b, A_c, B_c)) with A_c, B_c
+   * within a few ulps of 1/(255 std_c) and -mean_c/std_c; 1 = the chain
+   * with the division as an FMA by a split reciprocal; 0 = the chain with
+   * IEEE division (also for other transforms). */
+  uint32_t norm_path;
 } edp_info;
 
 /* Create a context on cfg->device over caller storage.  Fails with

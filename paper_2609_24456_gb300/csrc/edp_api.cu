@@ -131,6 +131,61 @@ bool norm_constants(edp_ctx *c) {
   return fast;
 }
 
+// bfloat16 bits of a finite float, rounded to nearest even (the device's
+// conversion).
+uint16_t bf16_rne(float f) {
+  uint32_t u;
+  std::memcpy(&u, &f, 4);
+  u += 0x7FFFu + ((u >> 16) & 1u);
+  return (uint16_t)(u >> 16);
+}
+
+float ulp_step(float x, int d) {
+  for (; d > 0; --d) x = std::nextafter(x, INFINITY);
+  for (; d < 0; ++d) x = std::nextafter(x, -INFINITY);
+  return x;
+}
+
+// The normalised bf16 of byte b in channel c is a function of (b, c) alone:
+// bf16(fl32(fl32(fl32(b/255) - mean_c) / std_c)).  One FMA,
+// bf16(fma(b, A_c, B_c)), reproduces it for all 256 bytes when A_c and B_c
+// are close enough to 1/(255 std_c) and -mean_c/std_c and no result of the
+// chain sits on a bf16 rounding boundary the FMA crosses; the constants are
+// searched within kAffineUlps ulps of those values (nearest first) and every
+// byte is checked.  False when some channel has no such pair.
+constexpr int kAffineUlps = 16;
+
+bool norm_affine_constants(edp_ctx *c) {
+  for (uint32_t ch = 0; ch < c->cfg.obs_c; ++ch) {
+    const float m = c->cfg.norm_mean[ch], s = c->cfg.norm_std[ch];
+    uint16_t want[256];
+    for (int b = 0; b < 256; ++b) {
+      const float x = (float)b / 255.0f;
+      const float t = x - m;
+      want[b] = bf16_rne(t / s);
+    }
+    const float a0 = (float)(1.0 / (255.0 * (double)s));
+    const float b0 = (float)(-(double)m / (double)s);
+    if (!std::isfinite(a0) || !std::isfinite(b0)) return false;
+    bool found = false;
+    for (int r = 0; r <= kAffineUlps && !found; ++r)
+      for (int da = -r; da <= r && !found; ++da)
+        for (int db = -r; db <= r && !found; ++db) {
+          if (std::max(std::abs(da), std::abs(db)) != r) continue;
+          const float A = ulp_step(a0, da), B = ulp_step(b0, db);
+          bool ok = std::isfinite(A) && std::isfinite(B);
+          for (int b = 0; b < 256 && ok; ++b) ok = bf16_rne(std::fma((float)b, A, B)) == want[b];
+          if (ok) {
+            c->naff_a[ch] = A;
+            c->naff_b[ch] = B;
+            found = true;
+          }
+        }
+    if (!found) return false;
+  }
+  return true;
+}
+
 }  // namespace
 
 void *edp::ctx_scratch(edp_ctx *ctx, size_t bytes) {
@@ -291,7 +346,10 @@ edp_status edp_create(const edp_config *cfg, const edp_storage *st,
     return bad("storage.done must be device memory");
 
   if (!unit_constants(&c->r1, &c->r2)) return bad("byte/255 self-check failed");
-  if (cfg->transform == EDP_XFORM_CHW_NORM_BF16) c->norm_fast = norm_constants(c);
+  if (cfg->transform == EDP_XFORM_CHW_NORM_BF16) {
+    c->norm_fast = norm_constants(c);
+    c->norm_affine = norm_affine_constants(c);
+  }
 
   int dev_sms = 0;
   cudaDeviceGetAttribute(&dev_sms, cudaDevAttrMultiProcessorCount, cfg->device);
@@ -601,6 +659,8 @@ edp_status edp_get_info(const edp_ctx *ctx, edp_info *o) {
   o->oldest = (ctx->total - o->size) % ctx->cap;
   o->n_valid = n_valid(ctx);
   o->tree_depth = ctx->depth;
+  if (ctx->cfg.transform == EDP_XFORM_CHW_NORM_BF16)
+    o->norm_path = ctx->norm_affine ? 2 : ctx->norm_fast ? 1 : 0;
   o->tree_fanout = kFanout;
   o->tree_leaves = ctx->leaves;
   for (uint32_t d = 0; d < ctx->depth && d < 8; ++d) o->tree_level[d] = ctx->level[d];

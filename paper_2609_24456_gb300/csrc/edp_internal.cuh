@@ -71,6 +71,9 @@ struct edp_ctx {
   // per-channel normalisation: t = x - mean; y = t*S1 + t*S2 (one rounding)
   float nmean[4] = {}, ns1[4] = {}, ns2[4] = {}, nstd[4] = {};
   int norm_fast = 1;  // 0: the constants do not reproduce t/std -> divide
+  // one-FMA normalisation bf16(fma(b, A, B)), where it reproduces the chain
+  float naff_a[4] = {}, naff_b[4] = {};
+  int norm_affine = 0;
   int coop_sms = 0;
   uint32_t work_seq = 0;  // delivery launches so far (work counter pairs)
   std::string err;

@@ -17,7 +17,10 @@
 // contiguous bytes.  The byte->float step is x = b (exact),
 // fl32(b/255) = fma(x, r1, x*r2) with one rounding (see unit_f32), then
 // optionally the per-channel normalisation and the round-to-nearest-even
-// bfloat16 conversion.
+// bfloat16 conversion.  Where one FMA per byte, bf16(fma(b, A_c, B_c)),
+// gives the same bf16 as that chain for all 256 bytes of every channel
+// (constants searched and checked on the host at creation), the
+// normalising delivery uses it instead of the five-operation chain.
 //
 // These kernels are HBM-bound: per sample they read the unique source bytes
 // once and write the (2-8x larger) output once.
@@ -392,12 +395,13 @@ struct NormArgs {
   uint32_t HW8;   // 8-byte units per channel plane
   uint32_t L16;   // 16-byte units of tokens per transition
   float mean[4], s1[4], s2[4], sd[4];
+  float aa[4], ab[4];  // one-FMA form (AFF): bf16(fma(b, aa, ab))
   int fast;
   __nv_bfloat16 *out;
   int32_t *tok_out;
 };
 
-template <int UN>
+template <int UN, bool AFF>
 __global__ void __launch_bounds__(kThreads)
 k_deliver_norm(Common c, NormArgs a) {
   const int lane = threadIdx.x & 31;
@@ -439,13 +443,20 @@ k_deliver_norm(Common c, NormArgs a) {
         const uint32_t w = u0 + u * 32;
         if (w >= u_hi) continue;
         const uint32_t ch = (w >= a.HW8) + (w >= 2 * a.HW8) + (w >= 3 * a.HW8);
-        const float mc = a.mean[ch], s1 = a.s1[ch], s2 = a.s2[ch];
         float fv[8];
+        if constexpr (AFF) {
+          const float A = a.aa[ch], Bc = a.ab[ch];
 #pragma unroll
-        for (int bb = 0; bb < 8; ++bb) {
-          const float x = unit_f32(byte_f(bb < 4 ? v[u].x : v[u].y, bb & 3), c.r1, c.r2);
-          const float tt = __fsub_rn(x, mc);
-          fv[bb] = a.fast ? __fmaf_rn(tt, s1, __fmul_rn(tt, s2)) : __fdiv_rn(tt, a.sd[ch]);
+          for (int bb = 0; bb < 8; ++bb)
+            fv[bb] = __fmaf_rn(byte_f(bb < 4 ? v[u].x : v[u].y, bb & 3), A, Bc);
+        } else {
+          const float mc = a.mean[ch], s1 = a.s1[ch], s2 = a.s2[ch];
+#pragma unroll
+          for (int bb = 0; bb < 8; ++bb) {
+            const float x = unit_f32(byte_f(bb < 4 ? v[u].x : v[u].y, bb & 3), c.r1, c.r2);
+            const float tt = __fsub_rn(x, mc);
+            fv[bb] = a.fast ? __fmaf_rn(tt, s1, __fmul_rn(tt, s2)) : __fdiv_rn(tt, a.sd[ch]);
+          }
         }
         uint4 o;
         o.x = pack_bf16x2(fv[0], fv[1]);
@@ -607,12 +618,15 @@ cudaError_t launch_deliver(edp_ctx *ctx, const int64_t *idx, uint32_t B,
       a.s1[i] = ctx->ns1[i];
       a.s2[i] = ctx->ns2[i];
       a.sd[i] = ctx->nstd[i] > 0.f ? ctx->nstd[i] : 1.f;
+      a.aa[i] = ctx->naff_a[i];
+      a.ab[i] = ctx->naff_b[i];
     }
     a.fast = ctx->norm_fast;
     a.out = (__nv_bfloat16 *)out->obs;
     a.tok_out = out->tokens;
     const uint64_t units = (uint64_t)B * a.F8;
-    auto kern = k_deliver_norm<kNormUnroll>;
+    auto kern = ctx->norm_affine ? k_deliver_norm<kNormUnroll, true>
+                                 : k_deliver_norm<kNormUnroll, false>;
     return launch_pdl(kern, dim3(grid_for(kern, units, 32 * kNormUnroll, kNormIters, sms)),
                       dim3(kThreads), s, c, a);
   }

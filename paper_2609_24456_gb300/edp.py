@@ -63,7 +63,7 @@ class edp_info(C.Structure):
                 ("n_valid", C.c_uint64), ("tree_depth", C.c_uint32),
                 ("tree_fanout", C.c_uint32), ("tree_leaves", C.c_void_p),
                 ("tree_level", C.c_void_p * 8), ("pending_q", C.c_void_p),
-                ("max_q", C.c_void_p)]
+                ("max_q", C.c_void_p), ("norm_path", C.c_uint32)]
 
 
 class edp_sched_costs(C.Structure):

@@ -73,7 +73,7 @@ def test_struct_layouts_match_binding(tmp_path):
 
 def test_host_validation_without_gpu(libpath):
     from paper_2609_24456_gb300 import edp
-    assert edp.edp_abi_version() == 1
+    assert edp.edp_abi_version() == 2
     st = edp.edp_storage()
     bad = [
         edp.make_config(0, (1, 84, 84), edp.EDP_XFORM_STACK_F32),       # capacity 0

@@ -81,13 +81,30 @@ def test_mm_single_tier_ragged(edp_lib, orc):
         _deliver_check(edp, orc, ring, lg, 101, seed=3, rnd=lg.total)
 
 
-def test_mm_all_byte_channel_pairs(edp_lib, orc):
-    """All 768 (byte, channel) pairs through the normalisation, bit-exact."""
+_RNG_NORM = np.random.default_rng(77)
+NORM_CASES = [
+    (MEAN, STD, 2),
+    # channel 0: mean within an ulp of 143/255, where no (A, B) within 16
+    # ulps reproduces the chain for every byte -> the chain is evaluated
+    ((0.560784519, 0.456, 0.406), (0.604448199, 0.224, 0.225), 1),
+    # a subnormal std: 1/(255 std) overflows -> the chain with IEEE division
+    ((0.485, 0.456, 0.406), (1e-40, 0.224, 0.225), 0),
+] + [(tuple(_RNG_NORM.uniform(0, 1, 3)), tuple(_RNG_NORM.uniform(0.05, 1.05, 3)), None)
+     for _ in range(3)]
+
+
+@pytest.mark.parametrize("mean,std,path", NORM_CASES)
+def test_mm_all_byte_channel_pairs(edp_lib, orc, mean, std, path):
+    """All 768 (byte, channel) pairs through the normalisation, bit-exact,
+    for each way the kernel evaluates it (one FMA, the chain with a split
+    reciprocal, the chain with IEEE division)."""
     edp = edp_lib
     cap = 4
     cfg = edp.make_config(cap, (C, 16, 16), edp.EDP_XFORM_CHW_NORM_BF16,
-                          norm_mean=MEAN, norm_std=STD)
+                          norm_mean=mean, norm_std=std)
     ring = edp.Ring(cfg, action=False, reward=False, done=False)
+    if path is not None:
+        assert ring.info().norm_path == path
     img = np.tile(np.arange(256, dtype=np.uint8), (cap, C)).reshape(cap, C * 256)
     edp.edp_ingest(ring.ctx, cuda(img), cap)
     idx = torch.arange(cap, dtype=torch.int64, device="cuda")
@@ -95,7 +112,7 @@ def test_mm_all_byte_channel_pairs(edp_lib, orc):
     edp.edp_deliver(ring.ctx, idx, cap, edp.make_batch(out))
     edp.edp_sync(ring.ctx)
     for c in range(C):
-        lut = np.array([orc.norm_bf16(b, MEAN[c], STD[c]) for b in range(256)],
+        lut = np.array([orc.norm_bf16(b, mean[c], std[c]) for b in range(256)],
                        np.uint16)
         assert np.array_equal(bits(out)[:, c].reshape(cap, 256), np.tile(lut, (cap, 1)))
 
