@@ -1340,6 +1340,7 @@ class MmReplay(Workload):
                     "predicted_ranking": [names[i] for i in sorted(range(4),
                                                                    key=lambda i: (t_pred[i], i))]}}
 
+    def cpu_setup(self, host_rows=16384):
         import numpy as np
         import oracle as orc
         from paper_2609_24456_gb300 import fixtures as fx
@@ -1678,7 +1679,9 @@ def run_edp(args):
                 "algorithmic_bytes_per_launch": wl.deliver_bytes,
                 "avg_launch_us": avg_deliver_s * 1e6, "launches_timed": Kd}
 
-    extra = wl.extra(device, mk, stream, deliver_us) if hasattr(wl, "extra") else {}
+    extra = {}
+    if hasattr(wl, "extra") and not args.no_extra:
+        extra = wl.extra(device, mk, stream, deliver_us)
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         wl.cpu_setup()
@@ -1728,6 +1731,9 @@ def main():
                     help="the workload's schedule timed as the main number "
                          "(default: its first); the others are reported too")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-extra", action="store_true",
+                    help="skip the workload's side measurements (ingest timing, "
+                         "scheduling and placement experiments)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--e2e-steps", type=int, default=200)
