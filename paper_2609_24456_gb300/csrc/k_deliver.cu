@@ -215,6 +215,21 @@ __device__ __forceinline__ void stack_span(const Common &c, const StackArgs &a,
     const bool ok = sample_slot(c, k, &slot, &off, head && lane == 0);
     if (head) collate(c, k, ok, slot, off, lane);
     const int64_t j = (int64_t)off - (int64_t)(a.K - 1) + (int64_t)m;
+    const bool has_obs = m < a.K;
+    const bool has_next = a.next && m >= 1;
+    // the payload words of the first iteration are loaded before the
+    // episode flags are known (a frame the flags zero is read for nothing),
+    // so the flag and payload round trips overlap
+    const bool src_ok = ok && j >= 0;
+    const uint64_t js = c.oldest + (uint64_t)(j < 0 ? 0 : j);
+    const uint32_t *src = reinterpret_cast<const uint32_t *>(
+        a.frames + (js >= c.cap ? js - c.cap : js) * a.F);
+    uint32_t v[UN];
+#pragma unroll
+    for (int u = 0; u < UN; ++u) {
+      const uint32_t w = w_lo + lane + u * 32;
+      v[u] = (src_ok && w < w_hi) ? ld_stream(src + w, pol) : 0u;
+    }
     bool end_before = false, end_at = false;
     if (ok && j >= 0 && (int64_t)off >= j) {
       const uint32_t span = (uint32_t)((int64_t)off - j + 1);  // 1..K
@@ -227,14 +242,9 @@ __device__ __forceinline__ void stack_span(const Common &c, const StackArgs &a,
       end_at = (bal >> (span - 1)) & 1u;
       end_before = (bal & ((1u << (span - 1)) - 1u)) != 0;
     }
-    const bool has_obs = m < a.K;
-    const bool has_next = a.next && m >= 1;
     const bool zo = !ok || j < 0 || end_before;
     const bool zn = zo || end_at;
     const bool load = (has_obs && !zo) || (has_next && !zn);
-    const uint64_t js = c.oldest + (uint64_t)(j < 0 ? 0 : j);
-    const uint32_t *src = reinterpret_cast<const uint32_t *>(
-        a.frames + (js >= c.cap ? js - c.cap : js) * a.F);
     float4 *dobs = has_obs ? reinterpret_cast<float4 *>(
                                  a.obs + ((uint64_t)k * a.K + m) * a.F)
                            : nullptr;
@@ -242,11 +252,12 @@ __device__ __forceinline__ void stack_span(const Common &c, const StackArgs &a,
                                    a.next + ((uint64_t)k * a.K + m - 1) * a.F)
                              : nullptr;
     for (uint32_t u0 = w_lo + lane; u0 < w_hi; u0 += 32 * UN) {
-      uint32_t v[UN];
+      if (u0 != w_lo + lane) {
 #pragma unroll
-      for (int u = 0; u < UN; ++u) {
-        const uint32_t w = u0 + u * 32;
-        v[u] = (load && w < w_hi) ? ld_stream(src + w, pol) : 0u;
+        for (int u = 0; u < UN; ++u) {
+          const uint32_t w = u0 + u * 32;
+          v[u] = (load && w < w_hi) ? ld_stream(src + w, pol) : 0u;
+        }
       }
 #pragma unroll
       for (int u = 0; u < UN; ++u) {
