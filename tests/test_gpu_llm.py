@@ -101,6 +101,39 @@ def test_pack_many_chunks(edp_lib, B):
     assert np.array_equal(bits(ov)[:n], ref_v.view(np.uint32))
 
 
+@pytest.mark.parametrize("tok_shift,val_shift", [(1, 2), (3, 0), (2, 3)])
+def test_pack_unaligned_outputs(edp_lib, tok_shift, val_shift):
+    """Output arrays starting 4, 8 or 12 bytes past a 16-byte boundary (each
+    its own offset), with sequences of every length 0..200 from every
+    source alignment: the vector body, the token-by-token ends and the
+    value fill all land where the oracle puts them."""
+    edp = edp_lib
+    ring = _ctx(edp)
+    from oracle import llm
+    lens = np.arange(0, 201, dtype=np.uint64)
+    seq_off = np.concatenate([[0], np.cumsum(lens)]).astype(np.uint64)
+    rng = np.random.default_rng(tok_shift * 7 + val_shift)
+    tokens = rng.integers(0, 152064, size=int(seq_off[-1]), dtype=np.int32)
+    value = rng.standard_normal(len(lens)).astype(np.float32)
+    idx = rng.permutation(len(lens)).astype(np.int64)
+    ref, ref_off, ref_v = llm.pack(tokens, seq_off, idx, value)
+    n = len(ref)
+    base_t = torch.full((n + 8,), -7, dtype=torch.int32, device="cuda")
+    base_v = torch.full((n + 8,), float("nan"), device="cuda")
+    out, ov = base_t[tok_shift:tok_shift + n], base_v[val_shift:val_shift + n]
+    assert out.data_ptr() % 16 == 4 * tok_shift and ov.data_ptr() % 16 == 4 * val_shift
+    ooff = torch.full((len(idx) + 1,), -1, dtype=torch.int64, device="cuda")
+    edp.edp_pack_deliver(ring.ctx, cuda(tokens), cuda(seq_off), len(lens), cuda(idx),
+                         len(idx), out, ooff, n, seq_value=cuda(value), out_value=ov)
+    edp.edp_sync(ring.ctx)
+    assert np.array_equal(to_np(ooff).view(np.uint64), ref_off)
+    assert np.array_equal(to_np(out), ref)
+    assert np.array_equal(bits(ov), ref_v.view(np.uint32))
+    # nothing written outside the output
+    assert (to_np(base_t[:tok_shift]) == -7).all() and (to_np(base_t[tok_shift + n:]) == -7).all()
+    assert np.isnan(to_np(base_v[:val_shift])).all() and np.isnan(to_np(base_v[val_shift + n:])).all()
+
+
 def test_pack_invalid_index_and_overflow(edp_lib):
     edp = edp_lib
     ring = _ctx(edp)
