@@ -180,6 +180,13 @@ def dev(a, device):
     return torch.from_numpy(a).to(device)
 
 
+def oracle_set_threads(n):
+    import oracle
+    L = oracle.lib()
+    L.orc_set_threads.argtypes = [ctypes.c_int]
+    L.orc_set_threads(int(n))
+
+
 def oracle_threads():
     import oracle
     L = oracle.lib()
@@ -1686,9 +1693,16 @@ def run_edp(args):
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         wl.cpu_setup()
         n, dt = time_cpu(wl, args.cpu_seconds)
+        cores = oracle_threads()
         cpu = {"value": wl.round_bytes * n / dt / 1e9, "unit": "GB/s",
-               "cores": oracle_threads(), "kind": "oracle",
+               "cores": cores, "kind": "oracle",
                "sample": "%d rounds: %s" % (n, wl.cpu_sample)}
+        # the same oracle on one core (a shorter sample)
+        oracle_set_threads(1)
+        n1, dt1 = time_cpu(wl, max(1.0, args.cpu_seconds / 3))
+        oracle_set_threads(cores)
+        cpu["single_thread"] = {"value": wl.round_bytes * n1 / dt1 / 1e9, "unit": "GB/s",
+                                "cores": 1, "sample": "%d rounds" % n1}
 
     if rank == 0:
         line = {"metric": "experience-delivery GB/s", "value": value,

@@ -31,6 +31,15 @@
 
 #define ORC_API __attribute__((visibility("default")))
 
+/* Set the threads of the OpenMP loops (timing only; no effect on results). */
+ORC_API void orc_set_threads(int n) {
+#ifdef _OPENMP
+  if (n > 0) omp_set_num_threads(n);
+#else
+  (void)n;
+#endif
+}
+
 /* Threads the OpenMP loops over batch rows use (1 without OpenMP). */
 ORC_API int orc_num_threads(void) {
 #ifdef _OPENMP
