@@ -115,6 +115,18 @@ __device__ __forceinline__ uint32_t batch_qmin(const Common &c, int lane) {
   return m;
 }
 
+// Importance weight (q_min / q_k)^beta in fp64, one rounding to fp32.
+__device__ __forceinline__ float is_weight(uint32_t m, uint32_t qk, double beta) {
+  if (qk == m) return 1.f;
+  if (!qk) return 0.f;
+  // m / qk with an fp32 seed and two Newton steps (no fp64 divide)
+  const double d = (double)qk;
+  double y = (double)(1.0f / (float)qk);
+  y = fma(y, fma(-d, y, 1.0), y);
+  y = fma(y, fma(-d, y, 1.0), y);
+  return (float)pow_pos<false>((double)m * y, beta);
+}
+
 // Per-sample collate, importance weight and scalar gathers (one warp).  The
 // head warp of each sample runs this before its payload span, so the fp64
 // chain of the weight overlaps the other warps' streaming.
@@ -130,21 +142,45 @@ __device__ void collate(const Common &c, uint32_t k, bool ok, uint64_t slot,
   if (c.isw) {
     // PER: w = (q_min / q_k)^beta, q_min over the batch; fp64, one rounding
     const uint32_t m = batch_qmin(c, lane);
-    if (lane == 0) {
-      const uint32_t qk = c.q[k];
-      float w = 0.f;
-      if (qk == m) {
-        w = 1.f;
-      } else if (qk) {
-        // m / qk with an fp32 seed and two Newton steps (no fp64 divide)
-        const double d = (double)qk;
-        double y = (double)(1.0f / (float)qk);
-        y = fma(y, fma(-d, y, 1.0), y);
-        y = fma(y, fma(-d, y, 1.0), y);
-        w = (float)pow_pos<false>((double)m * y, c.beta);
+    if (lane == 0) c.isw[k] = is_weight(m, c.q[k], c.beta);
+  }
+}
+
+// The whole batch's collate, importance weights and index reporting by one
+// CTA, for a frame-stack batch small enough to run one chunk per CTA: the
+// streaming CTAs then carry no collate latency (q_min over the batch once, a
+// block reduction, then one sample per thread).
+__device__ void collate_batch(const Common &c) {
+  __shared__ uint32_t s_min[kWarps];
+  const int lane = threadIdx.x & 31;
+  uint32_t m = 0xffffffffu;
+  if (c.isw) {
+    for (uint32_t i0 = threadIdx.x; i0 < c.B; i0 += kThreads * 4) {
+      uint32_t v[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const uint32_t i = i0 + u * kThreads;
+        v[u] = i < c.B ? __ldg(c.q + i) : 0xffffffffu;
       }
-      c.isw[k] = w;
+#pragma unroll
+      for (int u = 0; u < 4; ++u) m = min(m, v[u]);
     }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) m = min(m, __shfl_xor_sync(kFull, m, o));
+    if (lane == 0) s_min[threadIdx.x >> 5] = m;
+    __syncthreads();
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) m = min(m, s_min[w]);
+  }
+  for (uint32_t k = threadIdx.x; k < c.B; k += kThreads) {
+    uint64_t slot = 0, off = 0;
+    const bool ok = sample_slot(c, k, &slot, &off, true);
+    if (c.act_out) c.act_out[k] = ok ? c.action[slot] : 0;
+    if (c.rew_out) c.rew_out[k] = ok ? c.reward[slot] : 0.f;
+    if (c.done_out) c.done_out[k] = ok ? c.done[slot] : (uint8_t)0;
+    if (c.gdst0) c.gdst0[k] = ok ? c.gsrc0[off] : 0.f;
+    if (c.gdst1) c.gdst1[k] = ok ? c.gsrc1[off] : 0.f;
+    if (c.isw) c.isw[k] = is_weight(m, c.q[k], c.beta);
   }
 }
 
@@ -183,7 +219,11 @@ __device__ __forceinline__ float byte_f(uint32_t w, int i) {
 // delivery (the overlapped timing of Sec. 6.1) -- and its CTAs take chunks
 // from the launch's work counter until the batch is done, which balances
 // the tail without relying on all CTAs being resident.  A smaller batch
-// runs one chunk per CTA with no counter.
+// runs one chunk per CTA with no counter, and one more CTA collates the
+// whole batch (collate_batch) so that no streaming warp waits on it; on the
+// persistent grid the head warp of each sample collates it before its span
+// (measured: a collate CTA there made the isolated launch faster, 29.1 ->
+// 25.6 us, but the overlapped replay round slower, 21.0 -> 23-24 us).
 // ---------------------------------------------------------------------------
 struct StackArgs {
   const uint8_t *frames;
@@ -200,7 +240,7 @@ struct StackArgs {
 template <int UN>
 __device__ __forceinline__ void stack_span(const Common &c, const StackArgs &a,
                                            uint64_t f, uint64_t end, int lane,
-                                           uint64_t pol) {
+                                           uint64_t pol, bool head_collate) {
   const uint64_t per = (uint64_t)a.U * a.W;  // units per sample
   const float4 zero4 = make_float4(0.f, 0.f, 0.f, 0.f);
   while (f < end) {
@@ -210,7 +250,7 @@ __device__ __forceinline__ void stack_span(const Common &c, const StackArgs &a,
     const uint32_t w_lo = rem - m * a.W;
     const uint64_t seg_end = min(end, (uint64_t)k * per + (uint64_t)(m + 1) * a.W);
     const uint32_t w_hi = (uint32_t)(seg_end - (uint64_t)k * per - (uint64_t)m * a.W);
-    const bool head = rem == 0;
+    const bool head = head_collate && rem == 0;
     uint64_t slot = 0, off = 0;
     const bool ok = sample_slot(c, k, &slot, &off, head && lane == 0);
     if (head) collate(c, k, ok, slot, off, lane);
@@ -286,9 +326,13 @@ k_deliver_stack(Common c, StackArgs a) {
   pdl_launch();
   const uint64_t total = (uint64_t)c.B * a.U * a.W;
   const uint64_t per_chunk = (uint64_t)kWarps * a.span;
-  if (!c.work) {  // one chunk per CTA
-    const uint64_t f = (uint64_t)blockIdx.x * per_chunk + (uint64_t)warp * a.span;
-    if (f < total) stack_span<UN>(c, a, f, min(total, f + a.span), lane, pol);
+  if (!c.work) {  // one chunk per CTA; CTA 0 collates the batch
+    if (blockIdx.x == 0) {
+      collate_batch(c);
+      return;
+    }
+    const uint64_t f = (uint64_t)(blockIdx.x - 1) * per_chunk + (uint64_t)warp * a.span;
+    if (f < total) stack_span<UN>(c, a, f, min(total, f + a.span), lane, pol, false);
     return;
   }
   // Thread 0 grabs the next chunk while the CTA works on the current one
@@ -303,7 +347,7 @@ k_deliver_stack(Common c, StackArgs a) {
     uint32_t nxt = 0;
     if (threadIdx.x == 0) nxt = atomicAdd(&c.work[0], 1u);
     const uint64_t f = f0 + (uint64_t)warp * a.span;
-    if (f < total) stack_span<UN>(c, a, f, min(total, f + a.span), lane, pol);
+    if (f < total) stack_span<UN>(c, a, f, min(total, f + a.span), lane, pol, true);
     if (threadIdx.x == 0) s_chunk[p] = nxt;
     __syncthreads();
     cur = s_chunk[p];
@@ -577,7 +621,7 @@ cudaError_t launch_deliver(edp_ctx *ctx, const int64_t *idx, uint32_t B,
       chunks = n_chunks(a.span);
     }
     if (grid >= chunks) {
-      grid = chunks;  // one chunk per CTA, no work counter
+      grid = chunks + 1;  // one chunk per CTA and the collate CTA, no work counter
     } else {
       c.work = ctx->ctrl->work + 2 * (ctx->work_seq++ % kWorkSlots);
     }

@@ -114,6 +114,43 @@ def test_update_duplicates_invalid_and_deferred(edp_lib, orc):
     check_tree(orc, m.ring, m.st)
 
 
+@pytest.mark.parametrize("n", [1, 31, 33, 512, 2048, 2049, 5000])
+@pytest.mark.parametrize("path", ["u32", "td"])
+def test_update_batch_sizes(edp_lib, orc, n, path):
+    """Both entry points at batch sizes from one pair to several of the
+    update's 1,024-pair chunks: duplicates (last wins), the deferred newest
+    transition, slots outside the stored range, then the whole tree
+    bit-exact.  The TD-error path is checked against the oracle
+    applying the priorities the device's own rule gives for the same TD
+    errors (edp_priorities_from_td), so the tree comparison stays exact."""
+    edp = edp_lib
+    cap = 3000
+    frames, action, reward, done = fx.dqn_transitions(11, 2500, 84 * 4)
+    q = orc.priorities_from_td(fx.td_errors(11, 2500), ALPHA, EPS)
+    m = MirroredDqn(cap, prioritized=True, F=84 * 4)
+    m.ingest(orc, frames, action, reward, done, q=q)
+    rng = np.random.default_rng(n * 3 + (path == "td"))
+    for step in range(3):
+        idx = rng.integers(0, 2600, size=n).astype(np.int64)  # 2500.. hold nothing
+        idx[::7] = idx[0]
+        if n > 5:
+            idx[5] = m.total - 1  # the newest (deferred) transition
+        if path == "u32":
+            qu = rng.integers(0, 1 << 31, size=n).astype(np.uint32)
+            edp.edp_update_priorities(m.ring.ctx, cuda(idx), cuda(qu), n)
+        else:
+            td = rng.standard_normal(n).astype(np.float32) * 3
+            d_td = cuda(td)
+            qd = torch.zeros(n, dtype=torch.int32, device="cuda")
+            edp.edp_priorities_from_td(m.ring.ctx, d_td, n, ALPHA, EPS, qd)
+            edp.edp_update_priorities_td(m.ring.ctx, cuda(idx), d_td, n, ALPHA, EPS)
+            edp.edp_sync(m.ring.ctx)
+            qu = u32(qd)
+        orc.update_leaves(m.st, m.total, idx, qu)
+        edp.edp_sync(m.ring.ctx)
+        check_tree(orc, m.ring, m.st)
+
+
 def test_priorities_from_td_within_one(edp_lib, orc):
     edp = edp_lib
     m = MirroredDqn(64, prioritized=True)
