@@ -106,15 +106,27 @@ k_gae_scan(const float *__restrict__ r, const float *__restrict__ v,
       const int64_t ts = te - 32 * kJ > 0 ? te - 32 * kJ : 0;
       df del[kJ], cc[kJ];
       df a = one, b = zero;  // this lane's steps composed: x -> b + a x
+      // every input of the lane's steps is loaded before any is used, so
+      // the loads share one round trip
+      float rr[kJ], vv[kJ], vn[kJ];
+      bool dd[kJ];
+#pragma unroll
+      for (int i = 0; i < kJ; ++i) {
+        const int64_t t = ts + (int64_t)lane * kJ + i;
+        const uint64_t at = (uint64_t)(t < te ? t : ts) * E + e;
+        rr[i] = r[at];
+        vv[i] = v[at];
+        vn[i] = v[at + E];
+        dd[i] = d[at] != 0;
+      }
 #pragma unroll
       for (int i = kJ - 1; i >= 0; --i) {
         const int64_t t = ts + (int64_t)lane * kJ + i;
         if (t < te) {
-          const uint64_t at = (uint64_t)t * E + e;
-          const bool dn = d[at] != 0;
+          const bool dn = dd[i];
           // delta = r + gamma V' (1 - d) - V
-          df x = dn ? df{r[at], 0.f} : df_add_f(df_mul_f(g, v[at + E]), r[at]);
-          del[i] = df_add_f(x, -v[at]);
+          df x = dn ? df{rr[i], 0.f} : df_add_f(df_mul_f(g, vn[i]), rr[i]);
+          del[i] = df_add_f(x, -vv[i]);
           cc[i] = dn ? zero : gl;
           b = df_add(del[i], df_mul(cc[i], b));
           a = df_mul(cc[i], a);
@@ -143,7 +155,7 @@ k_gae_scan(const float *__restrict__ r, const float *__restrict__ v,
           A = df_add(del[i], df_mul(cc[i], A));
           const uint64_t at = (uint64_t)t * E + e;
           if (A_out) A_out[at] = A.hi;
-          if (ret) ret[at] = df_add_f(A, v[at]).hi;
+          if (ret) ret[at] = df_add_f(A, vv[i]).hi;
           const double Ad = df_to_d(A);
           s1 += Ad;
           s2 = fma(Ad, Ad, s2);
@@ -188,6 +200,9 @@ k_gae_norm(const float *A_src, float *adv_norm, uint64_t n, const double *partia
   __shared__ double stat[2];
   pdl_wait();
   pdl_launch();
+  // this thread's first element, loaded beside the partial sums
+  const uint64_t i0 = blockIdx.x * (uint64_t)kNormThreads + threadIdx.x;
+  const float a0 = i0 < n ? __ldcg(&A_src[i0]) : 0.f;
   double t1 = 0.0, t2 = 0.0;
   for (unsigned i = threadIdx.x; i < nparts; i += kNormThreads) {
     t1 += __ldcg(&partial[2 * i]);
@@ -213,7 +228,8 @@ k_gae_norm(const float *A_src, float *adv_norm, uint64_t n, const double *partia
   }
   __syncthreads();
   const double mean = stat[0], inv = stat[1];
-  for (uint64_t i = blockIdx.x * (uint64_t)kNormThreads + threadIdx.x; i < n;
+  if (i0 < n) adv_norm[i0] = (float)(((double)a0 - mean) * inv);
+  for (uint64_t i = i0 + (uint64_t)gridDim.x * kNormThreads; i < n;
        i += (uint64_t)gridDim.x * kNormThreads)
     adv_norm[i] = (float)(((double)__ldcg(&A_src[i]) - mean) * inv);
 }
