@@ -1029,6 +1029,19 @@ class MmReplay(Workload):
             (self.demote_bytes if self.tiered else 0)
         self.launches_per_round = 2 + (3 if ingest else 0)  # + swap obs, swap tokens, metadata
 
+    def split_bytes(self):
+        """Per-step bytes by where they move (two-tier only): over HBM, and
+        over the host link in each direction."""
+        if not self.tiered:
+            return None
+        row = self.F + 4 * self.L
+        host_frac = (self.cap - self.cap_h) / self.cap
+        host_reads = self.B * host_frac * row
+        return {"hbm": (2 * self.ingest * row + self.B * (1 - host_frac) * row
+                        + self.B * (2 * self.F + 4 * self.L + 4 + 8)),
+                "link_in": self.ingest * row + host_reads,
+                "link_out": self.ingest * row}
+
     def config(self):
         c = {"workload": self.name, "capacity": self.cap, "batch": self.B,
              "obs": "uint8 3x224x224 CHW -> bf16 normalised", "tokens": self.L,
@@ -1721,6 +1734,9 @@ def run_edp(args):
                 "clocks": clk}
         if others:
             line["other_schedules"] = others
+        split = wl.split_bytes() if hasattr(wl, "split_bytes") else None
+        if split:  # HBM and host-link throughput of the step, separately
+            line["split_GBs"] = {k: v * K * world / (ms / 1e3) / 1e9 for k, v in split.items()}
         line.update(extra)
         print(json.dumps(line))
     if dist:
