@@ -1600,7 +1600,12 @@ def run_edp(args):
     torch.cuda.set_device(local)
     device = torch.device("cuda", local)
     from paper_2609_24456_gb300 import build
-    build.build()
+    # one rank per node compiles (if anything is stale); the others wait
+    if local == 0:
+        build.build()
+    if dist:
+        dist.barrier()
+    build.build()  # up to date by now: only checks
 
     wl = WORKLOADS[args.workload](**({"capacity": args.capacity} if args.capacity else {}))
     if args.workload == "ppo" and args.capacity:
