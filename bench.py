@@ -1526,9 +1526,9 @@ WORKLOADS = {
     "ppo": PpoIteration,
     "mm200k": MmReplay,
     "grpo": LlmBatch,
-    # two-tier: 800,000 transitions (the 1.6M of the full configuration scaled
-    # to the GPU machine's host memory), newest half in HBM, 4,096 ingested per step
-    "tiered": lambda **kw: MmReplay(capacity=kw.get("capacity") or 800_000,
+    # two-tier: 1,600,000 transitions (~244 GB), newest half in HBM (122 GB),
+    # oldest half in page-locked host memory (122 GB), 4,096 ingested per step
+    "tiered": lambda **kw: MmReplay(capacity=kw.get("capacity") or 1_600_000,
                                     hbm_frac=0.5, ingest=4096),
 }
 

@@ -1,6 +1,6 @@
-"""Two-tier parity at the size the benchmark times: 800,000 transitions of
-3x224x224 images + 512 tokens, the newest 400,000 in HBM (61 GB) and the
-oldest 400,000 in page-locked host memory (61 GB), 4,096 transitions
+"""Two-tier parity at the size the benchmark times: 1,600,000 transitions
+of 3x224x224 images + 512 tokens, the newest 800,000 in HBM (122 GB) and
+the oldest 800,000 in page-locked host memory (122 GB), 4,096 transitions
 ingested per step from page-locked staging (the steady-state path where
 each new transition takes the HBM slot of the one it demotes), uniform batch
 1,024 read from both tiers.  Checked every step: all indices against the
@@ -18,7 +18,7 @@ from test_gpu_mm import C, F, H, L, MEAN, STD, W, _mm_ring
 
 pytestmark = pytest.mark.gpu
 
-CAP, CAP_H, SEED, B, STEP = 800_000, 400_000, 1240, 1024, 4096
+CAP, CAP_H, SEED, B, STEP = 1_600_000, 800_000, 1240, 1024, 4096
 
 
 def test_two_tier_full_size(edp_lib, orc):
@@ -87,4 +87,4 @@ def test_two_tier_full_size(edp_lib, orc):
         gc.collect()
         torch.cuda.empty_cache()
         if hasattr(torch._C, "_host_emptyCache"):
-            torch._C._host_emptyCache()  # the 61 GB of page-locked host tier
+            torch._C._host_emptyCache()  # the 122 GB of page-locked host tier
