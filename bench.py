@@ -1413,7 +1413,7 @@ class LlmBatch(Workload):
         # read 4, write 4 + 4
         self.deliver_bytes = n * (8 + 16 + 8 + 4) + 12 * T
         self.round_bytes = grpo + self.deliver_bytes
-        self.launches_per_round = 1 + 3
+        self.launches_per_round = 2  # advantages + length pass, then the gather
 
     def config(self):
         return {"workload": self.name, "prompts": self.P, "responses_per_prompt": self.G,
@@ -1472,12 +1472,21 @@ class LlmBatch(Workload):
         self._grpo()
         self._pack(r)
 
+    def round_fused(self, r):
+        ot, ov, oo, _ = self.outs[r % 2]
+        self.edp.edp_grpo_pack_deliver(self.ring.ctx, self.r, self.goff, self.P, 1e-6,
+                                       self.adv, self.tok, self.off, self.n,
+                                       self.perms[r % self.n_perm], self.n, ot, oo, self.T,
+                                       out_value=ov)
+
     def round_parts(self, r):
         self._grpo()
         self._pack(r, 8)
 
     def schedules(self):
-        return [("batched", self.round, "advantages, then one packed delivery of all "
+        return [("fused", self.round_fused, "edp_grpo_pack_deliver: advantages beside the "
+                 "batch's length pass, then one packed delivery of all 8,192 responses"),
+                ("batched", self.round, "advantages, then one packed delivery of all "
                  "8,192 responses (g_del = 1)"),
                 ("per-minibatch", self.round_parts, "advantages, then 8 packed deliveries "
                  "of 1,024 responses (g_del = 1/8)")]
@@ -1486,8 +1495,7 @@ class LlmBatch(Workload):
         self._pack(r)
 
     def latency_step(self, r, ev_end):
-        self._grpo()
-        self._pack(r)
+        self.round_fused(r)
         ev_end.record()
 
     def e2e_setup(self, device):
@@ -1503,7 +1511,7 @@ class LlmBatch(Workload):
     def e2e_round(self, r):
         self.r.copy_(self.h_in, non_blocking=True)
         self.perms[r % self.n_perm].copy_(self.h_idx[r % self.n_perm], non_blocking=True)
-        self.round(r)
+        self.round_fused(r)
         ot, ov, oo, _ = self.outs[r % 2]
         self.h_tok_out.copy_(ot, non_blocking=True)
         self.h_v_out.copy_(ov, non_blocking=True)

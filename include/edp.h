@@ -362,6 +362,23 @@ EDP_API edp_status edp_pack_deliver(edp_ctx *ctx, const int32_t *tokens,
                                     uint64_t *out_off, float *out_value, uint64_t out_cap,
                                     edp_stream stream);
 
+/* The GRPO step in one call: the group-relative advantages of
+ * edp_grpo_advantage (r, group_off, n_groups, eps -> adv) and the packed
+ * delivery of edp_pack_deliver with seq_value = adv, so sequence s is
+ * response s (n_seq = group_off[n_groups]; adv has n_seq entries).  The
+ * advantages are computed beside the batch's length pass (the two are
+ * independent until the copy), then the copy puts each response's advantage
+ * on its tokens; out_value may be NULL (advantages only written to adv).
+ * Same results, scratch use and errors as the two calls. */
+EDP_API edp_status edp_grpo_pack_deliver(edp_ctx *ctx, const float *r,
+                                         const uint64_t *group_off, uint32_t n_groups,
+                                         float eps, float *adv, const int32_t *tokens,
+                                         const uint64_t *seq_off, uint64_t n_seq,
+                                         const int64_t *idx, uint32_t batch,
+                                         int32_t *out_tokens, uint64_t *out_off,
+                                         float *out_value, uint64_t out_cap,
+                                         edp_stream stream);
+
 /* Wait for `stream`, then report (and clear) asynchronous CUDA errors and
  * device-side flags recorded since the previous edp_sync. */
 EDP_API edp_status edp_sync(edp_ctx *ctx, edp_stream stream);

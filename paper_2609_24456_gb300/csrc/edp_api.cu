@@ -1000,6 +1000,37 @@ edp_status edp_pack_deliver(edp_ctx *ctx, const int32_t *tokens, const uint64_t 
   return EDP_OK;
 }
 
+edp_status edp_grpo_pack_deliver(edp_ctx *ctx, const float *r, const uint64_t *group_off,
+                                 uint32_t n_groups, float eps, float *adv,
+                                 const int32_t *tokens, const uint64_t *seq_off,
+                                 uint64_t n_seq, const int64_t *idx, uint32_t batch,
+                                 int32_t *out_tokens, uint64_t *out_off, float *out_value,
+                                 uint64_t out_cap, edp_stream stream) {
+  if (!ctx) return EDP_ERR_INVALID;
+  if (!r || !group_off || !adv || n_groups == 0)
+    return fail(ctx, EDP_ERR_INVALID, "edp_grpo_pack_deliver: NULL array or no group");
+  if (!(eps >= 0.f) || !std::isfinite(eps))
+    return fail(ctx, EDP_ERR_INVALID, "edp_grpo_pack_deliver: eps must be finite and >= 0");
+  if (!tokens || !seq_off || !idx || !out_tokens || !out_off)
+    return fail(ctx, EDP_ERR_INVALID, "edp_grpo_pack_deliver: NULL array");
+  if (n_seq == 0 || batch == 0 || batch > (1u << 20))
+    return fail(ctx, EDP_ERR_INVALID,
+                "edp_grpo_pack_deliver: need n_seq > 0, 0 < batch <= 2^20");
+  const void *p;
+  const void *ptrs[] = {r, group_off, adv, tokens, seq_off, idx, out_tokens, out_off, out_value};
+  for (const void *o : ptrs)
+    if (o && !device_view(ctx, o, &p, false))
+      return fail(ctx, EDP_ERR_INVALID, "edp_grpo_pack_deliver: arrays must be device memory");
+  cudaSetDevice(ctx->cfg.device);
+  cudaError_t e = launch_grpo_pack(ctx, r, group_off, n_groups, eps, adv, tokens, seq_off,
+                                   n_seq, idx, batch, out_tokens, out_off, out_value, out_cap,
+                                   (cudaStream_t)stream);
+  if (e == cudaErrorMemoryAllocation)
+    return fail(ctx, EDP_ERR_OOM, "edp_grpo_pack_deliver: scratch allocation failed");
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_grpo_pack_deliver");
+  return EDP_OK;
+}
+
 edp_status edp_sync(edp_ctx *ctx, edp_stream stream) {
   if (!ctx) return EDP_ERR_INVALID;
   cudaSetDevice(ctx->cfg.device);

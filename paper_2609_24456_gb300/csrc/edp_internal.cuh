@@ -336,6 +336,11 @@ cudaError_t launch_pack(edp_ctx *ctx, const int32_t *tokens, const uint64_t *sof
                         uint64_t nseq, const int64_t *idx, uint32_t B, const float *sv,
                         int32_t *otok, uint64_t *ooff, float *osv, uint64_t cap,
                         cudaStream_t s);
+cudaError_t launch_grpo_pack(edp_ctx *ctx, const float *r, const uint64_t *goff, uint32_t ng,
+                             float eps, float *adv, const int32_t *tokens,
+                             const uint64_t *soff, uint64_t nseq, const int64_t *idx,
+                             uint32_t B, int32_t *otok, uint64_t *ooff, float *osv,
+                             uint64_t cap, cudaStream_t s);
 cudaError_t launch_tree_refresh(edp_ctx *ctx, uint64_t first_leaf,
                                 uint64_t count, cudaStream_t s);
 cudaError_t launch_tree_build_all(edp_ctx *ctx, cudaStream_t s);

@@ -34,14 +34,13 @@ __device__ __forceinline__ double warp_sum(double v) {
   return v;
 }
 
-__global__ void __launch_bounds__(kGrpoThreads)
-k_grpo(const float *__restrict__ r, const uint64_t *__restrict__ goff, uint32_t ng,
-       float eps, float *__restrict__ adv) {
+// Groups g = first, first + stride, ... of one warp.
+__device__ __forceinline__ void grpo_groups(const float *__restrict__ r,
+                                            const uint64_t *__restrict__ goff, uint32_t ng,
+                                            float eps, float *__restrict__ adv,
+                                            uint64_t first, uint64_t stride) {
   const int lane = threadIdx.x & 31;
-  pdl_wait();
-  pdl_launch();
-  for (uint64_t g = (uint64_t)blockIdx.x * kGrpoWarps + (threadIdx.x >> 5); g < ng;
-       g += (uint64_t)gridDim.x * kGrpoWarps) {
+  for (uint64_t g = first; g < ng; g += stride) {
     const uint64_t lo = goff[g], hi = goff[g + 1];
     if (hi <= lo) continue;
     const uint64_t n = hi - lo;
@@ -61,13 +60,24 @@ k_grpo(const float *__restrict__ r, const uint64_t *__restrict__ goff, uint32_t 
   }
 }
 
+__global__ void __launch_bounds__(kGrpoThreads)
+k_grpo(const float *__restrict__ r, const uint64_t *__restrict__ goff, uint32_t ng,
+       float eps, float *__restrict__ adv) {
+  pdl_wait();
+  pdl_launch();
+  grpo_groups(r, goff, ng, eps, adv, (uint64_t)blockIdx.x * kGrpoWarps + (threadIdx.x >> 5),
+              (uint64_t)gridDim.x * kGrpoWarps);
+}
+
 // What the copy of batch entry k needs, resolved once: where its tokens
-// start, how many there are, and the value they carry.
+// start, how many there are, and the sequence (for its value; kNoSeq when
+// the index is out of range).
 struct PackEntry {
   uint64_t src;
-  float value;
+  uint32_t seq;
   uint32_t len;
 };
+constexpr uint32_t kNoSeq = 0xffffffffu;
 
 __device__ __forceinline__ uint64_t block_sum(uint64_t v, uint64_t *red) {
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
@@ -87,49 +97,51 @@ __device__ __forceinline__ uint64_t block_sum(uint64_t v, uint64_t *red) {
 // kDirectChunks chunks) the last CTA to finish (a ticket on the launch's
 // work counter) turns those sums into exclusive prefixes and resets the
 // counter.
-__global__ void __launch_bounds__(kPackThreads)
-k_pack_lengths(const uint64_t *__restrict__ soff, uint64_t nseq,
-               const int64_t *__restrict__ idx, uint32_t B, const float *__restrict__ sv,
-               PackEntry *__restrict__ ent, uint64_t *__restrict__ part,
-               uint64_t *__restrict__ pre, uint32_t *work, Ctrl *ctrl) {
+// Chunk `cta` of `ncta` (the CTA's role; the fused GRPO kernel runs it
+// beside the advantages).
+__device__ __forceinline__ void pack_lengths_cta(const uint64_t *__restrict__ soff,
+                                                 uint64_t nseq,
+                                                 const int64_t *__restrict__ idx, uint32_t B,
+                                                 PackEntry *__restrict__ ent,
+                                                 uint64_t *__restrict__ part,
+                                                 uint64_t *__restrict__ pre, uint32_t *work,
+                                                 Ctrl *ctrl, uint32_t cta, uint32_t ncta) {
   __shared__ uint64_t red[kPackThreads / 32];
   __shared__ uint32_t ticket;
-  pdl_wait();
-  pdl_launch();
-  const uint64_t k = (uint64_t)blockIdx.x * kPackThreads + threadIdx.x;
+  const uint64_t k = (uint64_t)cta * kPackThreads + threadIdx.x;
   uint64_t len = 0;
   if (k < B) {
     const int64_t s = idx[k];
     uint64_t a = 0;
-    float value = 0.f;
+    uint32_t seq = kNoSeq;
     if (s >= 0 && (uint64_t)s < nseq) {
       a = soff[s];
       const uint64_t b = soff[s + 1];
       len = b > a ? b - a : 0;
-      if (sv) value = sv[s];
+      seq = (uint32_t)s;
     } else {
       flag(ctrl, DEVERR_INDEX, (unsigned long long)s);
     }
-    ent[k] = PackEntry{a, value, (uint32_t)len};
+    ent[k] = PackEntry{a, seq, (uint32_t)len};
   }
   const uint64_t sum = block_sum(len, red);
   if (!pre) {
-    if (threadIdx.x == 0) part[blockIdx.x] = sum;
+    if (threadIdx.x == 0) part[cta] = sum;
     return;
   }
   if (threadIdx.x == 0) {
-    part[blockIdx.x] = sum;
+    part[cta] = sum;
     __threadfence();
     ticket = atomicAdd(&work[0], 1u);
   }
   __syncthreads();
-  if (ticket != gridDim.x - 1) return;
+  if (ticket != ncta - 1) return;
   __threadfence();
   // the last CTA: exclusive prefix of the per-CTA sums, kPackThreads at a time
   uint64_t carry = 0;
-  for (uint32_t base = 0; base < gridDim.x; base += kPackThreads) {
+  for (uint32_t base = 0; base < ncta; base += kPackThreads) {
     const uint32_t i = base + threadIdx.x;
-    const uint64_t v = i < gridDim.x ? __ldcg(&part[i]) : 0;
+    const uint64_t v = i < ncta ? __ldcg(&part[i]) : 0;
     uint64_t incl = v;
     const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
 #pragma unroll
@@ -142,13 +154,46 @@ k_pack_lengths(const uint64_t *__restrict__ soff, uint64_t nseq,
     __syncthreads();
     uint64_t before = carry;
     for (int w = 0; w < wid; ++w) before += red[w];
-    if (i < gridDim.x) pre[i] = before + incl - v;
+    if (i < ncta) pre[i] = before + incl - v;
     uint64_t tile = 0;
 #pragma unroll
     for (int w = 0; w < kPackThreads / 32; ++w) tile += red[w];
     carry += tile;
   }
   if (threadIdx.x == 0) work[0] = 0u;  // every CTA has taken its ticket
+}
+
+__global__ void __launch_bounds__(kPackThreads)
+k_pack_lengths(const uint64_t *__restrict__ soff, uint64_t nseq,
+               const int64_t *__restrict__ idx, uint32_t B, PackEntry *__restrict__ ent,
+               uint64_t *__restrict__ part, uint64_t *__restrict__ pre, uint32_t *work,
+               Ctrl *ctrl) {
+  pdl_wait();
+  pdl_launch();
+  pack_lengths_cta(soff, nseq, idx, B, ent, part, pre, work, ctrl, blockIdx.x, gridDim.x);
+}
+
+// The GRPO step's first kernel: CTAs [0, ngc) compute the group advantages
+// (two warps each, so the groups spread over the SMs), the others the
+// batch's length pass, which needs no advantage (the gather reads them).
+__global__ void __launch_bounds__(kPackThreads)
+k_grpo_pack_lengths(const float *__restrict__ r, const uint64_t *__restrict__ goff,
+                    uint32_t ng, float eps, float *__restrict__ adv, uint32_t ngc,
+                    const uint64_t *__restrict__ soff, uint64_t nseq,
+                    const int64_t *__restrict__ idx, uint32_t B, PackEntry *__restrict__ ent,
+                    uint64_t *__restrict__ part, uint64_t *__restrict__ pre, uint32_t *work,
+                    Ctrl *ctrl) {
+  pdl_wait();
+  pdl_launch();
+  if (blockIdx.x < ngc) {
+    const uint32_t w = threadIdx.x >> 5;
+    if (w < kGrpoWarps)
+      grpo_groups(r, goff, ng, eps, adv, (uint64_t)blockIdx.x * kGrpoWarps + w,
+                  (uint64_t)ngc * kGrpoWarps);
+    return;
+  }
+  pack_lengths_cta(soff, nseq, idx, B, ent, part, pre, work, ctrl, blockIdx.x - ngc,
+                   gridDim.x - ngc);
 }
 
 // One CTA per sequence: its output offset is the prefix of its 256-entry
@@ -159,8 +204,8 @@ k_pack_lengths(const uint64_t *__restrict__ soff, uint64_t nseq,
 __global__ void __launch_bounds__(kPackThreads, 8)  // 32 registers: 8 CTAs per SM
 k_pack_gather(const int32_t *__restrict__ tokens, const PackEntry *__restrict__ ent,
               const uint64_t *__restrict__ part, const uint64_t *__restrict__ pre, uint32_t B,
-              int32_t *__restrict__ otok, uint64_t *__restrict__ ooff,
-              float *__restrict__ osv, uint64_t cap, Ctrl *ctrl) {
+              const float *__restrict__ sv, int32_t *__restrict__ otok,
+              uint64_t *__restrict__ ooff, float *__restrict__ osv, uint64_t cap, Ctrl *ctrl) {
   __shared__ uint64_t red[kPackThreads / 32];
   const uint64_t pol = policy_stream();
   pdl_wait();
@@ -184,6 +229,7 @@ k_pack_gather(const int32_t *__restrict__ tokens, const PackEntry *__restrict__ 
       }
     }
     if (e.len == 0 || dst >= cap) continue;
+    const float value = osv && e.seq != kNoSeq ? __ldcg(&sv[e.seq]) : 0.f;
     const uint64_t n = min((uint64_t)e.len, cap - dst);
     const int32_t *src = tokens + e.src;
     int32_t *out = otok + dst;
@@ -200,7 +246,7 @@ k_pack_gather(const int32_t *__restrict__ tokens, const PackEntry *__restrict__ 
         const uint64_t t = t0 + u * kPackThreads;
         if (t < n) {
           out[t] = w[u];
-          if (osv) osv[dst + t] = e.value;
+          if (osv) osv[dst + t] = value;
         }
       }
     }
@@ -220,25 +266,66 @@ cudaError_t launch_grpo(edp_ctx *c, const float *r, const uint64_t *goff, uint32
   return cudaGetLastError();
 }
 
+namespace {
+
+struct PackPlan {
+  PackEntry *ent;
+  uint64_t *part, *pre;
+  uint32_t *work;
+  uint32_t G;
+};
+
+bool pack_plan(edp_ctx *c, uint32_t B, PackPlan *p) {
+  p->G = (B + kPackThreads - 1) / kPackThreads;
+  const size_t ent_bytes = ((size_t)B * sizeof(PackEntry) + 255) & ~(size_t)255;
+  uint8_t *scr = (uint8_t *)ctx_scratch(c, ent_bytes + 2 * (size_t)p->G * sizeof(uint64_t));
+  if (!scr) return false;
+  p->ent = (PackEntry *)scr;
+  p->part = (uint64_t *)(scr + ent_bytes);
+  p->pre = p->G > kDirectChunks ? p->part + p->G : nullptr;
+  p->work = c->ctrl->work + 2 * (c->work_seq++ % kWorkSlots);
+  return true;
+}
+
+cudaError_t launch_gather(edp_ctx *c, const PackPlan &p, const int32_t *tokens, uint32_t B,
+                          const float *sv, int32_t *otok, uint64_t *ooff, float *osv,
+                          uint64_t cap, cudaStream_t s) {
+  const unsigned grid = B < 65535u * 16u ? B : 65535u * 16u;
+  return launch_pdl(k_pack_gather, dim3(grid), dim3(kPackThreads), s, tokens,
+                    (const PackEntry *)p.ent, (const uint64_t *)p.part,
+                    (const uint64_t *)p.pre, B, sv, otok, ooff, osv, cap, c->ctrl);
+}
+
+}  // namespace
+
 cudaError_t launch_pack(edp_ctx *c, const int32_t *tokens, const uint64_t *soff,
                         uint64_t nseq, const int64_t *idx, uint32_t B, const float *sv,
                         int32_t *otok, uint64_t *ooff, float *osv, uint64_t cap,
                         cudaStream_t s) {
-  const uint32_t G = (B + kPackThreads - 1) / kPackThreads;
-  const size_t ent_bytes = ((size_t)B * sizeof(PackEntry) + 255) & ~(size_t)255;
-  uint8_t *scr = (uint8_t *)ctx_scratch(c, ent_bytes + 2 * (size_t)G * sizeof(uint64_t));
-  if (!scr) return cudaErrorMemoryAllocation;
-  PackEntry *ent = (PackEntry *)scr;
-  uint64_t *part = (uint64_t *)(scr + ent_bytes);
-  uint64_t *pre = G > kDirectChunks ? part + G : nullptr;
-  uint32_t *work = c->ctrl->work + 2 * (c->work_seq++ % kWorkSlots);
-  cudaError_t e = launch_pdl(k_pack_lengths, dim3(G), dim3(kPackThreads), s, soff, nseq, idx,
-                             B, sv, ent, part, pre, work, c->ctrl);
+  PackPlan p;
+  if (!pack_plan(c, B, &p)) return cudaErrorMemoryAllocation;
+  cudaError_t e = launch_pdl(k_pack_lengths, dim3(p.G), dim3(kPackThreads), s, soff, nseq,
+                             idx, B, p.ent, p.part, p.pre, p.work, c->ctrl);
   if (e != cudaSuccess) return e;
-  const unsigned grid = B < 65535u * 16u ? B : 65535u * 16u;
-  return launch_pdl(k_pack_gather, dim3(grid), dim3(kPackThreads), s, tokens,
-                    (const PackEntry *)ent, (const uint64_t *)part, (const uint64_t *)pre, B,
-                    otok, ooff, osv, cap, c->ctrl);
+  return launch_gather(c, p, tokens, B, sv, otok, ooff, osv, cap, s);
+}
+
+cudaError_t launch_grpo_pack(edp_ctx *c, const float *r, const uint64_t *goff, uint32_t ng,
+                             float eps, float *adv, const int32_t *tokens,
+                             const uint64_t *soff, uint64_t nseq, const int64_t *idx,
+                             uint32_t B, int32_t *otok, uint64_t *ooff, float *osv,
+                             uint64_t cap, cudaStream_t s) {
+  PackPlan p;
+  if (!pack_plan(c, B, &p)) return cudaErrorMemoryAllocation;
+  uint64_t ngc = (ng + kGrpoWarps - 1) / kGrpoWarps;
+  if (ngc > 16ull * c->coop_sms) ngc = 16ull * c->coop_sms;
+  // a plain launch, as for k_grpo
+  k_grpo_pack_lengths<<<dim3((unsigned)(ngc + p.G)), dim3(kPackThreads), 0, s>>>(
+      r, goff, ng, eps, adv, (uint32_t)ngc, soff, nseq, idx, B, p.ent, p.part, p.pre, p.work,
+      c->ctrl);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  return launch_gather(c, p, tokens, B, adv, otok, ooff, osv, cap, s);
 }
 
 }  // namespace edp

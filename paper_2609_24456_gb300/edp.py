@@ -133,6 +133,8 @@ SIGNATURES = {
     "edp_grpo_advantage": (C.c_int, [_VP, _VP, _VP, _U32, C.c_float, _VP, _VP]),
     "edp_pack_deliver": (C.c_int, [_VP, _VP, _VP, _U64, _VP, _U32, _VP, _VP, _VP, _VP,
                                    _U64, _VP]),
+    "edp_grpo_pack_deliver": (C.c_int, [_VP, _VP, _VP, _U32, C.c_float, _VP, _VP, _VP, _U64,
+                                        _VP, _U32, _VP, _VP, _VP, _U64, _VP]),
 }
 
 _lib = None
@@ -462,6 +464,15 @@ def edp_pack_deliver(ctx, tokens, seq_off, n_seq, idx, batch, out_tokens, out_of
         ctx, ptr(tokens), ptr(seq_off), n_seq, ptr(idx), batch, ptr(seq_value),
         ptr(out_tokens), ptr(out_off), ptr(out_value), out_cap, stream_handle(stream)),
         "edp_pack_deliver")
+
+
+def edp_grpo_pack_deliver(ctx, r, group_off, n_groups, eps, adv, tokens, seq_off, n_seq,
+                          idx, batch, out_tokens, out_off, out_cap, out_value=None,
+                          stream=None):
+    return _check(ctx, lib().edp_grpo_pack_deliver(
+        ctx, ptr(r), ptr(group_off), n_groups, eps, ptr(adv), ptr(tokens), ptr(seq_off),
+        n_seq, ptr(idx), batch, ptr(out_tokens), ptr(out_off), ptr(out_value), out_cap,
+        stream_handle(stream)), "edp_grpo_pack_deliver")
 
 
 def edp_save(ctx, path, stream=None):

@@ -178,3 +178,51 @@ def test_grpo_batch_full_size(edp_lib):
     assert np.array_equal(to_np(ooff).view(np.uint64), ref_off)
     assert np.array_equal(to_np(out), ref)
     assert np.array_equal(bits(ov), ref_v.view(np.uint32))
+
+
+@pytest.mark.parametrize("case", ["full", "ragged_invalid", "no_values"])
+def test_grpo_pack_fused(edp_lib, case):
+    """edp_grpo_pack_deliver against the two calls it fuses (bit for bit:
+    advantages, tokens, offsets, per-token values) and the oracle, on the
+    512 x 16 batch and on a small ragged one with an index out of range."""
+    edp = edp_lib
+    ring = _ctx(edp)
+    from oracle import llm
+    if case == "full":
+        tokens, seq_off, r, goff = fx.llm_rollout(11, 512, 16)
+        idx = np.random.default_rng(12).permutation(len(r)).astype(np.int64)
+    else:
+        tokens, seq_off, r, goff = fx.llm_rollout(13, 9, 5, lmin=0, lmax=300)
+        idx = np.random.default_rng(14).integers(0, len(r), size=700).astype(np.int64)
+        if case == "ragged_invalid":
+            idx[[3, 500]] = [-2, len(r)]
+    n, B = len(r), len(idx)
+    adv_ref = llm.grpo_advantage(r, goff, 1e-6)
+    d_r, d_goff, d_tok, d_off, d_idx = cuda(r), cuda(goff), cuda(tokens), cuda(seq_off), \
+        cuda(idx)
+    total = int(sum(int(seq_off[s + 1] - seq_off[s]) for s in idx if 0 <= s < n))
+    outs = []
+    for fused in (False, True):
+        adv = torch.full((n,), float("nan"), device="cuda")
+        out = torch.full((max(total, 1),), -7, dtype=torch.int32, device="cuda")
+        ov = torch.full((max(total, 1),), float("nan"), device="cuda")
+        oo = torch.full((B + 1,), -1, dtype=torch.int64, device="cuda")
+        vals = None if case == "no_values" else ov
+        if fused:
+            edp.edp_grpo_pack_deliver(ring.ctx, d_r, d_goff, len(goff) - 1, 1e-6, adv, d_tok,
+                                      d_off, n, d_idx, B, out, oo, total, out_value=vals)
+        else:
+            edp.edp_grpo_advantage(ring.ctx, d_r, d_goff, len(goff) - 1, 1e-6, adv)
+            edp.edp_pack_deliver(ring.ctx, d_tok, d_off, n, d_idx, B, out, oo, total,
+                                 seq_value=None if vals is None else adv, out_value=vals)
+        status, _ = edp.edp_sync_status(ring.ctx)
+        assert status == (edp.EDP_ERR_INVALID if case == "ragged_invalid" else edp.EDP_OK)
+        outs.append((bits(adv), to_np(out), to_np(oo), bits(ov)))
+    for x, y in zip(*outs):
+        assert np.array_equal(x, y)
+    assert _ulps(outs[1][0].view(np.float32), adv_ref).max() <= 1
+    ref, ref_off, ref_v = llm.pack(tokens, seq_off, idx, outs[1][0].view(np.float32))
+    assert np.array_equal(outs[1][2].view(np.uint64), ref_off)
+    assert np.array_equal(outs[1][1][:len(ref)], ref)
+    if case != "no_values":
+        assert np.array_equal(outs[1][3][:len(ref)], ref_v.view(np.uint32))
