@@ -196,6 +196,13 @@ k_grpo_pack_lengths(const float *__restrict__ r, const uint64_t *__restrict__ go
                    gridDim.x - ngc);
 }
 
+// 4-byte store with the streaming (evict-first) L2 policy: the packed batch
+// is written once and read by the learner, not by this kernel.
+__device__ __forceinline__ void st_stream32(void *p, uint32_t v, uint64_t pol) {
+  asm volatile("st.global.L1::no_allocate.L2::cache_hint.b32 [%0], %1, %2;"
+               :: "l"(p), "r"(v), "l"(pol) : "memory");
+}
+
 // One CTA per sequence: its output offset is the prefix of its 256-entry
 // chunk (from `pre`, or the chunk sums before it) plus the lengths before it
 // in the chunk (one round trip and a block sum), then a thread keeps
@@ -245,8 +252,8 @@ k_pack_gather(const int32_t *__restrict__ tokens, const PackEntry *__restrict__ 
       for (int u = 0; u < kPackUnroll; ++u) {
         const uint64_t t = t0 + u * kPackThreads;
         if (t < n) {
-          out[t] = w[u];
-          if (osv) osv[dst + t] = value;
+          st_stream32(out + t, (uint32_t)w[u], pol);
+          if (osv) st_stream32(osv + dst + t, __float_as_uint(value), pol);
         }
       }
     }
