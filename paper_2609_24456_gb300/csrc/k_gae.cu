@@ -13,7 +13,8 @@
 // are processed from the end of the rollout backwards, carrying A across.
 //
 // Arithmetic: GB300's fp64 pipe is narrow (a dependent fp64 FMA costs ~64
-// cycles, fp32 ~4), so the scan runs in double-float arithmetic -- a value
+// cycles, fp32 ~4), so the scan -- and each lane's sums of A and A^2 over an
+// environment -- run in double-float arithmetic -- a value
 // is an unevaluated pair hi + lo of fp32 numbers, combined with the
 // error-free transformations TwoSum (Knuth) and TwoProd via FMA (Dekker),
 // as in the double-double arithmetic of Hida, Li and Bailey -- which keeps
@@ -89,6 +90,84 @@ __device__ __forceinline__ double df_to_d(df a) {
   return (double)a.hi + (double)a.lo;
 }
 
+// One environment's scan (one warp): writes its advantages and returns and
+// adds this lane's A and A^2 to s1, s2.
+__device__ __forceinline__ void gae_env(const float *__restrict__ r,
+                                        const float *__restrict__ v,
+                                        const uint8_t *__restrict__ d, uint32_t T, uint32_t E,
+                                        uint32_t e, df g, df gl, float *__restrict__ A_out,
+                                        float *__restrict__ ret, double &s1, double &s2) {
+  const int lane = threadIdx.x & 31;
+  const df one = {1.f, 0.f}, zero = {0.f, 0.f};
+  // this lane's A and A^2 summed in double-float (the fp32 pipe), added to
+  // the fp64 accumulators once per environment
+  df a1 = zero, a2 = zero;
+  df carry = zero;  // A at the step after the current chunk
+  for (int64_t te = T; te > 0; te -= 32 * kJ) {
+    const int64_t ts = te - 32 * kJ > 0 ? te - 32 * kJ : 0;
+    df del[kJ], cc[kJ];
+    df a = one, b = zero;  // this lane's steps composed: x -> b + a x
+    // every input of the lane's steps is loaded before any is used, so
+    // the loads share one round trip
+    float rr[kJ], vv[kJ], vn[kJ];
+    bool dd[kJ];
+#pragma unroll
+    for (int i = 0; i < kJ; ++i) {
+      const int64_t t = ts + (int64_t)lane * kJ + i;
+      const uint64_t at = (uint64_t)(t < te ? t : ts) * E + e;
+      rr[i] = r[at];
+      vv[i] = v[at];
+      vn[i] = v[at + E];
+      dd[i] = d[at] != 0;
+    }
+#pragma unroll
+    for (int i = kJ - 1; i >= 0; --i) {
+      const int64_t t = ts + (int64_t)lane * kJ + i;
+      if (t < te) {
+        const bool dn = dd[i];
+        // delta = r + gamma V' (1 - d) - V
+        df x = dn ? df{rr[i], 0.f} : df_add_f(df_mul_f(g, vn[i]), rr[i]);
+        del[i] = df_add_f(x, -vv[i]);
+        cc[i] = dn ? zero : gl;
+        b = df_add(del[i], df_mul(cc[i], b));
+        a = df_mul(cc[i], a);
+      } else {
+        del[i] = zero;
+        cc[i] = one;
+      }
+    }
+    // inclusive suffix scan: lane l gets lanes l..31 composed
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const df a2 = df_shfl_down(a, o);
+      const df b2 = df_shfl_down(b, o);
+      if (lane + o < 32) {
+        b = df_add(b, df_mul(a, b2));
+        a = df_mul(a, a2);
+      }
+    }
+    const df an = df_shfl_down(a, 1);
+    const df bn = df_shfl_down(b, 1);
+    df A = lane < 31 ? df_add(bn, df_mul(an, carry)) : carry;  // A after my steps
+#pragma unroll
+    for (int i = kJ - 1; i >= 0; --i) {
+      const int64_t t = ts + (int64_t)lane * kJ + i;
+      if (t < te) {
+        A = df_add(del[i], df_mul(cc[i], A));
+        const uint64_t at = (uint64_t)t * E + e;
+        if (A_out) A_out[at] = A.hi;
+        if (ret) ret[at] = df_add_f(A, vv[i]).hi;
+        a1 = df_add(a1, A);
+        a2 = df_add(a2, df_mul(A, A));
+      }
+    }
+    const df c0 = df_add(b, df_mul(a, carry));
+    carry = {__shfl_sync(kFull, c0.hi, 0), __shfl_sync(kFull, c0.lo, 0)};
+  }
+  s1 += df_to_d(a1);
+  s2 += df_to_d(a2);
+}
+
 __global__ void __launch_bounds__(kGaeThreads)
 k_gae_scan(const float *__restrict__ r, const float *__restrict__ v,
            const uint8_t *__restrict__ d, uint32_t T, uint32_t E, double gamma,
@@ -98,73 +177,9 @@ k_gae_scan(const float *__restrict__ r, const float *__restrict__ v,
   pdl_wait();
   const df g = df_split(gamma);
   const df gl = df_split(gamma * lambda);
-  const df one = {1.f, 0.f}, zero = {0.f, 0.f};
   double s1 = 0.0, s2 = 0.0;
-  for (uint32_t e = blockIdx.x * kGaeWarps + wid; e < E; e += gridDim.x * kGaeWarps) {
-    df carry = zero;  // A at the step after the current chunk
-    for (int64_t te = T; te > 0; te -= 32 * kJ) {
-      const int64_t ts = te - 32 * kJ > 0 ? te - 32 * kJ : 0;
-      df del[kJ], cc[kJ];
-      df a = one, b = zero;  // this lane's steps composed: x -> b + a x
-      // every input of the lane's steps is loaded before any is used, so
-      // the loads share one round trip
-      float rr[kJ], vv[kJ], vn[kJ];
-      bool dd[kJ];
-#pragma unroll
-      for (int i = 0; i < kJ; ++i) {
-        const int64_t t = ts + (int64_t)lane * kJ + i;
-        const uint64_t at = (uint64_t)(t < te ? t : ts) * E + e;
-        rr[i] = r[at];
-        vv[i] = v[at];
-        vn[i] = v[at + E];
-        dd[i] = d[at] != 0;
-      }
-#pragma unroll
-      for (int i = kJ - 1; i >= 0; --i) {
-        const int64_t t = ts + (int64_t)lane * kJ + i;
-        if (t < te) {
-          const bool dn = dd[i];
-          // delta = r + gamma V' (1 - d) - V
-          df x = dn ? df{rr[i], 0.f} : df_add_f(df_mul_f(g, vn[i]), rr[i]);
-          del[i] = df_add_f(x, -vv[i]);
-          cc[i] = dn ? zero : gl;
-          b = df_add(del[i], df_mul(cc[i], b));
-          a = df_mul(cc[i], a);
-        } else {
-          del[i] = zero;
-          cc[i] = one;
-        }
-      }
-      // inclusive suffix scan: lane l gets lanes l..31 composed
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const df a2 = df_shfl_down(a, o);
-        const df b2 = df_shfl_down(b, o);
-        if (lane + o < 32) {
-          b = df_add(b, df_mul(a, b2));
-          a = df_mul(a, a2);
-        }
-      }
-      const df an = df_shfl_down(a, 1);
-      const df bn = df_shfl_down(b, 1);
-      df A = lane < 31 ? df_add(bn, df_mul(an, carry)) : carry;  // A after my steps
-#pragma unroll
-      for (int i = kJ - 1; i >= 0; --i) {
-        const int64_t t = ts + (int64_t)lane * kJ + i;
-        if (t < te) {
-          A = df_add(del[i], df_mul(cc[i], A));
-          const uint64_t at = (uint64_t)t * E + e;
-          if (A_out) A_out[at] = A.hi;
-          if (ret) ret[at] = df_add_f(A, vv[i]).hi;
-          const double Ad = df_to_d(A);
-          s1 += Ad;
-          s2 = fma(Ad, Ad, s2);
-        }
-      }
-      const df c0 = df_add(b, df_mul(a, carry));
-      carry = {__shfl_sync(kFull, c0.hi, 0), __shfl_sync(kFull, c0.lo, 0)};
-    }
-  }
+  for (uint32_t e = blockIdx.x * kGaeWarps + wid; e < E; e += gridDim.x * kGaeWarps)
+    gae_env(r, v, d, T, E, e, g, gl, A_out, ret, s1, s2);
   pdl_launch();
   if (!partial) return;  // no normalisation requested
   // per-CTA partial sums (fixed order: warps, then lanes by xor tree)

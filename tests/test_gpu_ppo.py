@@ -31,7 +31,8 @@ def _gae(edp, ring, r, v, d, want=(True, True, True)):
 @pytest.mark.parametrize("T,E,done_p", [(128, 256, 0.005), (37, 5, 0.05),
                                         (200, 3, 0.01), (1, 2, 0.5),
                                         (2, 1, 0.0), (300, 130, 0.02),
-                                        (129, 8, 1.0)])
+                                        (129, 8, 1.0),
+                                        (5, 512, 0.02), (4, 513, 0.02), (3, 700, 0.01)])
 def test_gae_matches_oracle(edp_lib, orc, T, E, done_p):
     edp = edp_lib
     _, r, v, d = fx.ppo_rollout(T * 1000 + E, T, E, done_p=done_p, with_obs=False)
