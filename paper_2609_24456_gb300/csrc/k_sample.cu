@@ -38,7 +38,7 @@ constexpr uint32_t kMaxBuckets = 8192;  // bucket starts scanned in shared memor
 }  // namespace
 
 size_t perm_scratch_bytes(uint32_t n) {
-  return 3 * (kMaxBuckets + 64) * sizeof(uint32_t) + (size_t)n * (8 + 8 + 4) + 256;
+  return 3 * (kMaxBuckets + 64) * sizeof(uint32_t) + (size_t)n * (8 + 8 + 4 + 8) + 256;
 }
 size_t perm_zeroed_bytes() { return 2 * kMaxBuckets * sizeof(uint32_t); }
 
@@ -51,6 +51,7 @@ struct PermScratch {
   uint64_t *keys;    // [n]
   uint64_t *lkey;    // [n] bucketed keys
   uint32_t *lj;      // [n] bucketed offsets
+  uint2 *bounds;     // [n] each element's bucket [start, end)
 };
 
 __device__ __forceinline__ uint32_t bucket_of(uint64_t key, int lg) {
@@ -115,9 +116,11 @@ k_perm_scatter(uint32_t n, int lg, PermScratch sc) {
        j += gridDim.x * kPermThreads) {
     const uint64_t key = __ldcg(&sc.keys[j]);
     const uint32_t b = bucket_of(key, lg);
-    const uint32_t pos = start[pad32(b)] + atomicAdd(&sc.cursor[b], 1u);
+    const uint32_t lo = start[pad32(b)];
+    const uint32_t pos = lo + atomicAdd(&sc.cursor[b], 1u);
     sc.lkey[pos] = key;
     sc.lj[pos] = j;
+    sc.bounds[j] = make_uint2(lo, b + 1 < nb ? start[pad32(b + 1)] : n);
   }
 }
 
@@ -131,8 +134,8 @@ k_perm_rank(uint32_t n, int lg, PermScratch sc, uint64_t oldest, uint64_t cap,
   pdl_launch();
   for (uint32_t j = tid; j < n; j += stride) {
     const uint64_t key = __ldcg(&sc.keys[j]);
-    const uint32_t b = bucket_of(key, lg);
-    const uint32_t lo = __ldcg(&sc.start[b]), hi = __ldcg(&sc.start[b + 1]);
+    const uint2 bd = __ldcg(&sc.bounds[j]);
+    const uint32_t lo = bd.x, hi = bd.y;
     uint32_t r = 0;
     for (uint32_t i0 = lo; i0 < hi; i0 += 4) {  // members, 4 loads at a time
       uint64_t k2[4];
@@ -185,6 +188,7 @@ cudaError_t launch_permute(edp_ctx *c, uint32_t n, uint64_t seed,
   sc.keys = (uint64_t *)(base + 3 * (kMaxBuckets + 64) * sizeof(uint32_t));
   sc.lkey = sc.keys + n;
   sc.lj = (uint32_t *)(sc.lkey + n);
+  sc.bounds = (uint2 *)(sc.lj + n + (n & 1));  // 8-byte aligned
   const uint64_t size = c->total < c->cap ? c->total : c->cap;
   const uint64_t oldest = (c->total - size) % c->cap;
   uint64_t grid = (n + kPermThreads - 1) / kPermThreads;
