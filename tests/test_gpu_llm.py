@@ -226,3 +226,32 @@ def test_grpo_pack_fused(edp_lib, case):
     assert np.array_equal(outs[1][1][:len(ref)], ref)
     if case != "no_values":
         assert np.array_equal(outs[1][3][:len(ref)], ref_v.view(np.uint32))
+
+
+def test_grpo_pack_fused_argument_errors(edp_lib):
+    edp = edp_lib
+    ring = _ctx(edp)
+    tokens, seq_off, r, goff = fx.llm_rollout(15, 4, 3, lmin=1, lmax=20)
+    n = len(r)
+    d = dict(r=cuda(r), goff=cuda(goff), tok=cuda(tokens), off=cuda(seq_off),
+             idx=cuda(np.arange(n, dtype=np.int64)))
+    adv = torch.empty(n, device="cuda")
+    out = torch.empty(int(seq_off[-1]), dtype=torch.int32, device="cuda")
+    oo = torch.empty(n + 1, dtype=torch.int64, device="cuda")
+
+    def call(**kw):
+        a = dict(r=d["r"], goff=d["goff"], ng=len(goff) - 1, eps=1e-6, adv=adv,
+                 tok=d["tok"], off=d["off"], nseq=n, idx=d["idx"], B=n, out=out, oo=oo)
+        a.update(kw)
+        edp.edp_grpo_pack_deliver(ring.ctx, a["r"], a["goff"], a["ng"], a["eps"], a["adv"],
+                                  a["tok"], a["off"], a["nseq"], a["idx"], a["B"], a["out"],
+                                  a["oo"], int(seq_off[-1]))
+
+    call()
+    edp.edp_sync(ring.ctx)
+    for kw in (dict(ng=0), dict(eps=-1.0), dict(eps=float("nan")), dict(adv=None),
+               dict(idx=None), dict(B=0), dict(nseq=0), dict(B=(1 << 20) + 1),
+               dict(tok=torch.from_numpy(tokens))):  # host memory, not device
+        with pytest.raises(edp.EdpError) as e:
+            call(**kw)
+        assert e.value.status == edp.EDP_ERR_INVALID, kw
