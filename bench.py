@@ -483,20 +483,24 @@ class PerReplay(Workload):
         self.d_td = torch.empty(B, device=device)
         self.h2d = B * 4
         self.d2h = sum(t.numel() * t.element_size() for t in self.h_out.values())
+        # the batch's outputs are the host buffers themselves; q stays on the
+        # device (written there by the sampler)
+        h = self.h_out
+        self.h_batch = self.edp.make_batch(h["obs"], h["nxt"], h["act"], h["rew"], h["done"],
+                                           q=self.outs[0]["q"], isw=h["isw"], beta=BETA)
 
     def e2e_round(self, r):
-        """User path with host buffers: TD errors in, learner batch out."""
-        o = self.outs[r % self.R]
+        """User path with host buffers: TD errors in, learner batch out --
+        delivered by the kernel straight into the page-locked host batch
+        (one output set: the e2e rounds run on one stream)."""
+        o = self.outs[0]
+        h = self.h_out
         self.d_td.copy_(self.h_td[r % self.td_rounds], non_blocking=True)
         self._sample(r, o)
-        self.edp.edp_deliver(self.ring.ctx, o["idx"], self.B, o["batch"])
+        self.edp.edp_deliver(self.ring.ctx, o["idx"], self.B, self.h_batch)
         self.edp.edp_update_priorities_td(self.ring.ctx, o["idx"], self.d_td,
                                           self.B, ALPHA, EPS)
-        h = self.h_out
-        for key, src in [("obs", "obs"), ("nxt", "nxt"), ("act", "act"),
-                         ("rew", "rew"), ("done", "done"), ("isw", "isw"),
-                         ("idx", "idx")]:
-            h[key].copy_(o[src], non_blocking=True)
+        h["idx"].copy_(o["idx"], non_blocking=True)
 
     def cpu_setup(self, host_frames=262_144):
         import numpy as np
@@ -613,12 +617,17 @@ class DqnTiny(Workload):
                           done=pin(B, dt=torch.uint8), idx=pin(B, dt=torch.int64))
         self.h2d = 0
         self.d2h = sum(t.numel() * t.element_size() for t in self.h_out.values())
+        h = self.h_out
+        self.h_batch = self.edp.make_batch(h["obs"], h["nxt"], h["act"], h["rew"], h["done"])
 
     def e2e_round(self, r):
-        self.round(r)
-        o = self.outs[r % self.R]
-        for key in ["obs", "nxt", "act", "rew", "done", "idx"]:
-            self.h_out[key].copy_(o[key], non_blocking=True)
+        """The main schedule's call with host buffers: the kernel draws the
+        batch and writes it straight into the page-locked host batch; the
+        indices (device) follow with a copy."""
+        o = self.outs[0]
+        self.edp.edp_sample_deliver(self.ring.ctx, self.B, self.seed, r, o["idx"],
+                                    self.h_batch)
+        self.h_out["idx"].copy_(o["idx"], non_blocking=True)
 
     def cpu_setup(self):
         import numpy as np

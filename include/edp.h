@@ -182,8 +182,12 @@ typedef struct {
   const uint8_t *done;   /* [n] or NULL (stores 0) */
 } edp_fields;
 
-/* Learner batch written by edp_deliver.  Device pointers; NULL skips an
- * output.  B = the `batch` argument of edp_deliver. */
+/* Learner batch written by edp_deliver.  NULL skips an output.  Outputs
+ * (obs, next_obs, action, reward, done, tokens, isw, gather_dst) are device
+ * memory, or page-locked host memory that the kernel then writes over the
+ * host link (a learner on the host gets its batch with no separate copy);
+ * the inputs q and gather_src are device memory.  B = the `batch` argument
+ * of edp_deliver. */
 typedef struct {
   void *obs;      /* see edp_transform; required */
   void *next_obs; /* STACK_F32 with next_obs == 1: float [B][K][h][w] */

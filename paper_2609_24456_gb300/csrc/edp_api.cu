@@ -812,9 +812,12 @@ edp_status edp_sample(edp_ctx *ctx, edp_sample_mode mode, uint32_t batch,
   return EDP_OK;
 }
 
-// Argument checks shared by edp_deliver and edp_sample_deliver.
+// Argument checks shared by edp_deliver and edp_sample_deliver; *res is
+// the batch with every output resolved to a device-usable address (an
+// output may be page-locked host memory: the kernel then writes it over the
+// host link).
 static edp_status deliver_checks(edp_ctx *ctx, const int64_t *idx, uint32_t batch,
-                                 const edp_batch *out) {
+                                 const edp_batch *out, edp_batch *res) {
   if (!idx || !out || !out->obs)
     return fail(ctx, EDP_ERR_INVALID, "edp_deliver: idx/out/out->obs is NULL");
   if (batch == 0) return fail(ctx, EDP_ERR_INVALID, "edp_deliver: batch == 0");
@@ -837,15 +840,27 @@ static edp_status deliver_checks(edp_ctx *ctx, const int64_t *idx, uint32_t batc
     if ((out->gather_src[i] == nullptr) != (out->gather_dst[i] == nullptr))
       return fail(ctx, EDP_ERR_INVALID, "edp_deliver: gather pair %d half-NULL", i);
   const void *p;
-  const void *outs[] = {idx, out->obs, out->next_obs, out->action, out->reward,
-                        out->done, out->tokens, out->q, out->isw,
-                        out->gather_src[0], out->gather_dst[0],
-                        out->gather_src[1], out->gather_dst[1]};
-  for (const void *o : outs)
+  const void *ins[] = {idx, out->q, out->gather_src[0], out->gather_src[1]};
+  for (const void *o : ins)
     if (o && !device_view(ctx, o, &p, false))
-      return fail(ctx, EDP_ERR_INVALID, "edp_deliver: pointers must be device memory");
-  if (!aligned16(out->obs) || (out->next_obs && !aligned16(out->next_obs)) ||
-      (out->tokens && !aligned16(out->tokens)))
+      return fail(ctx, EDP_ERR_INVALID, "edp_deliver: inputs must be device memory");
+  *res = *out;
+  void **outs[] = {&res->obs, &res->next_obs, reinterpret_cast<void **>(&res->action),
+                   reinterpret_cast<void **>(&res->reward),
+                   reinterpret_cast<void **>(&res->done),
+                   reinterpret_cast<void **>(&res->tokens),
+                   reinterpret_cast<void **>(&res->isw),
+                   reinterpret_cast<void **>(&res->gather_dst[0]),
+                   reinterpret_cast<void **>(&res->gather_dst[1])};
+  for (void **o : outs) {
+    if (!*o) continue;
+    if (!device_view(ctx, *o, &p, true))
+      return fail(ctx, EDP_ERR_INVALID,
+                  "edp_deliver: outputs must be device or page-locked host memory");
+    *o = const_cast<void *>(p);
+  }
+  if (!aligned16(res->obs) || (res->next_obs && !aligned16(res->next_obs)) ||
+      (res->tokens && !aligned16(res->tokens)))
     return fail(ctx, EDP_ERR_INVALID, "edp_deliver: obs/next_obs/tokens 16-B aligned");
   return EDP_OK;
 }
@@ -853,10 +868,11 @@ static edp_status deliver_checks(edp_ctx *ctx, const int64_t *idx, uint32_t batc
 edp_status edp_deliver(edp_ctx *ctx, const int64_t *idx, uint32_t batch,
                        const edp_batch *out, edp_stream stream) {
   if (!ctx) return EDP_ERR_INVALID;
-  const edp_status st = deliver_checks(ctx, idx, batch, out);
+  edp_batch res;
+  const edp_status st = deliver_checks(ctx, idx, batch, out, &res);
   if (st != EDP_OK) return st;
   cudaSetDevice(ctx->cfg.device);
-  cudaError_t e = launch_deliver(ctx, idx, batch, out, (cudaStream_t)stream);
+  cudaError_t e = launch_deliver(ctx, idx, batch, &res, (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_deliver");
   return EDP_OK;
 }
@@ -869,11 +885,12 @@ edp_status edp_sample_deliver(edp_ctx *ctx, uint32_t batch, uint64_t seed, uint6
   if (out && (out->isw || out->q))
     return fail(ctx, EDP_ERR_INVALID,
                 "edp_sample_deliver: uniform draws carry no priorities (q/isw must be NULL)");
-  const edp_status st = deliver_checks(ctx, idx, batch, out);
+  edp_batch res;
+  const edp_status st = deliver_checks(ctx, idx, batch, out, &res);
   if (st != EDP_OK) return st;
   cudaSetDevice(ctx->cfg.device);
   DrawUniform d{seed, round, idx};
-  cudaError_t e = launch_deliver(ctx, idx, batch, out, (cudaStream_t)stream, &d);
+  cudaError_t e = launch_deliver(ctx, idx, batch, &res, (cudaStream_t)stream, &d);
   if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_sample_deliver");
   return EDP_OK;
 }
