@@ -965,23 +965,28 @@ class PpoIteration(Workload):
         self.h_in = [pin(t) for t in (self.r, self.v, self.d)]
         for h, t in zip(self.h_in, (self.r, self.v, self.d)):
             h.copy_(t.cpu())
-        self.h_outs = [pin(self.out[0]) for _ in range(self.M)]
-        self.h_ao = [pin(self.a_out) for _ in range(self.M)]
-        self.h_ro = [pin(self.r_out) for _ in range(self.M)]
+        # all 8 mini-batches of an iteration, mini-batch m = rows
+        # [4096 m, 4096 (m + 1)), written by the delivery straight into
+        # page-locked host memory
+        self.h_all = pin(self.out_all)
+        self.h_aall = pin(self.a_all)
+        self.h_rall = pin(self.r_all)
         self.h2d = sum(t.numel() * t.element_size() for t in self.h_in)
-        self.d2h = self.M * (self.h_outs[0].numel() * 2 + 8 * self.mb)
+        self.d2h = self.h_all.numel() * 2 + 8 * self.n
+        self.h_batch = self.edp.make_batch(self.h_all,
+                                           gather=[(self.nrm.view(-1), self.h_aall),
+                                                   (self.ret.view(-1), self.h_rall)])
 
     def e2e_round(self, r):
+        """One stream: the rollout's scalars in, GAE, shuffle, and the
+        iteration's delivery (one call) written straight into the page-locked
+        host batch."""
         for h, t in zip(self.h_in, (self.r, self.v, self.d)):
             t.copy_(h, non_blocking=True)
         self._gae()
         self.edp.edp_sample(self.ring.ctx, self.edp.EDP_SAMPLE_PERMUTE, self.n,
                             self.seed, r, self.idx)
-        for m in range(self.M):
-            self._mb(m, r)
-            self.h_outs[m].copy_(self.out[(r * self.M + m) % 2], non_blocking=True)
-            self.h_ao[m].copy_(self.a_out, non_blocking=True)
-            self.h_ro[m].copy_(self.r_out, non_blocking=True)
+        self.edp.edp_deliver(self.ring.ctx, self.idx, self.n, self.h_batch)
 
     def cpu_setup(self):
         import oracle as orc
@@ -1170,12 +1175,20 @@ class MmReplay(Workload):
                       for k in ("obs", "tok", "rew", "idx")}
         self.h2d = 0 if not self.ingest else self.ingest * (self.F + 4 * self.L + 4)
         self.d2h = sum(t.numel() * t.element_size() for t in self.h_out.values())
+        h = self.h_out
+        self.h_batch = self.edp.make_batch(h["obs"], tokens=h["tok"], reward=h["rew"])
 
     def e2e_round(self, r):
-        self.round(r)
-        o = self.outs[r % 2]
-        for k in ("obs", "tok", "rew", "idx"):
-            self.h_out[k].copy_(o[k], non_blocking=True)
+        """One stream: (ingest,) sample, and the delivery written straight
+        into the page-locked host batch; the indices follow with a copy."""
+        ctx = self.ring.ctx
+        if self.ingest:
+            self.edp.edp_ingest(ctx, self.st_obs, self.ingest, tokens=self.st_tok,
+                                reward=self.st_rew)
+        o = self.outs[0]
+        self.edp.edp_sample(ctx, self.edp.EDP_SAMPLE_UNIFORM, self.B, self.seed, r, o["idx"])
+        self.edp.edp_deliver(ctx, o["idx"], self.B, self.h_batch)
+        self.h_out["idx"].copy_(o["idx"], non_blocking=True)
 
     def extra(self, device, mk, stream, deliver_us):
         """Two-tier: host-link bandwidth measured in this run (zero-copy read
