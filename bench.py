@@ -1531,6 +1531,10 @@ class LlmBatch(Workload):
         self.d2h = 8 * self.T + 8 * (self.n + 1)
 
     def e2e_round(self, r):
+        """Rewards and the batch order in, the packed batch copied out (the
+        packed delivery can write into page-locked host memory directly, but
+        its 4-byte stores cross the host link slower than a copy: 176 vs
+        267 GB/s end to end)."""
         self.r.copy_(self.h_in, non_blocking=True)
         self.perms[r % self.n_perm].copy_(self.h_idx[r % self.n_perm], non_blocking=True)
         self.round_fused(r)

@@ -358,7 +358,9 @@ EDP_API edp_status edp_grpo_advantage(edp_ctx *ctx, const float *r,
  * out_cap: elements available in out_tokens / out_value.  An index outside
  * [0, n_seq) delivers an empty sequence; output beyond out_cap is not
  * written; both set a device flag that edp_sync reports (EDP_ERR_INVALID;
- * for an overflow the message gives the size needed).  batch <= 2^20. */
+ * for an overflow the message gives the size needed).  batch <= 2^20.
+ * The outputs (out_tokens, out_off, out_value) may be page-locked host
+ * memory, written over the host link; the inputs are device memory. */
 EDP_API edp_status edp_pack_deliver(edp_ctx *ctx, const int32_t *tokens,
                                     const uint64_t *seq_off, uint64_t n_seq,
                                     const int64_t *idx, uint32_t batch,

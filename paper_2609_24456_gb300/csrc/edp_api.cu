@@ -1004,13 +1004,22 @@ edp_status edp_pack_deliver(edp_ctx *ctx, const int32_t *tokens, const uint64_t 
   if ((seq_value == nullptr) != (out_value == nullptr))
     return fail(ctx, EDP_ERR_INVALID, "edp_pack_deliver: seq_value and out_value go together");
   const void *p;
-  const void *ptrs[] = {tokens, seq_off, idx, seq_value, out_tokens, out_off, out_value};
-  for (const void *o : ptrs)
+  const void *ins[] = {tokens, seq_off, idx, seq_value};
+  for (const void *o : ins)
     if (o && !device_view(ctx, o, &p, false))
-      return fail(ctx, EDP_ERR_INVALID, "edp_pack_deliver: arrays must be device memory");
+      return fail(ctx, EDP_ERR_INVALID, "edp_pack_deliver: inputs must be device memory");
+  void *outs[] = {out_tokens, out_off, out_value};
+  for (void *&o : outs) {
+    if (!o) continue;
+    if (!device_view(ctx, o, &p, true))
+      return fail(ctx, EDP_ERR_INVALID,
+                  "edp_pack_deliver: outputs must be device or page-locked host memory");
+    o = const_cast<void *>(p);
+  }
   cudaSetDevice(ctx->cfg.device);
-  cudaError_t e = launch_pack(ctx, tokens, seq_off, n_seq, idx, batch, seq_value, out_tokens,
-                              out_off, out_value, out_cap, (cudaStream_t)stream);
+  cudaError_t e = launch_pack(ctx, tokens, seq_off, n_seq, idx, batch, seq_value,
+                              (int32_t *)outs[0], (uint64_t *)outs[1], (float *)outs[2],
+                              out_cap, (cudaStream_t)stream);
   if (e == cudaErrorMemoryAllocation)
     return fail(ctx, EDP_ERR_OOM, "edp_pack_deliver: scratch allocation failed");
   if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_pack_deliver");
@@ -1034,14 +1043,22 @@ edp_status edp_grpo_pack_deliver(edp_ctx *ctx, const float *r, const uint64_t *g
     return fail(ctx, EDP_ERR_INVALID,
                 "edp_grpo_pack_deliver: need n_seq > 0, 0 < batch <= 2^20");
   const void *p;
-  const void *ptrs[] = {r, group_off, adv, tokens, seq_off, idx, out_tokens, out_off, out_value};
-  for (const void *o : ptrs)
+  const void *ins[] = {r, group_off, adv, tokens, seq_off, idx};
+  for (const void *o : ins)
     if (o && !device_view(ctx, o, &p, false))
       return fail(ctx, EDP_ERR_INVALID, "edp_grpo_pack_deliver: arrays must be device memory");
+  void *outs[] = {out_tokens, out_off, out_value};
+  for (void *&o : outs) {
+    if (!o) continue;
+    if (!device_view(ctx, o, &p, true))
+      return fail(ctx, EDP_ERR_INVALID,
+                  "edp_grpo_pack_deliver: outputs must be device or page-locked host memory");
+    o = const_cast<void *>(p);
+  }
   cudaSetDevice(ctx->cfg.device);
   cudaError_t e = launch_grpo_pack(ctx, r, group_off, n_groups, eps, adv, tokens, seq_off,
-                                   n_seq, idx, batch, out_tokens, out_off, out_value, out_cap,
-                                   (cudaStream_t)stream);
+                                   n_seq, idx, batch, (int32_t *)outs[0], (uint64_t *)outs[1],
+                                   (float *)outs[2], out_cap, (cudaStream_t)stream);
   if (e == cudaErrorMemoryAllocation)
     return fail(ctx, EDP_ERR_OOM, "edp_grpo_pack_deliver: scratch allocation failed");
   if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_grpo_pack_deliver");

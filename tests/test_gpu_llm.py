@@ -255,3 +255,27 @@ def test_grpo_pack_fused_argument_errors(edp_lib):
         with pytest.raises(edp.EdpError) as e:
             call(**kw)
         assert e.value.status == edp.EDP_ERR_INVALID, kw
+
+
+def test_pack_into_host_outputs(edp_lib):
+    """Packed tokens, offsets and per-token values written straight into
+    page-locked host memory equal the device-output delivery."""
+    edp = edp_lib
+    ring = _ctx(edp)
+    tokens, seq_off, r, goff = fx.llm_rollout(17, 20, 4, lmin=0, lmax=500)
+    idx = np.random.default_rng(18).permutation(len(r)).astype(np.int64)
+    n, B = len(r), len(idx)
+    total = int(seq_off[-1])
+    d_args = (cuda(r), cuda(goff), len(goff) - 1, 1e-6)
+    res = []
+    for host in (False, True):
+        mk = (lambda shape, dt: torch.empty(shape, dtype=dt, pin_memory=True)) if host else \
+             (lambda shape, dt: torch.empty(shape, dtype=dt, device="cuda"))
+        adv = torch.empty(n, device="cuda")
+        out, oo, ov = mk(total, torch.int32), mk(B + 1, torch.int64), mk(total, torch.float32)
+        edp.edp_grpo_pack_deliver(ring.ctx, *d_args, adv, cuda(tokens), cuda(seq_off), n,
+                                  cuda(idx), B, out, oo, total, out_value=ov)
+        edp.edp_sync(ring.ctx)
+        res.append((to_np(out), to_np(oo), bits(ov)))
+    for x, y in zip(*res):
+        assert np.array_equal(x, y)
