@@ -476,31 +476,37 @@ class PerReplay(Workload):
         pin = lambda *s, dt=torch.float32: torch.empty(s, dtype=dt, pin_memory=True)
         self.h_td = pin(self.td_rounds, B)
         self.h_td.copy_(self.td.cpu())
-        self.h_out = dict(obs=pin(B, K, F), nxt=pin(B, K, F),
-                          act=pin(B, dt=torch.int32), rew=pin(B),
-                          done=pin(B, dt=torch.uint8), isw=pin(B),
-                          idx=pin(B, dt=torch.int64))
+        # one page-locked host batch per rotating output set; the batch's
+        # outputs are these host buffers, q stays on the device (the
+        # sampler's)
+        self.h_outs = [dict(obs=pin(B, K, F), nxt=pin(B, K, F),
+                            act=pin(B, dt=torch.int32), rew=pin(B),
+                            done=pin(B, dt=torch.uint8), isw=pin(B),
+                            idx=pin(B, dt=torch.int64)) for _ in range(self.R)]
+        self.h_batches = [self.edp.make_batch(h["obs"], h["nxt"], h["act"], h["rew"],
+                                              h["done"], q=o["q"], isw=h["isw"], beta=BETA)
+                          for h, o in zip(self.h_outs, self.outs)]
         self.d_td = torch.empty(B, device=device)
         self.h2d = B * 4
-        self.d2h = sum(t.numel() * t.element_size() for t in self.h_out.values())
-        # the batch's outputs are the host buffers themselves; q stays on the
-        # device (written there by the sampler)
-        h = self.h_out
-        self.h_batch = self.edp.make_batch(h["obs"], h["nxt"], h["act"], h["rew"], h["done"],
-                                           q=self.outs[0]["q"], isw=h["isw"], beta=BETA)
+        self.d2h = sum(t.numel() * t.element_size() for t in self.h_outs[0].values())
 
     def e2e_round(self, r):
-        """User path with host buffers: TD errors in, learner batch out --
-        delivered by the kernel straight into the page-locked host batch
-        (one output set: the e2e rounds run on one stream)."""
-        o = self.outs[0]
-        h = self.h_out
+        """User path with host buffers, in the main schedule: TD errors in,
+        and each round's learner batch delivered by the kernel straight into
+        a page-locked host batch on a side stream while the update and the
+        next sampling run (the indices follow with a copy)."""
+        k = r % self.R
+        o, h = self.outs[k], self.h_outs[k]
+
+        def deliver(st):
+            self.edp.edp_deliver(self.ring.ctx, o["idx"], self.B, self.h_batches[k], stream=st)
+            h["idx"].copy_(o["idx"], non_blocking=True)
+
         self.d_td.copy_(self.h_td[r % self.td_rounds], non_blocking=True)
-        self._sample(r, o)
-        self.edp.edp_deliver(self.ring.ctx, o["idx"], self.B, self.h_batch)
-        self.edp.edp_update_priorities_td(self.ring.ctx, o["idx"], self.d_td,
-                                          self.B, ALPHA, EPS)
-        h["idx"].copy_(o["idx"], non_blocking=True)
+        self._overlapped(
+            k, lambda: self._sample(r, o), deliver,
+            lambda: self.edp.edp_update_priorities_td(
+                self.ring.ctx, o["idx"], self.d_td, self.B, ALPHA, EPS))
 
     def cpu_setup(self, host_frames=262_144):
         import numpy as np
@@ -1714,6 +1720,7 @@ def run_edp(args):
         Ke = min(K, args.e2e_steps)
         for r in range(3):
             wl.e2e_round(r)
+        wl.join()
         torch.cuda.synchronize()
         if dist:
             dist.barrier()
@@ -1721,6 +1728,7 @@ def run_edp(args):
         e0.record(stream)
         for r in range(Ke):
             wl.e2e_round(r)
+        wl.join()  # side streams a schedule used
         e1.record(stream)
         torch.cuda.synchronize()
         ems = job_ms(e0.elapsed_time(e1), dist, device)
