@@ -623,17 +623,31 @@ class DqnTiny(Workload):
                           done=pin(B, dt=torch.uint8), idx=pin(B, dt=torch.int64))
         self.h2d = 0
         self.d2h = sum(t.numel() * t.element_size() for t in self.h_out.values())
-        h = self.h_out
-        self.h_batch = self.edp.make_batch(h["obs"], h["nxt"], h["act"], h["rew"], h["done"])
+        self.h_outs = [self.h_out] + [{k: torch.empty_like(t, pin_memory=True)
+                                       for k, t in self.h_out.items()}]
+        self.h_batches = [self.edp.make_batch(h["obs"], h["nxt"], h["act"], h["rew"],
+                                              h["done"]) for h in self.h_outs]
+        self.sides = [torch.cuda.Stream(device=device) for _ in range(2)]
 
     def e2e_round(self, r):
         """The main schedule's call with host buffers: the kernel draws the
-        batch and writes it straight into the page-locked host batch; the
-        indices (device) follow with a copy."""
-        o = self.outs[0]
-        self.edp.edp_sample_deliver(self.ring.ctx, self.B, self.seed, r, o["idx"],
-                                    self.h_batch)
-        self.h_out["idx"].copy_(o["idx"], non_blocking=True)
+        batch and writes it straight into a page-locked host batch, the
+        calls alternating between two side streams (each writes its own host
+        batch, so stream order protects its reuse) so consecutive batches
+        overlap; the indices (device) follow with a copy."""
+        import torch
+        k = r % 2
+        o, side = self.outs[k], self.sides[k]
+        if not getattr(self, "side_used", False):
+            fork = torch.cuda.Event()
+            fork.record()
+            for st in self.sides:
+                st.wait_event(fork)
+        self.side_used = True
+        with torch.cuda.stream(side):
+            self.edp.edp_sample_deliver(self.ring.ctx, self.B, self.seed, r, o["idx"],
+                                        self.h_batches[k], stream=side)
+            self.h_outs[k]["idx"].copy_(o["idx"], non_blocking=True)
 
     def cpu_setup(self):
         import numpy as np
