@@ -259,7 +259,8 @@ EDP_API edp_status edp_sample(edp_ctx *ctx, edp_sample_mode mode, uint32_t batch
 /* Delivery (Sec. 2.2: the chosen transitions are materialised in the
  * learner's batch layout): fused gather + transform + collate (+ IS
  * weights) of the `batch` slots in idx (device int64).  A slot outside the
- * sampleable range is reported by edp_sync and its outputs are zeroed. */
+ * sampleable range is reported by edp_sync and its outputs are zeroed.
+ * The batch's outputs may be device or page-locked host memory (edp_batch). */
 EDP_API edp_status edp_deliver(edp_ctx *ctx, const int64_t *idx, uint32_t batch,
                        const edp_batch *out, edp_stream stream);
 
