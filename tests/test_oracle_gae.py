@@ -75,4 +75,16 @@ def test_normalize_matches_numpy(orc):
     out, m, s = orc.normalize(a)
     assert np.isclose(m, a.mean(), rtol=0, atol=1e-12)
     assert np.isclose(s, a.std(ddof=1), rtol=1e-12)
-    assert np.allclose(out, (a - a.mean()) / (a.std(ddof=1) + 1e-8), atol=1e-12)
+    ref = (a - a.mean()) / (a.std(ddof=1) + 1e-8)
+    assert np.allclose(out, ref, rtol=0, atol=1e-12)
+    # the 1e-8 sits in the denominator: it is visible at a small spread
+    b = np.random.default_rng(6).standard_normal(4096) * 1e-6
+    outb, _, _ = orc.normalize(b)
+    assert np.allclose(outb, (b - b.mean()) / (b.std(ddof=1) + 1e-8), rtol=1e-12, atol=0)
+
+
+def test_normalize_constant_rollout_is_zero(orc):
+    # zero spread: the advantages are all equal and normalise to 0, not NaN
+    out, m, s = orc.normalize(np.full(1024, 0.5))
+    assert m == 0.5 and s == 0.0
+    assert np.array_equal(out, np.zeros(1024))

@@ -10,6 +10,7 @@ def test_permutation_is_sorted_random_keys(orc, n):
     keys = np.array([orc.philox_u64(123, j, 4, 2) for j in range(n)],
                     dtype=np.uint64)
     ref = np.lexsort((np.arange(n), keys))  # numpy: by key, then index
+    assert len(np.unique(keys)) == n  # so the index tie-break never decides
     assert np.array_equal(perm, ref)
 
 

@@ -75,3 +75,19 @@ def test_uniform_sampler_offsets_follow_ring(orc):
     offs = (idx - oldest) % cap
     assert offs.max() < cap - 1  # the newest transition is never drawn
     assert len(np.unique(offs)) > 90
+
+
+def test_uniform_sampler_is_stream_zero(orc):
+    # draw k of the uniform sampler is the Philox block at counter
+    # (k, round lo32, stream 0, round hi32) -- the block function is pinned by
+    # the known answers above -- reduced to an offset by an exact 128-bit
+    # multiply-high; streams 1 and 2 belong to the stratified sampler and
+    # the shuffle keys, so reusing one of them would correlate the two
+    cap, total, n_valid, seed, rnd = 1000, 2345, 999, 0xDEADBEEF12345678, (3 << 32) | 7
+    idx = orc.sample_uniform(cap, total, n_valid, 64, seed, rnd)
+    key = [seed & 0xFFFFFFFF, seed >> 32]
+    oldest = total % cap
+    for k in range(64):
+        o = orc.philox4x32_10([k, rnd & 0xFFFFFFFF, 0, rnd >> 32], key)
+        u = (int(o[1]) << 32) | int(o[0])
+        assert idx[k] == (oldest + ((u * n_valid) >> 64)) % cap

@@ -68,3 +68,45 @@ def test_norm_chw_matches_per_element(orc):
         lut = np.array([orc.norm_bf16(b, MEANS[c], STDS[c]) for b in range(256)],
                        np.uint16)
         assert np.array_equal(out[c], lut[img[c]])
+
+
+def _bf16(x):
+    import torch
+    return torch.from_numpy(np.ascontiguousarray(x, np.float32)).to(
+        torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+
+
+def test_deliver_ppo_scalars_follow_logical_offset(orc):
+    # a wrapped ring: ids 5..12 in 8 slots, id L in slot L mod 8; a sample's
+    # advantage and return are those of its logical offset (its position
+    # from the oldest stored transition), its image the slot's, CHW
+    H, W, Cc, cap, total = 2, 3, 3, 8, 13
+    rng = np.random.default_rng(11)
+    ring = rng.integers(0, 256, (cap, H * W * Cc), dtype=np.uint8)
+    ids = list(range(total - cap, total))
+    adv = np.arange(cap, dtype=np.float32) + 100
+    ret = -np.arange(cap, dtype=np.float32)
+    idx = np.array([0, 4, 5, 7, 4, 2], np.int64)
+    out, a, r = orc.deliver_ppo(ring, cap, total, H, W, Cc, idx, adv, ret)
+    for b, s in enumerate(idx):
+        k = [L % cap for L in ids].index(s)
+        assert a[b] == 100 + k and r[b] == -k
+        img = ring[s].reshape(H, W, Cc).transpose(2, 0, 1).astype(np.float32) / np.float32(255)
+        assert np.array_equal(out[b], _bf16(img))
+
+
+def test_deliver_mm_collates(orc):
+    Cc, HW, L, cap = 3, 10, 5, 7
+    rng = np.random.default_rng(12)
+    ring = rng.integers(0, 256, (cap, Cc * HW), dtype=np.uint8)
+    tok = rng.integers(0, 32000, (cap, L), dtype=np.int32)
+    rew = rng.standard_normal(cap).astype(np.float32)
+    idx = np.array([6, 0, 3, 3, 1], np.int64)
+    m = np.array(MEANS, np.float32)
+    sd = np.array(STDS, np.float32)
+    out, t, r = orc.deliver_mm(ring, tok, rew, Cc, HW, idx, m, sd)
+    assert np.array_equal(t, tok[idx])
+    assert np.array_equal(r, rew[idx])
+    x = ring[idx].reshape(len(idx), Cc, HW).astype(np.float32) / np.float32(255)
+    y = (x - m[None, :, None]) / sd[None, :, None]
+    assert np.array_equal(out.reshape(len(idx), Cc, HW), _bf16(y))
