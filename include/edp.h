@@ -423,8 +423,10 @@ EDP_API edp_status edp_migrate(const edp_ctx *src, edp_ctx *dst, edp_stream stre
  * the newest min(saved, capacity) transitions become its first insertions,
  * placed by its own tier map, and its tree is rebuilt on `stream`.  Both
  * stage the data through 64 MiB of host memory and synchronise.
- * EDP_ERR_INVALID for an unreadable, foreign or truncated file (the context
- * is left empty), EDP_ERR_STATE for a non-empty context or another layout. */
+ * EDP_ERR_INVALID for an unreadable or foreign file, or one whose size is
+ * not the size its header describes (checked before anything is written;
+ * after a later read error the context is reset to empty, priorities
+ * included), EDP_ERR_STATE for a non-empty context or another layout. */
 EDP_API edp_status edp_save(edp_ctx *ctx, const char *path, edp_stream stream);
 EDP_API edp_status edp_load(edp_ctx *ctx, const char *path, edp_stream stream);
 

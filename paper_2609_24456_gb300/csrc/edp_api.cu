@@ -381,6 +381,7 @@ edp_status edp_create(const edp_config *cfg, const edp_storage *st,
     }
     const size_t bytes = internal * 8 + n * 4;
     c->tree_mem = al(cfg->alloc_user, bytes);
+    c->tree_bytes = bytes;
     if (!c->tree_mem) {
       free_all(c);
       delete c;
@@ -498,6 +499,19 @@ void slot_runs(uint64_t cap, uint64_t L0, uint64_t n, F fn) {
   }
 }
 
+// Bytes a checkpoint of n transitions with header h occupies: the header,
+// then per transition its payload rows and the metadata arrays it carries.
+// False when the count cannot be a real checkpoint's (the product would
+// overflow).
+bool ckpt_bytes(const CkptHeader &h, uint64_t *out) {
+  const uint64_t per = h.obs_bytes + h.tok_bytes + 4u * (h.has_action != 0) +
+                       4u * (h.has_reward != 0) + 1u * (h.has_done != 0) +
+                       4u * (h.prioritized != 0);
+  if (h.n > (UINT64_MAX - sizeof(CkptHeader)) / (per ? per : 1)) return false;
+  *out = sizeof(CkptHeader) + h.n * per;
+  return true;
+}
+
 bool same_layout(const edp_ctx *c, const CkptHeader &h) {
   const edp_config &g = c->cfg;
   return h.transform == g.transform && h.obs_c == g.obs_c && h.obs_h == g.obs_h &&
@@ -594,6 +608,17 @@ edp_status edp_load(edp_ctx *ctx, const char *path, edp_stream stream) {
     std::fclose(f);
     return fail(ctx, EDP_ERR_STATE, "edp_load: the checkpoint's layout differs from the context's");
   }
+  // a truncated or padded file is refused before anything is written
+  uint64_t want = 0;
+  long have = -1;
+  if (std::fseek(f, 0, SEEK_END) == 0) have = std::ftell(f);
+  if (!ckpt_bytes(h, &want) || have < 0 || (uint64_t)have != want ||
+      std::fseek(f, (long)sizeof h, SEEK_SET) != 0) {
+    std::fclose(f);
+    return fail(ctx, EDP_ERR_INVALID,
+                "edp_load: %s holds %ld bytes, its header describes %llu (truncated file?)", path,
+                have, (unsigned long long)want);
+  }
   cudaSetDevice(ctx->cfg.device);
   const uint64_t n = h.n < ctx->cap ? h.n : ctx->cap;  // the newest n are kept
   const uint64_t skip = h.n - n;
@@ -640,10 +665,19 @@ edp_status edp_load(edp_ctx *ctx, const char *path, edp_stream stream) {
     if (e == cudaSuccess) e = launch_tree_build_all(ctx, (cudaStream_t)stream);
   }
   if (!ok || e != cudaSuccess) {
+    // back to an empty context: no transition, and no leaf or sum left over
+    // from the rows read before the failure
     ctx->total = 0;
     cudaGetLastError();
-    return fail(ctx, staged ? EDP_ERR_INVALID : EDP_ERR_OOM,
-                "edp_load: reading %s failed (truncated file?)", path);
+    if (ctx->depth) {
+      const uint32_t pm[2] = {0, 1u << 20};
+      cudaStreamSynchronize((cudaStream_t)stream);
+      cudaMemset(ctx->tree_mem, 0, ctx->tree_bytes);
+      cudaMemcpy(&ctx->ctrl->pending_q, pm, sizeof pm, cudaMemcpyHostToDevice);
+      cudaGetLastError();
+    }
+    return fail(ctx, staged ? EDP_ERR_INVALID : EDP_ERR_OOM, "edp_load: reading %s failed",
+                path);
   }
   return EDP_OK;
 }

@@ -57,6 +57,7 @@ struct edp_ctx {
   uint32_t *leaves = nullptr;
   uint64_t *level[edp::kMaxDepth] = {};
   void *tree_mem = nullptr;
+  size_t tree_bytes = 0;  // internal sums and leaves, one block
   edp::Ctrl *ctrl = nullptr;
   // lazily grown scratch (shuffle, GAE partials)
   void *scratch = nullptr;

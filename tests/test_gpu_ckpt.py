@@ -104,3 +104,39 @@ def test_load_errors(edp_lib, orc, tmp_path):
             edp.edp_load(dst.ctx, str(f))
         assert e.value.status == edp.EDP_ERR_INVALID
         assert dst.info().total == 0
+
+
+def test_failed_load_leaves_prioritized_context_empty(edp_lib, orc, tmp_path):
+    """A truncated or padded checkpoint is refused before anything reaches
+    the context; the context then works as a fresh one (every leaf and sum,
+    the deferred and running-maximum priorities)."""
+    edp = edp_lib
+    Fb = 84 * 16
+    frames, action, reward, done = fx.dqn_transitions(71, 700, Fb, done_p=0.05)
+    q = orc.priorities_from_td(fx.td_errors(71, 700), 0.6, 1e-6)
+    src = MirroredDqn(500, prioritized=True, F=Fb)
+    src.ingest(orc, frames[:400], action[:400], reward[:400], done[:400], q=q[:400])
+    src.ingest(orc, frames[400:600], action[400:600], reward[400:600], done[400:600],
+               q=q[400:600])
+    good = tmp_path / "per.edp"
+    edp.edp_save(src.ring.ctx, str(good))
+    raw = good.read_bytes()
+    cut = tmp_path / "cut.edp"
+    cut.write_bytes(raw[:-100])  # ends inside the leaves
+    pad = tmp_path / "pad.edp"
+    pad.write_bytes(raw + bytes(4))
+    dst = MirroredDqn(500, prioritized=True, F=Fb)
+    for f in (cut, pad):
+        with pytest.raises(edp.EdpError) as e:
+            edp.edp_load(dst.ring.ctx, str(f))
+        assert e.value.status == edp.EDP_ERR_INVALID
+        assert dst.ring.info().total == 0
+    sl = slice(600, 700)
+    dst.ingest(orc, frames[sl], action[sl], reward[sl], done[sl], q=q[sl])
+    edp.edp_sync(dst.ring.ctx)
+    check_tree(orc, dst.ring, dst.st)
+    # and the intact file still loads into a fresh context
+    fresh = MirroredDqn(500, prioritized=True, F=Fb)
+    edp.edp_load(fresh.ring.ctx, str(good))
+    edp.edp_sync(fresh.ring.ctx)
+    assert fresh.ring.info().total == 500
