@@ -1759,6 +1759,11 @@ def run_edp(args):
                 "traffic": kernel_traffic(wl.kernel, wl.name),
                 "algorithmic_bytes_per_launch": wl.deliver_bytes,
                 "avg_launch_us": avg_deliver_s * 1e6, "launches_timed": Kd}
+    if getattr(wl, "tiered", False):
+        # the HBM fraction understates this launch: its host-tier share is
+        # read over the host link, whose fraction host_link reports
+        roofline["note"] = ("two-tier: %.0f%% of the samples are read over the host link; "
+                            "see host_link.frac_of_link" % (100.0 * (wl.cap - wl.cap_h) / wl.cap))
 
     extra = {}
     if hasattr(wl, "extra") and not args.no_extra:
