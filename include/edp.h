@@ -323,7 +323,8 @@ EDP_API edp_status edp_priorities_from_td(edp_ctx *ctx, const float *td, uint32_
  *   ret_t = A_t + V_t
  *   adv_norm = (A - mean(A)) / (std(A) + 1e-8), std with n-1, over T*E
  * Computed in fp64, stored fp32 [T][E].  adv/ret/adv_norm may be NULL
- * individually.  T*E >= 2. */
+ * individually.  T, E >= 1 and T*E < 2^31 (else EDP_ERR_INVALID); with a
+ * single value (T*E == 1) the spread is 0 and adv_norm is 0. */
 EDP_API edp_status edp_gae(edp_ctx *ctx, const float *r, const float *v,
                    const uint8_t *d, uint32_t T, uint32_t E, double gamma,
                    double lambda, float *adv, float *ret, float *adv_norm,

@@ -989,8 +989,8 @@ edp_status edp_gae(edp_ctx *ctx, const float *r, const float *v,
                    edp_stream stream) {
   if (!ctx) return EDP_ERR_INVALID;
   if (!r || !v || !d) return fail(ctx, EDP_ERR_INVALID, "edp_gae: r/v/d NULL");
-  if (T == 0 || E == 0 || (uint64_t)T * E < 2 || (uint64_t)T * E > 0x7FFFFFFFull)
-    return fail(ctx, EDP_ERR_INVALID, "edp_gae: need 2 <= T*E < 2^31");
+  if (T == 0 || E == 0 || (uint64_t)T * E > 0x7FFFFFFFull)
+    return fail(ctx, EDP_ERR_INVALID, "edp_gae: need T, E >= 1 and T*E < 2^31");
   if (!std::isfinite(gamma) || !std::isfinite(lambda))
     return fail(ctx, EDP_ERR_INVALID, "edp_gae: gamma/lambda not finite");
   const void *p;

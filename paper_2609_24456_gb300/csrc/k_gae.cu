@@ -236,10 +236,13 @@ k_gae_norm(const float *A_src, float *adv_norm, uint64_t n, const double *partia
   if (threadIdx.x == 0) {
     const double nn = (double)n;
     const double mean = r1[0] / nn;
-    double var = (r2[0] - r1[0] * mean) / (nn - 1.0);
+    double var = n > 1 ? (r2[0] - r1[0] * mean) / (nn - 1.0) : 0.0;
     if (var < 0.0) var = 0.0;
     stat[0] = mean;
-    stat[1] = 1.0 / (sqrt(var) + 1e-8);
+    // a single value equals its mean and normalises to exactly 0; the scale
+    // is 0 so that the fp32 rounding of the stored A (A - mean ~ 2^-24 |A|
+    // here) is not multiplied by 1 / 1e-8
+    stat[1] = n > 1 ? 1.0 / (sqrt(var) + 1e-8) : 0.0;
   }
   __syncthreads();
   const double mean = stat[0], inv = stat[1];

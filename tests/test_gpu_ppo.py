@@ -32,7 +32,8 @@ def _gae(edp, ring, r, v, d, want=(True, True, True)):
                                         (200, 3, 0.01), (1, 2, 0.5),
                                         (2, 1, 0.0), (300, 130, 0.02),
                                         (129, 8, 1.0),
-                                        (5, 512, 0.02), (4, 513, 0.02), (3, 700, 0.01)])
+                                        (5, 512, 0.02), (4, 513, 0.02), (3, 700, 0.01),
+                                        (1, 1, 0.0), (1, 1, 1.0)])
 def test_gae_matches_oracle(edp_lib, orc, T, E, done_p):
     edp = edp_lib
     _, r, v, d = fx.ppo_rollout(T * 1000 + E, T, E, done_p=done_p, with_obs=False)
@@ -43,6 +44,25 @@ def test_gae_matches_oracle(edp_lib, orc, T, E, done_p):
     assert np.abs(to_np(adv) - ra).max() <= 1e-5
     assert np.abs(to_np(ret) - rr).max() <= 1e-5
     assert np.abs(to_np(nrm).ravel() - rn).max() <= 1e-5
+
+
+def test_gae_single_value_and_bad_shapes(edp_lib, orc):
+    # one step of one environment: A = delta, and it normalises to 0
+    edp = edp_lib
+    ring = _ppo_ring(edp, 64)
+    r = np.array([[0.75]], np.float32)
+    v = np.array([[0.5], [2.0]], np.float32)
+    d = np.zeros((1, 1), np.uint8)
+    adv, ret, nrm = _gae(edp, ring, r, v, d)
+    delta = 0.75 + G * 2.0 - 0.5
+    assert abs(float(adv[0, 0]) - delta) <= 1e-6
+    assert abs(float(ret[0, 0]) - (delta + 0.5)) <= 1e-6
+    assert float(nrm[0, 0]) == 0.0
+    z = torch.zeros(4, device="cuda")
+    for T, E in [(0, 4), (4, 0), (1 << 16, 1 << 15)]:
+        with pytest.raises(edp.EdpError) as e:
+            edp.edp_gae(ring.ctx, z, z, z, T, E, G, LAM, z, None, None)
+        assert e.value.status == edp.EDP_ERR_INVALID
 
 
 def test_gae_optional_outputs(edp_lib, orc):
