@@ -162,3 +162,7 @@ def test_priority_from_td(orc):
     ref = np.rint((np.abs(td.astype(np.float64)) + 1e-6) ** 0.6 * 2.0**20)
     ref = np.clip(ref, 1, 2**32 - 1).astype(np.uint32)
     assert np.array_equal(q, ref)
+    # both ends of the clamp to [1, 2^32 - 1]: a zero error without eps, and
+    # errors whose priority exceeds 32 bits
+    q0 = orc.priorities_from_td(np.array([0.0, 1e9, -1e9], np.float32), 0.6, 0.0)
+    assert q0.tolist() == [1, 2**32 - 1, 2**32 - 1]

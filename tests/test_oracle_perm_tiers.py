@@ -35,8 +35,10 @@ def test_tier_map_against_physical_simulation(orc):
         cap = cap_h + cap_c
         hbm, host = [], []  # logical ids, oldest first
         total = 0
-        for _ in range(25):
-            n = int(rng.integers(0, cap + 1))
+        for step in range(25 + 2 * cap):
+            # one at a time while the tiers fill (HBM partly full, then the
+            # host tier), then random batches
+            n = 1 if step < 2 * cap else int(rng.integers(0, cap + 1))
             for j in range(n):
                 if len(hbm) == cap_h:
                     if len(host) == cap_c:

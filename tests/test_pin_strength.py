@@ -142,6 +142,35 @@ MUTANTS = [
     ("tier-boundary", C, "} else if (L >= total - in_hbm) {", "} else if (L > total - in_hbm) {"),
     ("tier-host-slot", C, "*slot = L % (cap - cap_h);", "*slot = L % cap_h;"),
     ("tier-evicted-kept", C, "if (L >= total || L < total - size) {", "if (L >= total) {"),
+    # more row lookups, bounds and clamps
+    ("philox-key-bumped-first", C, "    if (r > 0) {\n      k0 += PHILOX_W0;",
+     "    if (r >= 0) {\n      k0 += PHILOX_W0;"),
+    ("philox-key-word-swap", C, "uint32_t n0 = (uint32_t)(p1 >> 32) ^ x1 ^ k0;",
+     "uint32_t n0 = (uint32_t)(p1 >> 32) ^ x1 ^ k1;"),
+    ("leaf-sum-drops-last", C, "for (uint64_t i = lo; i < hi; ++i) s += leaves[i];",
+     "for (uint64_t i = lo; i + 1 < hi; ++i) s += leaves[i];"),
+    ("scan-q-of-next", C, "qout[k] = leaves[i];", "qout[k] = leaves[(i + 1) % cap];"),
+    ("bisect-prefix-offset", C, "  prefix[0] = 0;\n", "  prefix[0] = 1;\n"),
+    ("td-clamp-low", C, "if (!(r >= 1.0)) r = 1.0;", "if (!(r >= 0.0)) r = 0.0;"),
+    ("td-clamp-high", C, "if (r > 4294967295.0) r = 4294967295.0;",
+     "if (r > 4294967294.0) r = 4294967294.0;"),
+    ("dqn-done-of-next", C, "if (done_out) done_out[b] = done[s];",
+     "if (done_out) done_out[b] = done[(s + 1) % cap];"),
+    ("ppo-image-of-previous", C,
+     "orc_hwc_to_chw_bf16(obs_ring + s * F, H, W, C, obs_out + (uint64_t)b * F);",
+     "orc_hwc_to_chw_bf16(obs_ring + (s ? s - 1 : 0) * F, H, W, C, obs_out + (uint64_t)b * F);"),
+    ("mm-image-of-previous", C, "orc_norm_chw_bf16(obs_ring + s * F, C, HW, mean, stdv,",
+     "orc_norm_chw_bf16(obs_ring + (s ? s - 1 : 0) * F, C, HW, mean, stdv,"),
+    ("normalize-mean-n-minus-1", C, "double mean = s / (double)n;",
+     "double mean = s / (double)(n - 1);"),
+    ("tier-hbm-window-always-full", C, "uint64_t in_hbm = total < cap_h ? total : cap_h;",
+     "uint64_t in_hbm = cap_h;"),
+    ("sched-iteration-max", "sched.py", "return a, b, a + b", "return a, b, max(a, b)"),
+    ("sched-overlap-always", "sched.py", "    if overlap:\n", "    if True:\n"),
+    ("sched-rollout-not-counted", "sched.py", "t = t_neighbour + per_unit(t_of_g, g)",
+     "t = per_unit(t_of_g, g)"),
+    ("place-first-candidate-skipped", "place.py", "for i, o in enumerate(opts):",
+     "for i, o in list(enumerate(opts))[1:]:"),
     # group-relative advantages and packing (Python)
     ("grpo-population-std", "llm.py", "/ (n - 1) if n > 1 else 0.0", "/ n if n > 1 else 0.0"),
     ("grpo-eps-inside-sqrt", "llm.py", "den = math.sqrt(var) + float(np.float32(eps))",
