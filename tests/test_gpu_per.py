@@ -163,6 +163,14 @@ def test_priorities_from_td_within_one(edp_lib, orc):
     diff = np.abs(u32(q).astype(np.int64) - ref)
     assert diff.max() <= 1
     assert (diff > 0).mean() < 1e-3
+    # the ends of the clamp are exact: a zero error without eps, and errors
+    # whose priority exceeds 32 bits
+    ends = np.array([0.0, 1e9, -1e9, 0.0], np.float32)
+    qe = torch.zeros(4, dtype=torch.int32, device="cuda")
+    edp.edp_priorities_from_td(m.ring.ctx, cuda(ends), 4, ALPHA, 0.0, qe)
+    edp.edp_sync(m.ring.ctx)
+    assert u32(qe).tolist() == orc.priorities_from_td(ends, ALPHA, 0.0).tolist()
+    assert u32(qe).tolist() == [1, 2**32 - 1, 2**32 - 1, 1]
 
 
 def test_all_zero_priorities_report_empty(edp_lib, orc):
