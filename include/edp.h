@@ -232,7 +232,8 @@ typedef struct {
 EDP_API edp_status edp_create(const edp_config *cfg, const edp_storage *st,
                       edp_ctx **out);
 
-/* Free libedp-owned memory.  Waits for the device to finish with it. */
+/* Free libedp-owned memory.  Waits for the device to finish with it.
+ * EDP_ERR_INVALID for a NULL context. */
 EDP_API edp_status edp_destroy(edp_ctx *ctx);
 
 /* Ingestion (Sec. 2.2 "experience ingestion", off-policy insertion with
@@ -242,7 +243,13 @@ EDP_API edp_status edp_destroy(edp_ctx *ctx);
  * (evicting the oldest host entries), then writes the new payload to HBM.
  * PER: q (device [n] or NULL) gives each new transition's priority (NULL =
  * the running maximum, initially 2^20 = 1.0).  With next_obs, the newest
- * transition's priority is deferred until its successor arrives. */
+ * transition's priority is deferred until its successor arrives.
+ * Errors: EDP_ERR_INVALID when n > capacity, src or src->obs is NULL, a
+ * field is neither device nor page-locked memory, obs or tokens are not
+ * 16-byte aligned, tokens are given to a context without tokens (or
+ * missing for one with them), or q is not device memory; EDP_ERR_STATE for
+ * q on a context without priorities; EDP_ERR_CUDA when a launch fails.
+ * n == 0 does nothing. */
 EDP_API edp_status edp_ingest(edp_ctx *ctx, const edp_fields *src, uint64_t n,
                       const uint32_t *q, edp_stream stream);
 
@@ -260,7 +267,14 @@ EDP_API edp_status edp_sample(edp_ctx *ctx, edp_sample_mode mode, uint32_t batch
  * learner's batch layout): fused gather + transform + collate (+ IS
  * weights) of the `batch` slots in idx (device int64).  A slot outside the
  * sampleable range is reported by edp_sync and its outputs are zeroed.
- * The batch's outputs may be device or page-locked host memory (edp_batch). */
+ * The batch's outputs may be device or page-locked host memory (edp_batch).
+ * Errors: EDP_ERR_INVALID for a NULL idx, out or out->obs, batch == 0,
+ * inputs (idx, q, gather sources) outside device memory, outputs neither
+ * device nor page-locked memory, obs / next_obs / tokens not 16-byte
+ * aligned, isw without q or with beta < 0, or a half-NULL gather pair;
+ * EDP_ERR_EMPTY for an empty ring; EDP_ERR_STATE for an output the context
+ * does not store (next_obs without next_obs = 1, tokens, action, reward,
+ * done). */
 EDP_API edp_status edp_deliver(edp_ctx *ctx, const int64_t *idx, uint32_t batch,
                        const edp_batch *out, edp_stream stream);
 
@@ -278,7 +292,11 @@ EDP_API edp_status edp_sample_deliver(edp_ctx *ctx, uint32_t batch, uint64_t see
 /* Priority callback (Appendix C, Invariant 2; PER).  Sets the priority of
  * each (idx[p], q[p]); for a repeated slot the last pair wins.  Pairs whose
  * slot holds no transition are skipped; the newest transition's priority is
- * deferred (next_obs).  Ancestor sums change by exact integer deltas. */
+ * deferred (next_obs).  Ancestor sums change by exact integer deltas.
+ * Errors: EDP_ERR_STATE for a context without priorities; EDP_ERR_INVALID
+ * for NULL inputs or inputs outside device memory (and, for the TD forms,
+ * alpha or eps < 0); EDP_ERR_OOM when the TD form cannot allocate its
+ * scratch.  n == 0 does nothing. */
 EDP_API edp_status edp_update_priorities(edp_ctx *ctx, const int64_t *idx,
                                  const uint32_t *q, uint32_t n,
                                  edp_stream stream);
@@ -344,7 +362,9 @@ EDP_API edp_status edp_gae(edp_ctx *ctx, const float *r, const float *v,
  * std_g the sample standard deviation (divisor n_g - 1; 0 for n_g = 1).
  * Computed in fp64, stored fp32; A_i = 0 where std_g + eps = 0.  r, adv:
  * device float[group_off[n_groups]]; group_off: device uint64[n_groups + 1],
- * non-decreasing, group_off[0] = 0.  A group of equal rewards gets A = 0. */
+ * non-decreasing, group_off[0] = 0.  A group of equal rewards gets A = 0.
+ * Errors: EDP_ERR_INVALID for a NULL array, n_groups == 0, eps negative or
+ * not finite, or arrays outside device memory. */
 EDP_API edp_status edp_grpo_advantage(edp_ctx *ctx, const float *r,
                                       const uint64_t *group_off, uint32_t n_groups,
                                       float eps, float *adv, edp_stream stream);
@@ -362,7 +382,11 @@ EDP_API edp_status edp_grpo_advantage(edp_ctx *ctx, const float *r,
  * written; both set a device flag that edp_sync reports (EDP_ERR_INVALID;
  * for an overflow the message gives the size needed).  batch <= 2^20.
  * The outputs (out_tokens, out_off, out_value) may be page-locked host
- * memory, written over the host link; the inputs are device memory. */
+ * memory, written over the host link; the inputs are device memory.
+ * Errors: EDP_ERR_INVALID for a NULL array, n_seq == 0, batch == 0 or
+ * > 2^20, seq_value without out_value (or the reverse), inputs outside
+ * device memory, or outputs neither device nor page-locked memory;
+ * EDP_ERR_OOM when the batch's scratch cannot be allocated. */
 EDP_API edp_status edp_pack_deliver(edp_ctx *ctx, const int32_t *tokens,
                                     const uint64_t *seq_off, uint64_t n_seq,
                                     const int64_t *idx, uint32_t batch,
@@ -392,7 +416,7 @@ EDP_API edp_status edp_grpo_pack_deliver(edp_ctx *ctx, const float *r,
 EDP_API edp_status edp_sync(edp_ctx *ctx, edp_stream stream);
 
 /* Describe the context's last failure ("" if none).  Valid until the next
- * call on the context. */
+ * call on the context.  "null context" for NULL. */
 EDP_API const char *edp_last_error(const edp_ctx *ctx);
 
 /* Online placement migration (Sec. 5.3, Alg. 2): move the experience state
@@ -431,13 +455,17 @@ EDP_API edp_status edp_migrate(const edp_ctx *src, edp_ctx *dst, edp_stream stre
 EDP_API edp_status edp_save(edp_ctx *ctx, const char *path, edp_stream stream);
 EDP_API edp_status edp_load(edp_ctx *ctx, const char *path, edp_stream stream);
 
-/* Fill *out with the context's cursors and tree layout. */
+/* Fill *out with the context's cursors and tree layout.  EDP_ERR_INVALID
+ * for a NULL argument. */
 EDP_API edp_status edp_get_info(const edp_ctx *ctx, edp_info *out);
 
 /* Host-link probe: streams `bytes` (a multiple of 16) of page-locked host
  * memory through the GPU with 16-byte loads, xor-folding them into
  * *d_fold (device uint64).  Used to measure achievable host-link read
- * bandwidth for the two-tier ring. */
+ * bandwidth for the two-tier ring.  Takes no context.  EDP_ERR_INVALID for
+ * NULL pointers, bytes not a multiple of 16, or a source that is not
+ * 16-byte aligned page-locked host or device memory; EDP_ERR_CUDA when the
+ * launch fails. */
 EDP_API edp_status edp_probe_host_read(const void *host_src, uint64_t bytes,
                                uint64_t *d_fold, edp_stream stream);
 
