@@ -13,20 +13,26 @@ def test_ring_against_list_model(orc):
     rng = np.random.default_rng(11)
     for cap in range(1, 18):
         ring = np.zeros((cap, 3), np.uint8)
-        model = []  # logical history of records
+        act = np.zeros(cap, np.int32)  # a multi-byte field beside it
+        model, amodel = [], []  # logical history of records
         total = 0
         for _ in range(12):
             n = int(rng.integers(0, cap + 1))
             src = rng.integers(0, 256, size=(n, 3), dtype=np.uint8)
+            a = rng.integers(-2**31, 2**31, size=n, dtype=np.int32)
             orc.ring_write(ring, cap, total, src)
+            orc.ring_write(act, cap, total, a)
             model.extend(src.tolist())
+            amodel.extend(a.tolist())
             total += n
             size = orc.ring_size(cap, total)
             assert size == min(total, cap)
             kept = model[len(model) - size:]
+            akept = amodel[len(amodel) - size:]
             for k in range(size):
                 s = orc.ring_slot(cap, total, k)
                 assert ring[s].tolist() == kept[k]
+                assert int(act[s]) == akept[k]
                 assert orc.ring_offset(cap, total, s) == k
                 # logical id total-size+k lives in slot id mod cap
                 assert s == (total - size + k) % cap

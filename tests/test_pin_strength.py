@@ -171,6 +171,27 @@ MUTANTS = [
      "t = per_unit(t_of_g, g)"),
     ("place-first-candidate-skipped", "place.py", "for i, o in enumerate(opts):",
      "for i, o in list(enumerate(opts))[1:]:"),
+    # the Python marshalling in front of the C oracle
+    ("wrap-uniform-seed-round-swapped", "oracle.py",
+     "lib().orc_sample_uniform(cap, total, n_valid, B, seed, round_,",
+     "lib().orc_sample_uniform(cap, total, n_valid, B, round_, seed,"),
+    ("wrap-ppo-adv-ret-swapped", "oracle.py",
+     "_p(idx, C.c_int64), B, _p(adv, C.c_float),\n                          _p(ret, C.c_float),",
+     "_p(idx, C.c_int64), B, _p(ret, C.c_float),\n                          _p(adv, C.c_float),"),
+    ("wrap-gae-gamma-lambda-swapped", "oracle.py", "                  gamma, lam, _p(adv, C.c_double)",
+     "                  lam, gamma, _p(adv, C.c_double)"),
+    ("wrap-normalize-std-as-mean", "oracle.py", "return out, float(m[0]), float(s[0])",
+     "return out, float(s[0]), float(m[0])"),
+    ("wrap-ingest-defer-dropped", "oracle.py",
+     "lib().orc_ingest_leaves(_p(st.leaves, C.c_uint32), st.cap, total, st.defer,\n"
+     "                            _p(qq, C.c_uint32)",
+     "lib().orc_ingest_leaves(_p(st.leaves, C.c_uint32), st.cap, total, 0,\n"
+     "                            _p(qq, C.c_uint32)"),
+    ("wrap-dqn-reward-as-action", "oracle.py", "_p(action, C.c_int32), _p(reward, C.c_float), cap,",
+     "_p(action, C.c_int32), _p(action, C.c_float), cap,"),
+    ("wrap-ring-write-rec", "oracle.py", "rec = ring.nbytes // cap", "rec = ring.nbytes // cap // ring.itemsize"),
+    ("wrap-isw-beta-fixed", "oracle.py", "lib().orc_is_weights(_p(q, C.c_uint32), len(q), beta,",
+     "lib().orc_is_weights(_p(q, C.c_uint32), len(q), 0.4,"),
     # group-relative advantages and packing (Python)
     ("grpo-population-std", "llm.py", "/ (n - 1) if n > 1 else 0.0", "/ n if n > 1 else 0.0"),
     ("grpo-eps-inside-sqrt", "llm.py", "den = math.sqrt(var) + float(np.float32(eps))",
