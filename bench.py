@@ -1444,10 +1444,14 @@ class LlmBatch(Workload):
     P, G = 512, 16
 
     def __init__(self, seed=1238, perms=8):
+        import numpy as np
         self.seed, self.n_perm = seed, perms
         from paper_2609_24456_gb300 import fixtures as fx
         self.h_tok, self.h_off, self.h_r, self.h_goff = fx.llm_rollout(seed, self.P, self.G)
         self.n = len(self.h_r)
+        # the delivery orders, on the host (the CPU legs use them too)
+        rng = np.random.default_rng(self.seed)
+        self.h_perms = [rng.permutation(self.n).astype(np.int64) for _ in range(self.n_perm)]
         self.T = int(self.h_off[-1])
         n, T = self.n, self.T
         grpo = 4 * n + 8 * (self.P + 1) + 4 * n
@@ -1475,8 +1479,6 @@ class LlmBatch(Workload):
         self.r = dev(self.h_r, device)
         self.goff = dev(self.h_goff.view(np.int64), device)
         self.adv = torch.empty(self.n, device=device)
-        rng = np.random.default_rng(self.seed)
-        self.h_perms = [rng.permutation(self.n).astype(np.int64) for _ in range(self.n_perm)]
         self.perms = [dev(p, device) for p in self.h_perms]
         self.outs = [(torch.empty(self.T, dtype=torch.int32, device=device),
                       torch.empty(self.T, device=device),

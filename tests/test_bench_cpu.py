@@ -25,10 +25,17 @@ def test_workload_has_every_leg(name):
         assert hasattr(wl, attr), (name, attr)
 
 
+class _SmallGrpo(bench.LlmBatch):
+    P, G = 8, 4
+
+
 @pytest.mark.parametrize("make,kw", [
     (lambda: bench.PerReplay(capacity=4096, batch=16), {"host_frames": 512}),
     (lambda: bench.MmReplay(capacity=64, batch=8), {"host_rows": 16}),
     (lambda: bench.MmReplay(capacity=64, batch=8, hbm_frac=0.5, ingest=4), {"host_rows": 16}),
+    (lambda: bench.DqnTiny(capacity=256, batch=8), {}),
+    (lambda: bench.PpoIteration(), {}),
+    (lambda: _SmallGrpo(), {}),
 ])
 def test_cpu_rounds_run(make, kw):
     wl = make()
