@@ -60,3 +60,47 @@ def test_create_rejects_bad_configs(edp_lib):
                            hbm_capacity=5)
     with pytest.raises(edp.EdpError):  # two tiers only for CHW_NORM_BF16
         edp.Ring(cfg3)
+
+
+def test_failing_allocator(edp_lib, orc):
+    """Fault injection on the host through the allocator callback.  A
+    creation whose allocation fails returns EDP_ERR_OOM and holds nothing.
+    A call whose scratch allocation fails returns EDP_ERR_OOM and leaves the
+    context usable: the same call succeeds once memory is granted."""
+    edp = edp_lib
+    grant = {"n": 0}
+    live = {}
+
+    def _alloc(user, nbytes):
+        if grant["n"] <= 0:
+            return None
+        grant["n"] -= 1
+        t = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
+        live[t.data_ptr()] = t
+        return t.data_ptr()
+
+    def _free(user, p):
+        live.pop(p, None)
+
+    alloc, free = edp.ALLOC_FN(_alloc), edp.FREE_FN(_free)  # kept alive here
+    cfg = edp.make_config(64, (3, 16, 16), edp.EDP_XFORM_HWC_CHW_BF16)
+    cfg.alloc, cfg.free = alloc, free
+    with pytest.raises(edp.EdpError) as e:
+        edp.Ring(cfg, action=False, reward=False, done=False)
+    assert e.value.status == edp.EDP_ERR_OOM
+    assert not live
+    grant["n"] = 1  # the control block, and nothing more
+    ring = edp.Ring(cfg, action=False, reward=False, done=False)
+    assert len(live) == 1
+    obs = torch.randint(0, 256, (64, 768), dtype=torch.uint8, device="cuda")
+    edp.edp_ingest(ring.ctx, obs, 64)
+    idx = torch.full((64,), -1, dtype=torch.int64, device="cuda")
+    with pytest.raises(edp.EdpError) as e:  # the shuffle's scratch
+        edp.edp_sample(ring.ctx, edp.EDP_SAMPLE_PERMUTE, 64, 5, 0, idx)
+    assert e.value.status == edp.EDP_ERR_OOM
+    grant["n"] = 4
+    edp.edp_sample(ring.ctx, edp.EDP_SAMPLE_PERMUTE, 64, 5, 0, idx)
+    edp.edp_sync(ring.ctx)
+    assert np.array_equal(to_np(idx), orc.permutation(64, 5, 0))
+    ring.close()
+    assert not live  # everything libedp took went back through free
