@@ -30,7 +30,12 @@
  *   (4 bytes per pair), the PERMUTE sampling mode, edp_gae with
  *   normalisation and edp_pack_deliver (16 bytes per batch entry).  Before
  *   capturing calls into a CUDA graph, make each of them once at its
- *   largest size, outside the capture.
+ *   largest size, outside the capture: a call that would have to grow its
+ *   scratch while its stream is being captured returns EDP_ERR_STATE and
+ *   enqueues nothing.
+ * - Current device: a call makes its context's device current while it
+ *   runs and gives the calling thread its previous current device back
+ *   before it returns.
  * - Asynchrony: every call validates its arguments on the host, enqueues its
  *   kernels on `stream` and returns without synchronising.  Results are
  *   valid once the stream has reached that point.  Host-side cursors
@@ -43,13 +48,12 @@
  *   edp_sample, edp_update_priorities*, edp_priorities_from_td, edp_gae and
  *   other deliveries of the same context, once the sampling that wrote its
  *   `idx` has completed (an event) and while nothing overwrites `idx`, `q`
- *   or the rows it reads (edp_ingest).  A large frame-stack delivery takes
- *   one of 32 work counters of its context, round robin in issue order (for
- *   a captured graph, the order at capture): deliveries that run at the
- *   same time must have been issued fewer than 32 deliveries apart.
+ *   or the rows it reads (edp_ingest).  Any number of deliveries may be in
+ *   flight at once, on any streams or in one graph.
  *   edp_gae likewise may overlap edp_sample (GAE scratch and shuffle
- *   scratch are separate); edp_gae and edp_pack_deliver share scratch.  Every other pair of calls on one context shares
- *   the priority tree or the context's scratch and must be ordered.
+ *   scratch are separate); edp_gae and edp_pack_deliver share scratch.
+ *   Every other pair of calls on one context shares the priority tree or
+ *   the context's scratch and must be ordered.
  * - Errors: argument and state errors are returned synchronously and leave
  *   the context unchanged.  A CUDA launch error returns EDP_ERR_CUDA.
  *   Data-dependent faults found on the device (an index out of range, an
@@ -319,8 +323,12 @@ EDP_API edp_status edp_update_priorities_td(edp_ctx *ctx, const int64_t *idx,
  * 16384 pairs (64 KiB), held by every GPU that loads libedp until the process
  * exits.  n > 16384 returns EDP_ERR_INVALID.  The first call on a device
  * looks up the array's device address (make it before any stream capture).
- * All calls on a device share the array, so calls that overlap on the GPU --
- * on any stream or context -- race; the array keeps the last call's
+ * All calls on a device share the array.  Calls queued on one stream are
+ * ordered (a call touches the array only after the previous kernel on its
+ * stream has finished), so they may follow each other with no
+ * synchronisation; calls that can run at the same time on different streams
+ * -- of one context or of several on the device -- race on the array and
+ * must be ordered by the caller (an event).  The array keeps the last call's
  * contents, which a call never reads before writing.  Results equal those of
  * edp_update_priorities_td for the same arguments. */
 EDP_API edp_status edp_update_priorities_td_static(edp_ctx *ctx, const int64_t *idx,

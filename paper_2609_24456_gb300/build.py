@@ -83,6 +83,25 @@ def build(force: bool = False, verbose: bool = False, ptxas_v: bool = False) -> 
     return LIB
 
 
+PROBE_SRC = os.path.join(ROOT, "tests", "curand_philox_probe.cu")
+PROBE_LIB = os.path.join(ROOT, "tests", "_build", "curand_philox_probe.so")
+
+
+def build_curand_probe(force: bool = False) -> str:
+    """Compile the tests' cuRAND Philox probe (test infrastructure, not part
+    of libedp) with the same nvcc and target."""
+    if not force and not _stale(PROBE_LIB, [PROBE_SRC, os.path.abspath(__file__)]):
+        return PROBE_LIB
+    os.makedirs(os.path.dirname(PROBE_LIB), exist_ok=True)
+    tmp = PROBE_LIB + ".tmp.%d" % os.getpid()
+    cmd = [nvcc()] + ARCH + ["-O2", "-shared", "-Xcompiler", "-fPIC", PROBE_SRC, "-o", tmp]
+    p = subprocess.run(cmd, capture_output=True, text=True)
+    if p.returncode != 0:
+        raise RuntimeError("nvcc failed for %s:\n%s%s" % (PROBE_SRC, p.stdout, p.stderr))
+    os.replace(tmp, PROBE_LIB)
+    return PROBE_LIB
+
+
 if __name__ == "__main__":
     print(build(force="--force" in sys.argv, verbose=True,
                 ptxas_v="--ptxas-v" in sys.argv))

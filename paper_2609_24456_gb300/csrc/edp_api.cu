@@ -26,42 +26,8 @@ void *default_alloc(void *, size_t bytes) {
 
 void default_free(void *, void *p) { cudaFree(p); }
 
-edp_status fail(edp_ctx *c, edp_status s, const char *fmt, ...) {
-  if (c) {
-    char buf[512];
-    va_list ap;
-    va_start(ap, fmt);
-    vsnprintf(buf, sizeof buf, fmt, ap);
-    va_end(ap);
-    c->err = buf;
-  }
-  return s;
-}
-
 edp_status cuda_fail(edp_ctx *c, cudaError_t e, const char *where) {
   return fail(c, EDP_ERR_CUDA, "%s: %s", where, cudaGetErrorString(e));
-}
-
-// Resolve a caller pointer to a device-usable address.  Device memory of the
-// context's GPU passes through; page-locked host memory is translated to its
-// mapped device address; pageable or foreign memory is rejected.
-bool device_view(const edp_ctx *c, const void *p, const void **out,
-                 bool allow_host) {
-  cudaPointerAttributes a;
-  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
-    cudaGetLastError();
-    return false;
-  }
-  if (a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged) {
-    if (a.device != c->cfg.device) return false;
-    *out = p;
-    return true;
-  }
-  if (a.type == cudaMemoryTypeHost && allow_host && a.devicePointer) {
-    *out = a.devicePointer;
-    return true;
-  }
-  return false;
 }
 
 edp_status create_fail(edp_ctx *c, const char *fmt, ...) {
@@ -188,63 +154,121 @@ bool norm_affine_constants(edp_ctx *c) {
 
 }  // namespace
 
-void *edp::ctx_scratch(edp_ctx *ctx, size_t bytes) {
-  if (bytes <= ctx->scratch_bytes) return ctx->scratch;
-  edp_alloc_fn al = ctx->cfg.alloc ? ctx->cfg.alloc : default_alloc;
-  edp_free_fn fr = ctx->cfg.free ? ctx->cfg.free : default_free;
-  if (ctx->scratch) {
-    cudaDeviceSynchronize();  // the old block may still be in use
-    fr(ctx->cfg.alloc_user, ctx->scratch);
-    ctx->scratch = nullptr;
-    ctx->scratch_bytes = 0;
+edp_status edp::fail(edp_ctx *c, edp_status s, const char *fmt, ...) {
+  if (c) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    c->err = buf;
   }
-  bytes = (bytes + 255) & ~(size_t)255;
-  void *p = al(ctx->cfg.alloc_user, bytes);
-  if (!p) return nullptr;
-  ctx->scratch = p;
-  ctx->scratch_bytes = bytes;
-  return p;
+  return s;
 }
 
-void *edp::ctx_perm_scratch(edp_ctx *ctx, size_t bytes) {
-  if (bytes <= ctx->perm_bytes) return ctx->perm_scratch;
+bool edp::device_view(const edp_ctx *c, const void *p, const void **out,
+                      bool allow_host) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  if (a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged) {
+    if (a.device != c->cfg.device) return false;
+    *out = p;
+    return true;
+  }
+  if (a.type == cudaMemoryTypeHost && allow_host && a.devicePointer) {
+    *out = a.devicePointer;
+    return true;
+  }
+  return false;
+}
+
+edp_status edp::launch_fail(edp_ctx *c, cudaError_t e, const char *where) {
+  if (e == cudaErrorMemoryAllocation)
+    return fail(c, EDP_ERR_OOM, "%s: scratch allocation failed", where);
+  if (e == cudaErrorStreamCaptureUnsupported)
+    return fail(c, EDP_ERR_STATE,
+                "%s: not allowed while the stream is being captured (its scratch "
+                "would have to grow: make one call of this size before capture)",
+                where);
+  return fail(c, EDP_ERR_CUDA, "%s: %s", where, cudaGetErrorString(e));
+}
+
+edp_status edp::update_args(edp_ctx *ctx, const char *who, const int64_t *idx,
+                            const uint32_t *q, const float *td, uint32_t n,
+                            double alpha, double eps) {
+  if (!ctx) return EDP_ERR_INVALID;
+  if (!ctx->depth) return fail(ctx, EDP_ERR_STATE, "%s: context has no priorities", who);
+  if (n == 0) return EDP_OK;
+  if (!idx || (!q && !td)) return fail(ctx, EDP_ERR_INVALID, "%s: NULL input", who);
+  const void *p;
+  if (!device_view(ctx, idx, &p, false) || (q && !device_view(ctx, q, &p, false)) ||
+      (td && !device_view(ctx, td, &p, false)))
+    return fail(ctx, EDP_ERR_INVALID, "%s: inputs must be device memory", who);
+  if (td && !(alpha >= 0.0 && eps >= 0.0))
+    return fail(ctx, EDP_ERR_INVALID, "%s: alpha, eps >= 0", who);
+  return EDP_OK;
+}
+
+namespace {
+
+// Grow-only block (*blk, *have bytes) to at least `want` bytes; the first
+// `zero_head` bytes of a new block are zeroed.
+cudaError_t grow(edp_ctx *ctx, void **blk, size_t *have, size_t want, size_t zero_head,
+                 cudaStream_t s) {
+  if (want <= *have) return cudaSuccess;
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(s, &cs) != cudaSuccess) {
+    cudaGetLastError();  // e.g. the legacy stream while another captures
+    return cudaErrorStreamCaptureUnsupported;
+  }
+  if (cs != cudaStreamCaptureStatusNone) return cudaErrorStreamCaptureUnsupported;
   edp_alloc_fn al = ctx->cfg.alloc ? ctx->cfg.alloc : default_alloc;
   edp_free_fn fr = ctx->cfg.free ? ctx->cfg.free : default_free;
-  if (ctx->perm_scratch) {
-    cudaDeviceSynchronize();
-    fr(ctx->cfg.alloc_user, ctx->perm_scratch);
-    ctx->perm_scratch = nullptr;
-    ctx->perm_bytes = 0;
+  if (*blk) {
+    cudaDeviceSynchronize();  // the old block may still be in use
+    fr(ctx->cfg.alloc_user, *blk);
+    *blk = nullptr;
+    *have = 0;
   }
-  bytes = (bytes + 255) & ~(size_t)255;
-  void *p = al(ctx->cfg.alloc_user, bytes);
-  if (!p) return nullptr;
-  if (cudaMemset(p, 0, perm_zeroed_bytes()) != cudaSuccess) {
+  want = (want + 255) & ~(size_t)255;
+  void *p = al(ctx->cfg.alloc_user, want);
+  if (!p) return cudaErrorMemoryAllocation;
+  if (zero_head && cudaMemset(p, 0, zero_head) != cudaSuccess) {
     cudaGetLastError();
     fr(ctx->cfg.alloc_user, p);
-    return nullptr;
+    return cudaErrorMemoryAllocation;
   }
-  ctx->perm_scratch = p;
-  ctx->perm_bytes = bytes;
-  return p;
+  *blk = p;
+  *have = want;
+  return cudaSuccess;
 }
 
-uint32_t *edp::ctx_qbuf(edp_ctx *ctx, size_t n) {
-  if (n <= ctx->qbuf_n) return ctx->qbuf;
-  edp_alloc_fn al = ctx->cfg.alloc ? ctx->cfg.alloc : default_alloc;
-  edp_free_fn fr = ctx->cfg.free ? ctx->cfg.free : default_free;
-  if (ctx->qbuf) {
-    cudaDeviceSynchronize();
-    fr(ctx->cfg.alloc_user, ctx->qbuf);
-    ctx->qbuf = nullptr;
-    ctx->qbuf_n = 0;
-  }
-  n = n < 4096 ? 4096 : n;
-  void *p = al(ctx->cfg.alloc_user, n * 4);
-  if (!p) return nullptr;
-  ctx->qbuf = (uint32_t *)p;
-  ctx->qbuf_n = n;
-  return ctx->qbuf;
+}  // namespace
+
+cudaError_t edp::ctx_scratch(edp_ctx *ctx, size_t bytes, cudaStream_t s, void **out) {
+  const cudaError_t e = grow(ctx, &ctx->scratch, &ctx->scratch_bytes, bytes, 0, s);
+  *out = ctx->scratch;
+  return e;
+}
+
+cudaError_t edp::ctx_perm_scratch(edp_ctx *ctx, size_t bytes, cudaStream_t s, void **out) {
+  const cudaError_t e =
+      grow(ctx, &ctx->perm_scratch, &ctx->perm_bytes, bytes, perm_zeroed_bytes(), s);
+  *out = ctx->perm_scratch;
+  return e;
+}
+
+cudaError_t edp::ctx_qbuf(edp_ctx *ctx, size_t n, cudaStream_t s, uint32_t **out) {
+  void *blk = ctx->qbuf;
+  size_t have = ctx->qbuf_n * 4;
+  const cudaError_t e = grow(ctx, &blk, &have, (n < 4096 ? 4096 : n) * 4, 0, s);
+  ctx->qbuf = (uint32_t *)blk;
+  ctx->qbuf_n = have / 4;
+  *out = ctx->qbuf;
+  return e;
 }
 
 extern "C" {
@@ -303,10 +327,8 @@ edp_status edp_create(const edp_config *cfg, const edp_storage *st,
     cudaGetLastError();
     return bad("no CUDA device %d", cfg->device);
   }
-  if (cudaSetDevice(cfg->device) != cudaSuccess) {
-    cudaGetLastError();
-    return bad("cudaSetDevice failed");
-  }
+  DeviceGuard dg(cfg->device);
+  if (!dg.ok()) return bad("cudaSetDevice failed");
   c->cap = cfg->capacity;
   c->cap_h = cfg->hbm_capacity;
   c->cap_c = cfg->capacity - cfg->hbm_capacity;
@@ -411,7 +433,7 @@ edp_status edp_create(const edp_config *cfg, const edp_storage *st,
 
 edp_status edp_destroy(edp_ctx *ctx) {
   if (!ctx) return EDP_ERR_INVALID;
-  cudaSetDevice(ctx->cfg.device);
+  DeviceGuard dg(ctx->cfg.device);
   cudaDeviceSynchronize();
   free_all(ctx);
   delete ctx;
@@ -433,7 +455,7 @@ edp_status edp_migrate(const edp_ctx *src, edp_ctx *dst, edp_stream stream) {
       (src->st.reward != nullptr) != (dst->st.reward != nullptr) ||
       (src->st.done != nullptr) != (dst->st.done != nullptr))
     return fail(dst, EDP_ERR_STATE, "edp_migrate: metadata arrays differ");
-  cudaSetDevice(b.device);
+  DeviceGuard dg(b.device);
   cudaStream_t s = (cudaStream_t)stream;
   const uint64_t size = ring_size(src);
   const uint64_t n = size < dst->cap ? size : dst->cap;
@@ -528,7 +550,7 @@ extern "C" {
 edp_status edp_save(edp_ctx *ctx, const char *path, edp_stream stream) {
   if (!ctx) return EDP_ERR_INVALID;
   if (!path) return fail(ctx, EDP_ERR_INVALID, "edp_save: path is NULL");
-  cudaSetDevice(ctx->cfg.device);
+  DeviceGuard dg(ctx->cfg.device);
   cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_save");
   CkptHeader h{};
@@ -619,7 +641,7 @@ edp_status edp_load(edp_ctx *ctx, const char *path, edp_stream stream) {
                 "edp_load: %s holds %ld bytes, its header describes %llu (truncated file?)", path,
                 have, (unsigned long long)want);
   }
-  cudaSetDevice(ctx->cfg.device);
+  DeviceGuard dg(ctx->cfg.device);
   const uint64_t n = h.n < ctx->cap ? h.n : ctx->cap;  // the newest n are kept
   const uint64_t skip = h.n - n;
   uint8_t *stage = (uint8_t *)std::malloc(kStage);
@@ -711,7 +733,7 @@ edp_status edp_ingest(edp_ctx *ctx, const edp_fields *src, uint64_t n,
     return fail(ctx, EDP_ERR_INVALID, "edp_ingest: n=%llu exceeds capacity",
                 (unsigned long long)n);
   if (n == 0) return EDP_OK;
-  cudaSetDevice(ctx->cfg.device);
+  DeviceGuard dg(ctx->cfg.device);
   cudaStream_t s = (cudaStream_t)stream;
   edp_fields f{};
   const void *p;
@@ -812,7 +834,7 @@ edp_status edp_sample(edp_ctx *ctx, edp_sample_mode mode, uint32_t batch,
   const void *p;
   if (!device_view(ctx, idx, &p, false) || (q && !device_view(ctx, q, &p, false)))
     return fail(ctx, EDP_ERR_INVALID, "edp_sample: outputs must be device memory");
-  cudaSetDevice(ctx->cfg.device);
+  DeviceGuard dg(ctx->cfg.device);
   cudaStream_t s = (cudaStream_t)stream;
   cudaError_t e;
   switch (mode) {
@@ -840,9 +862,7 @@ edp_status edp_sample(edp_ctx *ctx, edp_sample_mode mode, uint32_t batch,
     default:
       return fail(ctx, EDP_ERR_INVALID, "edp_sample: unknown mode %d", (int)mode);
   }
-  if (e == cudaErrorMemoryAllocation)
-    return fail(ctx, EDP_ERR_OOM, "edp_sample: scratch allocation failed");
-  if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_sample");
+  if (e != cudaSuccess) return launch_fail(ctx, e, "edp_sample");
   return EDP_OK;
 }
 
@@ -905,7 +925,7 @@ edp_status edp_deliver(edp_ctx *ctx, const int64_t *idx, uint32_t batch,
   edp_batch res;
   const edp_status st = deliver_checks(ctx, idx, batch, out, &res);
   if (st != EDP_OK) return st;
-  cudaSetDevice(ctx->cfg.device);
+  DeviceGuard dg(ctx->cfg.device);
   cudaError_t e = launch_deliver(ctx, idx, batch, &res, (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_deliver");
   return EDP_OK;
@@ -922,32 +942,21 @@ edp_status edp_sample_deliver(edp_ctx *ctx, uint32_t batch, uint64_t seed, uint6
   edp_batch res;
   const edp_status st = deliver_checks(ctx, idx, batch, out, &res);
   if (st != EDP_OK) return st;
-  cudaSetDevice(ctx->cfg.device);
+  DeviceGuard dg(ctx->cfg.device);
   DrawUniform d{seed, round, idx};
   cudaError_t e = launch_deliver(ctx, idx, batch, &res, (cudaStream_t)stream, &d);
   if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_sample_deliver");
   return EDP_OK;
 }
 
-static edp_status update_common(edp_ctx *ctx, const int64_t *idx,
+static edp_status update_common(edp_ctx *ctx, const char *who, const int64_t *idx,
                                 const uint32_t *q, const float *td, uint32_t n,
                                 double alpha, double eps, edp_stream stream) {
-  if (!ctx) return EDP_ERR_INVALID;
-  if (!ctx->depth)
-    return fail(ctx, EDP_ERR_STATE, "edp_update_priorities: context has no priorities");
-  if (n == 0) return EDP_OK;
-  if (!idx || (!q && !td))
-    return fail(ctx, EDP_ERR_INVALID, "edp_update_priorities: NULL input");
-  const void *p;
-  if (!device_view(ctx, idx, &p, false) ||
-      (q && !device_view(ctx, q, &p, false)) ||
-      (td && !device_view(ctx, td, &p, false)))
-    return fail(ctx, EDP_ERR_INVALID, "edp_update_priorities: inputs must be device memory");
-  cudaSetDevice(ctx->cfg.device);
+  const edp_status st = update_args(ctx, who, idx, q, td, n, alpha, eps);
+  if (st != EDP_OK || n == 0) return st;
+  DeviceGuard dg(ctx->cfg.device);
   cudaError_t e = launch_update(ctx, idx, q, td, alpha, eps, n, (cudaStream_t)stream);
-  if (e == cudaErrorMemoryAllocation)
-    return fail(ctx, EDP_ERR_OOM, "edp_update_priorities: scratch allocation failed");
-  if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_update_priorities");
+  if (e != cudaSuccess) return launch_fail(ctx, e, who);
   return EDP_OK;
 }
 
@@ -955,16 +964,15 @@ edp_status edp_update_priorities(edp_ctx *ctx, const int64_t *idx,
                                  const uint32_t *q, uint32_t n,
                                  edp_stream stream) {
   if (ctx && n && !q) return fail(ctx, EDP_ERR_INVALID, "edp_update_priorities: q NULL");
-  return update_common(ctx, idx, q, nullptr, n, 0.0, 0.0, stream);
+  return update_common(ctx, "edp_update_priorities", idx, q, nullptr, n, 0.0, 0.0, stream);
 }
 
 edp_status edp_update_priorities_td(edp_ctx *ctx, const int64_t *idx,
                                     const float *td, uint32_t n, double alpha,
                                     double eps, edp_stream stream) {
   if (ctx && n && !td) return fail(ctx, EDP_ERR_INVALID, "edp_update_priorities_td: td NULL");
-  if (ctx && !(alpha >= 0.0 && eps >= 0.0))
-    return fail(ctx, EDP_ERR_INVALID, "edp_update_priorities_td: alpha, eps >= 0");
-  return update_common(ctx, idx, nullptr, td, n, alpha, eps, stream);
+  return update_common(ctx, "edp_update_priorities_td", idx, nullptr, td, n, alpha, eps,
+                       stream);
 }
 
 edp_status edp_priorities_from_td(edp_ctx *ctx, const float *td, uint32_t n,
@@ -977,7 +985,7 @@ edp_status edp_priorities_from_td(edp_ctx *ctx, const float *td, uint32_t n,
     return fail(ctx, EDP_ERR_INVALID, "edp_priorities_from_td: device arrays required");
   if (!(alpha >= 0.0 && eps >= 0.0))
     return fail(ctx, EDP_ERR_INVALID, "edp_priorities_from_td: alpha, eps >= 0");
-  cudaSetDevice(ctx->cfg.device);
+  DeviceGuard dg(ctx->cfg.device);
   cudaError_t e = launch_prio_from_td(td, n, alpha, eps, q, (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_priorities_from_td");
   return EDP_OK;
@@ -998,12 +1006,10 @@ edp_status edp_gae(edp_ctx *ctx, const float *r, const float *v,
   for (const void *o : ptrs)
     if (o && !device_view(ctx, o, &p, false))
       return fail(ctx, EDP_ERR_INVALID, "edp_gae: arrays must be device memory");
-  cudaSetDevice(ctx->cfg.device);
+  DeviceGuard dg(ctx->cfg.device);
   cudaError_t e = launch_gae(ctx, r, v, d, T, E, gamma, lambda, adv, ret, adv_norm,
                              (cudaStream_t)stream);
-  if (e == cudaErrorMemoryAllocation)
-    return fail(ctx, EDP_ERR_OOM, "edp_gae: scratch allocation failed");
-  if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_gae");
+  if (e != cudaSuccess) return launch_fail(ctx, e, "edp_gae");
   return EDP_OK;
 }
 
@@ -1019,7 +1025,7 @@ edp_status edp_grpo_advantage(edp_ctx *ctx, const float *r, const uint64_t *grou
   for (const void *o : ptrs)
     if (!device_view(ctx, o, &p, false))
       return fail(ctx, EDP_ERR_INVALID, "edp_grpo_advantage: arrays must be device memory");
-  cudaSetDevice(ctx->cfg.device);
+  DeviceGuard dg(ctx->cfg.device);
   cudaError_t e = launch_grpo(ctx, r, group_off, n_groups, eps, adv, (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_grpo_advantage");
   return EDP_OK;
@@ -1050,13 +1056,11 @@ edp_status edp_pack_deliver(edp_ctx *ctx, const int32_t *tokens, const uint64_t 
                   "edp_pack_deliver: outputs must be device or page-locked host memory");
     o = const_cast<void *>(p);
   }
-  cudaSetDevice(ctx->cfg.device);
+  DeviceGuard dg(ctx->cfg.device);
   cudaError_t e = launch_pack(ctx, tokens, seq_off, n_seq, idx, batch, seq_value,
                               (int32_t *)outs[0], (uint64_t *)outs[1], (float *)outs[2],
                               out_cap, (cudaStream_t)stream);
-  if (e == cudaErrorMemoryAllocation)
-    return fail(ctx, EDP_ERR_OOM, "edp_pack_deliver: scratch allocation failed");
-  if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_pack_deliver");
+  if (e != cudaSuccess) return launch_fail(ctx, e, "edp_pack_deliver");
   return EDP_OK;
 }
 
@@ -1089,19 +1093,17 @@ edp_status edp_grpo_pack_deliver(edp_ctx *ctx, const float *r, const uint64_t *g
                   "edp_grpo_pack_deliver: outputs must be device or page-locked host memory");
     o = const_cast<void *>(p);
   }
-  cudaSetDevice(ctx->cfg.device);
+  DeviceGuard dg(ctx->cfg.device);
   cudaError_t e = launch_grpo_pack(ctx, r, group_off, n_groups, eps, adv, tokens, seq_off,
                                    n_seq, idx, batch, (int32_t *)outs[0], (uint64_t *)outs[1],
                                    (float *)outs[2], out_cap, (cudaStream_t)stream);
-  if (e == cudaErrorMemoryAllocation)
-    return fail(ctx, EDP_ERR_OOM, "edp_grpo_pack_deliver: scratch allocation failed");
-  if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_grpo_pack_deliver");
+  if (e != cudaSuccess) return launch_fail(ctx, e, "edp_grpo_pack_deliver");
   return EDP_OK;
 }
 
 edp_status edp_sync(edp_ctx *ctx, edp_stream stream) {
   if (!ctx) return EDP_ERR_INVALID;
-  cudaSetDevice(ctx->cfg.device);
+  DeviceGuard dg(ctx->cfg.device);
   cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
   if (e == cudaSuccess) e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_sync");

@@ -23,9 +23,9 @@ enum : uint32_t {
 };
 
 // Small device-resident control block (one per context).
-// Work counters of the dynamically scheduled delivery kernels: launch n of
-// a context uses pair n mod kWorkSlots (chunks handed out, CTAs retired);
-// the last CTA of the launch resets its pair to zero.
+// Work words of the dynamically scheduled frame-stack delivery: launch n of
+// a context starts at word n mod kWorkSlots (see k_deliver.cu for the claim
+// protocol, which stays correct whatever the number of launches in flight).
 constexpr int kWorkSlots = 32;
 
 struct Ctrl {
@@ -34,9 +34,10 @@ struct Ctrl {
   uint32_t max_q;      // running maximum priority
   uint32_t pad0[2];
   uint32_t upd_count;  // priority update: CTAs done with phase 1
-  uint32_t pad[2];
+  uint32_t pack_ticket;  // packed delivery: length CTAs done (calls are ordered)
+  uint32_t pad;
   unsigned long long bad_index;  // first offending index (diagnostics)
-  uint32_t work[2 * kWorkSlots];
+  unsigned long long work[kWorkSlots];
 };
 
 constexpr int kFanout = 32;
@@ -76,7 +77,7 @@ struct edp_ctx {
   float naff_a[4] = {}, naff_b[4] = {};
   int norm_affine = 0;
   int coop_sms = 0;
-  uint32_t work_seq = 0;  // delivery launches so far (work counter pairs)
+  uint64_t work_seq = 0;  // frame-stack delivery launches so far (work words)
   std::string err;
 };
 
@@ -364,14 +365,73 @@ cudaError_t launch_gae(edp_ctx *ctx, const float *r, const float *v,
 cudaError_t launch_probe_read(const void *src, uint64_t bytes, uint64_t *fold,
                               cudaStream_t s);
 
-// scratch owned by the context, grown on demand (not stream-ordered: the
-// caller makes the first call of a given size outside graph capture)
-void *ctx_scratch(edp_ctx *ctx, size_t bytes);
+// Scratch owned by the context, grown on demand.  Growing allocates, and
+// first waits for the device (the old block may still be in use); neither
+// is allowed while `s` is being captured into a CUDA graph, so a call that
+// would grow there returns cudaErrorStreamCaptureUnsupported and changes
+// nothing (the caller makes one call of its largest size before capture).
+// cudaErrorMemoryAllocation when the allocator fails.
+cudaError_t ctx_scratch(edp_ctx *ctx, size_t bytes, cudaStream_t s, void **out);
 // shuffle scratch: its first perm_zeroed_bytes() start zeroed and are left
 // zeroed by every shuffle
-void *ctx_perm_scratch(edp_ctx *ctx, size_t bytes);
+cudaError_t ctx_perm_scratch(edp_ctx *ctx, size_t bytes, cudaStream_t s, void **out);
 size_t perm_scratch_bytes(uint32_t n);
 size_t perm_zeroed_bytes();
-uint32_t *ctx_qbuf(edp_ctx *ctx, size_t n);
+cudaError_t ctx_qbuf(edp_ctx *ctx, size_t n, cudaStream_t s, uint32_t **out);
+
+// ---------------------------------------------------------------------------
+// Host helpers shared by the entry points
+// ---------------------------------------------------------------------------
+
+// Makes `dev` the calling thread's current device for the guard's lifetime
+// and gives the thread its previous current device back afterwards, so an
+// entry point never changes the device its caller selected.
+class DeviceGuard {
+ public:
+  explicit DeviceGuard(int dev) {
+    if (cudaGetDevice(&prev_) != cudaSuccess) {
+      cudaGetLastError();
+      prev_ = -1;
+    }
+    if (prev_ != dev && cudaSetDevice(dev) != cudaSuccess) {
+      cudaGetLastError();
+      ok_ = false;
+    }
+    switched_ = ok_ && prev_ >= 0 && prev_ != dev;
+  }
+  ~DeviceGuard() {
+    if (switched_) cudaSetDevice(prev_);
+  }
+  bool ok() const { return ok_; }
+  DeviceGuard(const DeviceGuard &) = delete;
+  DeviceGuard &operator=(const DeviceGuard &) = delete;
+
+ private:
+  int prev_ = -1;
+  bool ok_ = true;
+  bool switched_ = false;
+};
+
+// Resolve a caller pointer to a device-usable address.  Device memory of the
+// context's GPU passes through; page-locked host memory is translated to its
+// mapped device address when allow_host; pageable or foreign memory is
+// rejected (false).
+bool device_view(const edp_ctx *c, const void *p, const void **out, bool allow_host);
+
+// Record a printf-style message as the context's last error; returns s.
+edp_status fail(edp_ctx *c, edp_status s, const char *fmt, ...);
+
+// The status and message for a failed launcher: EDP_ERR_OOM when scratch
+// could not be allocated, EDP_ERR_STATE when scratch would have to grow
+// during stream capture, EDP_ERR_CUDA otherwise.
+edp_status launch_fail(edp_ctx *c, cudaError_t e, const char *where);
+
+// Argument and state checks shared by the priority-update entry points
+// (`who` names the entry point in messages): a context with a tree; for
+// n > 0, idx and one of q / td given, all device memory of the context's
+// GPU; with td, alpha and eps >= 0.
+edp_status update_args(edp_ctx *ctx, const char *who, const int64_t *idx,
+                       const uint32_t *q, const float *td, uint32_t n, double alpha,
+                       double eps);
 
 }  // namespace edp

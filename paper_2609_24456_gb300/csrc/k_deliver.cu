@@ -58,7 +58,8 @@ struct Common {
   const float *gsrc0, *gsrc1;
   float *gdst0, *gdst1;
   Ctrl *ctrl;
-  uint32_t *work;  // this launch's work counter pair, or null (one chunk per CTA)
+  unsigned long long *work;  // this launch's work word, or null (one chunk per CTA)
+  unsigned long long work_tag;
   float r1, r2;
   // fused uniform sampling: idx is then an output, sample k is drawn here
   int draw;
@@ -201,6 +202,70 @@ __device__ __forceinline__ float byte_f(uint32_t w, int i) {
 }
 
 // ---------------------------------------------------------------------------
+// Work claims of a persistent delivery grid.  The CTAs of a launch take
+// chunks in order from one 64-bit work word of the context, laid out as
+//   [63:28] owner tag   [27:0] chunks handed out;
+// tag 0 means free.  A launch's tag is 1 + its call number on the context
+// (host side: unique for every call, and for every node of a captured
+// graph).  A CTA claims from the word if its launch owns it, takes the word
+// over if it is free (claiming chunk 0), and otherwise -- another launch
+// still owns it -- takes a fixed share: chunks blockIdx.x, blockIdx.x +
+// gridDim.x, ...  A one-thread release kernel, queued after the delivery
+// on the same stream, frees the word once every CTA of the launch has
+// finished, so an owned word never changes hands while its owner runs, a
+// replayed graph finds its words free again, and no claim of one launch
+// can land on another's count.  Every chunk is processed: if any CTA of
+// the launch owns the word, the owning CTAs claim until the chunks run out;
+// if none does, the fixed shares cover them all; where both happen some
+// chunks are written twice, with the same bytes.  (Only the same captured
+// node running twice at once could meet its own tag on a live word; the
+// two share the claims and, having the same arguments, still write every
+// chunk of the one batch.)
+// ---------------------------------------------------------------------------
+constexpr int kWorkTagShift = 28;
+constexpr unsigned long long kWorkClaimMask = (1ull << kWorkTagShift) - 1;
+constexpr uint32_t kWorkMaxChunks = 1u << 27;  // chunks + grid stay below 2^28
+constexpr uint32_t kWorkFixed = 0xffffffffu;   // first claim: take the fixed share
+constexpr uint32_t kWorkDone = 0xfffffffeu;    // no chunk left for this launch
+
+// A chunk of the launch with tag `tag` (or kWorkDone).
+__device__ __forceinline__ uint32_t work_claim(unsigned long long *wd,
+                                               unsigned long long tag) {
+  const unsigned long long old = atomicAdd(wd, 1ull);
+  return (old >> kWorkTagShift) == tag ? (uint32_t)(old & kWorkClaimMask) : kWorkDone;
+}
+
+// A CTA's first claim: a chunk, or kWorkFixed when another launch owns the
+// word.
+__device__ __forceinline__ uint32_t work_first(unsigned long long *wd,
+                                               unsigned long long tag) {
+  unsigned long long w = *reinterpret_cast<volatile unsigned long long *>(wd);
+  for (int tries = 0; tries < 8; ++tries) {
+    const unsigned long long owner = w >> kWorkTagShift;
+    if (owner == tag) return work_claim(wd, tag);
+    if (owner != 0) return kWorkFixed;
+    const unsigned long long mine = (tag << kWorkTagShift) | 1ull;  // chunk 0 taken
+    const unsigned long long prev = atomicCAS(wd, w, mine);
+    if (prev == w) return 0;
+    w = prev;
+  }
+  return kWorkFixed;
+}
+
+// Frees the word of the launch with tag `tag`, after that launch (the
+// preceding kernel on the stream) has completed.
+__global__ void k_work_release(unsigned long long *wd, unsigned long long tag) {
+  pdl_wait();
+  pdl_launch();
+  unsigned long long w = *reinterpret_cast<volatile unsigned long long *>(wd);
+  for (int tries = 0; tries < 8 && (w >> kWorkTagShift) == tag; ++tries) {
+    const unsigned long long prev = atomicCAS(wd, w, 0ull);
+    if (prev == w) break;
+    w = prev;
+  }
+}
+
+// ---------------------------------------------------------------------------
 // Frame stack, float32 (DQN), on the load / store units.  A unit is one
 // 32-bit word of frame m in [0, U) of sample k -- the frame at logical
 // offset j = off - K + 1 + m, which is obs slot m (m < K) and next_obs slot
@@ -216,9 +281,9 @@ __device__ __forceinline__ float byte_f(uint32_t w, int i) {
 // more chunks than the grid holds runs on a persistent grid that leaves
 // kStackHeadroom CTA slots of every SM free -- so the small sampling and
 // priority-update kernels of the next round find room beside a running
-// delivery (the overlapped timing of Sec. 6.1) -- and its CTAs take chunks
-// from the launch's work counter until the batch is done, which balances
-// the tail without relying on all CTAs being resident.  A smaller batch
+// delivery (the overlapped timing of Sec. 6.1) -- and its CTAs claim chunks
+// from a work word (above) until the batch is done, which balances the
+// tail without relying on all CTAs being resident.  A smaller batch
 // runs one chunk per CTA with no counter, and one more CTA collates the
 // whole batch (collate_batch) so that no streaming warp waits on it; on the
 // persistent grid the head warp of each sample collates it before its span
@@ -335,27 +400,29 @@ k_deliver_stack(Common c, StackArgs a) {
     if (f < total) stack_span<UN>(c, a, f, min(total, f + a.span), lane, pol, false);
     return;
   }
-  // Thread 0 grabs the next chunk while the CTA works on the current one
-  // and publishes it in the other half of s_chunk before the one barrier
-  // per chunk; the half it overwrites was read before the previous barrier.
-  if (threadIdx.x == 0) s_chunk[0] = atomicAdd(&c.work[0], 1u);
+  // Thread 0 makes the CTA's first claim (or takes the fixed share), grabs
+  // the next chunk while the CTA works on the current one and publishes it
+  // in the other half of s_chunk before the one barrier per chunk; the half
+  // it overwrites was read before the previous barrier.
+  __shared__ uint32_t s_owned;
+  if (threadIdx.x == 0) {
+    const uint32_t first = work_first(c.work, c.work_tag);
+    s_owned = first != kWorkFixed;
+    s_chunk[0] = first != kWorkFixed ? first : blockIdx.x;
+  }
   __syncthreads();
+  const bool owned = s_owned != 0;
   uint32_t cur = s_chunk[0];
   for (int p = 1;; p ^= 1) {
     const uint64_t f0 = (uint64_t)cur * per_chunk;
     if (f0 >= total) break;  // uniform across the CTA
     uint32_t nxt = 0;
-    if (threadIdx.x == 0) nxt = atomicAdd(&c.work[0], 1u);
+    if (threadIdx.x == 0) nxt = owned ? work_claim(c.work, c.work_tag) : cur + gridDim.x;
     const uint64_t f = f0 + (uint64_t)warp * a.span;
     if (f < total) stack_span<UN>(c, a, f, min(total, f + a.span), lane, pol, true);
     if (threadIdx.x == 0) s_chunk[p] = nxt;
     __syncthreads();
     cur = s_chunk[p];
-  }
-  // every CTA has made its last grab: the last to retire resets the pair
-  if (threadIdx.x == 0 && atomicAdd(&c.work[1], 1u) == gridDim.x - 1) {
-    c.work[0] = 0u;
-    c.work[1] = 0u;
   }
 }
 
@@ -620,12 +687,17 @@ cudaError_t launch_deliver(edp_ctx *ctx, const int64_t *idx, uint32_t B,
       a.span = 32 * kStackUnroll;
       chunks = n_chunks(a.span);
     }
-    if (grid >= chunks) {
-      grid = chunks + 1;  // one chunk per CTA and the collate CTA, no work counter
-    } else {
-      c.work = ctx->ctrl->work + 2 * (ctx->work_seq++ % kWorkSlots);
+    if (grid >= chunks || chunks + grid >= kWorkMaxChunks) {
+      grid = chunks + 1;  // one chunk per CTA and the collate CTA, no work word
+      if (grid > 0x7FFFFFFFull) return cudaErrorInvalidValue;
+      return launch_pdl(kern, dim3((unsigned)grid), dim3(kThreads), s, c, a);
     }
-    return launch_pdl(kern, dim3((unsigned)grid), dim3(kThreads), s, c, a);
+    const uint64_t seq = ctx->work_seq++;
+    c.work = ctx->ctrl->work + (seq % kWorkSlots);
+    c.work_tag = seq % ((1ull << (64 - kWorkTagShift)) - 1) + 1;
+    cudaError_t e = launch_pdl(kern, dim3((unsigned)grid), dim3(kThreads), s, c, a);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(k_work_release, dim3(1), dim3(32), s, c.work, c.work_tag);
   } else if (cfg.transform == EDP_XFORM_HWC_CHW_BF16) {
     ChwArgs a{};
     a.obs = ctx->st.obs;

@@ -261,8 +261,10 @@ cudaError_t launch_gae(edp_ctx *c, const float *r, const float *v,
   const uint64_t grid = (E + kGaeWarps - 1) / kGaeWarps;
   double *partial = nullptr;
   if (adv_norm) {
-    partial = (double *)ctx_scratch(c, grid * 2 * sizeof(double));
-    if (!partial) return cudaErrorMemoryAllocation;
+    void *blk = nullptr;
+    const cudaError_t e = ctx_scratch(c, grid * 2 * sizeof(double), s, &blk);
+    if (e != cudaSuccess) return e;
+    partial = (double *)blk;
   }
   // A is kept between the kernels in adv, or in adv_norm itself (fp32; the
   // normalisation error this adds is below 2^-24 |A| / std)

@@ -94,9 +94,9 @@ __device__ __forceinline__ uint64_t block_sum(uint64_t v, uint64_t *red) {
 
 // One thread per batch entry: its entry (0 tokens and a flag for an index
 // out of range); per CTA the sum of its 256 lengths.  With `pre` (more than
-// kDirectChunks chunks) the last CTA to finish (a ticket on the launch's
-// work counter) turns those sums into exclusive prefixes and resets the
-// counter.
+// kDirectChunks chunks) the last CTA to finish (a ticket that the context's
+// ordered packed deliveries share) turns those sums into exclusive prefixes
+// and resets the ticket.
 // Chunk `cta` of `ncta` (the CTA's role; the fused GRPO kernel runs it
 // beside the advantages).
 __device__ __forceinline__ void pack_lengths_cta(const uint64_t *__restrict__ soff,
@@ -282,16 +282,21 @@ struct PackPlan {
   uint32_t G;
 };
 
-bool pack_plan(edp_ctx *c, uint32_t B, PackPlan *p) {
+cudaError_t pack_plan(edp_ctx *c, uint32_t B, cudaStream_t s, PackPlan *p) {
   p->G = (B + kPackThreads - 1) / kPackThreads;
   const size_t ent_bytes = ((size_t)B * sizeof(PackEntry) + 255) & ~(size_t)255;
-  uint8_t *scr = (uint8_t *)ctx_scratch(c, ent_bytes + 2 * (size_t)p->G * sizeof(uint64_t));
-  if (!scr) return false;
+  void *blk = nullptr;
+  const cudaError_t e =
+      ctx_scratch(c, ent_bytes + 2 * (size_t)p->G * sizeof(uint64_t), s, &blk);
+  if (e != cudaSuccess) return e;
+  uint8_t *scr = (uint8_t *)blk;
   p->ent = (PackEntry *)scr;
   p->part = (uint64_t *)(scr + ent_bytes);
   p->pre = p->G > kDirectChunks ? p->part + p->G : nullptr;
-  p->work = c->ctrl->work + 2 * (c->work_seq++ % kWorkSlots);
-  return true;
+  // packed deliveries share the scratch above, so they are ordered, and one
+  // ticket serves them all
+  p->work = &c->ctrl->pack_ticket;
+  return cudaSuccess;
 }
 
 cudaError_t launch_gather(edp_ctx *c, const PackPlan &p, const int32_t *tokens, uint32_t B,
@@ -310,8 +315,9 @@ cudaError_t launch_pack(edp_ctx *c, const int32_t *tokens, const uint64_t *soff,
                         int32_t *otok, uint64_t *ooff, float *osv, uint64_t cap,
                         cudaStream_t s) {
   PackPlan p;
-  if (!pack_plan(c, B, &p)) return cudaErrorMemoryAllocation;
-  cudaError_t e = launch_pdl(k_pack_lengths, dim3(p.G), dim3(kPackThreads), s, soff, nseq,
+  cudaError_t e = pack_plan(c, B, s, &p);
+  if (e != cudaSuccess) return e;
+  e = launch_pdl(k_pack_lengths, dim3(p.G), dim3(kPackThreads), s, soff, nseq,
                              idx, B, p.ent, p.part, p.pre, p.work, c->ctrl);
   if (e != cudaSuccess) return e;
   return launch_gather(c, p, tokens, B, sv, otok, ooff, osv, cap, s);
@@ -323,14 +329,15 @@ cudaError_t launch_grpo_pack(edp_ctx *c, const float *r, const uint64_t *goff, u
                              uint32_t B, int32_t *otok, uint64_t *ooff, float *osv,
                              uint64_t cap, cudaStream_t s) {
   PackPlan p;
-  if (!pack_plan(c, B, &p)) return cudaErrorMemoryAllocation;
+  cudaError_t e = pack_plan(c, B, s, &p);
+  if (e != cudaSuccess) return e;
   uint64_t ngc = (ng + kGrpoWarps - 1) / kGrpoWarps;
   if (ngc > 16ull * c->coop_sms) ngc = 16ull * c->coop_sms;
   // a plain launch, as for k_grpo
   k_grpo_pack_lengths<<<dim3((unsigned)(ngc + p.G)), dim3(kPackThreads), 0, s>>>(
       r, goff, ng, eps, adv, (uint32_t)ngc, soff, nseq, idx, B, p.ent, p.part, p.pre, p.work,
       c->ctrl);
-  cudaError_t e = cudaGetLastError();
+  e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   return launch_gather(c, p, tokens, B, adv, otok, ooff, osv, cap, s);
 }

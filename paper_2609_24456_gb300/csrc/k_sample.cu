@@ -179,8 +179,10 @@ cudaError_t launch_permute(edp_ctx *c, uint32_t n, uint64_t seed,
   int lg = 0;
   while ((1ull << (lg + 2)) < n && (1u << lg) < kMaxBuckets) ++lg;  // nb ~ n/4
   const uint32_t nb = 1u << lg;
-  uint8_t *base = (uint8_t *)ctx_perm_scratch(c, perm_scratch_bytes(n));
-  if (!base) return cudaErrorMemoryAllocation;
+  void *block = nullptr;
+  const cudaError_t ge = ctx_perm_scratch(c, perm_scratch_bytes(n), s, &block);
+  if (ge != cudaSuccess) return ge;
+  uint8_t *base = (uint8_t *)block;
   PermScratch sc;
   sc.count = (uint32_t *)base;  // the zeroed head of the block
   sc.cursor = sc.count + kMaxBuckets;

@@ -179,9 +179,10 @@ __device__ __forceinline__ uint32_t tab_hash(uint32_t x, uint32_t mask) {
 // Priority update.  Phase 1 (all CTAs): the priority of every pair -- the
 // given u32, or PER's rule from the TD error, whose fp64 pow is spread over
 // the CTAs -- goes to qbuf.  The last CTA to finish (ticket counter, no
-// waiting) then applies the pairs in batch order, in chunks of 2048 (two pairs per thread): a
-// shared-memory hash table keeps, per slot, the largest batch position
-// (atomicMax), so only the last occurrence of a slot writes its leaf.  The
+// waiting) then applies the pairs in batch order, in chunks of 1024 (two
+// pairs per thread): a shared-memory hash table keeps, per slot, the largest
+// batch position (atomicMax), so only the last occurrence of a slot writes
+// its leaf.  The
 // exact signed delta of each written leaf is added to its ancestors
 // (two's complement wrap makes negative deltas exact); the two top levels,
 // which every pair shares, are summed on chip first.
@@ -196,26 +197,26 @@ k_update(TreeView t, const int64_t *__restrict__ idx,
   __shared__ uint32_t acc_lo[32], acc_hi[32];
   __shared__ unsigned long long warp_root[kUpdThreads / 32];
   const uint32_t *qv_src = q;
+  // Nothing is read or written before the wait on the preceding kernel: it
+  // may be the kernel that writes the TD errors, or the previous update,
+  // whose last CTA may still be reading qbuf.
+  pdl_wait();
+  pdl_launch();
   if (td) {
-    // phase 1 reads only the caller's TD errors, so it runs before the wait
-    // on the preceding kernel (overlapping it when SMs are free); one warp
-    // per CTA, one CTA per 32 pairs, so the fp64 work spreads over SMs
+    // phase 1: one warp per CTA, one CTA per 32 pairs, so the fp64 work
+    // spreads over SMs
     if (threadIdx.x < 32)
       for (uint32_t p = blockIdx.x * 32 + threadIdx.x; p < n; p += gridDim.x * 32)
         qbuf[p] = prio_td(td[p], alpha, eps);
     __threadfence();
-    pdl_wait();
-    pdl_launch();
     __syncthreads();
     if (threadIdx.x == 0) ticket = atomicAdd(&ctrl->upd_count, 1u);
     __syncthreads();
     if (ticket != gridDim.x - 1) return;
     __threadfence();
     qv_src = qbuf;
-  } else {
-    pdl_wait();
-    pdl_launch();
-    if (blockIdx.x != 0) return;
+  } else if (blockIdx.x != 0) {
+    return;
   }
   const uint32_t tsize = n >= kUpdChunk ? kUpdTable
                                         : max(64u, 2u << (31 - __clz(max(n, 1u))));
@@ -402,8 +403,8 @@ cudaError_t launch_update(edp_ctx *c, const int64_t *idx, const uint32_t *q,
   uint32_t *qbuf = nullptr;
   unsigned grid = 1;
   if (td) {
-    qbuf = ctx_qbuf(c, n);
-    if (!qbuf) return cudaErrorMemoryAllocation;
+    const cudaError_t e = ctx_qbuf(c, n, s, &qbuf);
+    if (e != cudaSuccess) return e;
     // 32 priorities (one warp) per CTA: the fp64 work spreads over SMs
     grid = (n + 31) / 32;
     if (grid > 2u * (unsigned)c->coop_sms) grid = 2u * (unsigned)c->coop_sms;
@@ -431,9 +432,11 @@ cudaError_t launch_prio_from_td(const float *td, uint32_t n, double alpha,
 // capture), and runtimes that hand out all device memory up front and forbid
 // allocation later, or that cannot afford the device-wide synchronisation a
 // cudaMalloc/cudaFree may bring.  The array is per device and lives until
-// the process exits; every call on that device shares it, so calls that
-// overlap on the GPU race.  Nothing in it needs to start at zero: a call
-// writes priorities [0, n) before it reads them.
+// the process exits; every call on that device shares it.  Calls queued on
+// one stream are ordered (the kernel touches the array only after its wait
+// on the preceding kernel); calls that can run at the same time on different
+// streams race.  Nothing in it needs to start at zero: a call writes
+// priorities [0, n) before it reads them.
 // ---------------------------------------------------------------------------
 #include <mutex>
 
@@ -461,16 +464,6 @@ cudaError_t static_qbuf(int dev, uint32_t **out) {
   return cudaSuccess;
 }
 
-bool is_device_ptr(const void *p, int dev) {
-  cudaPointerAttributes a;
-  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
-    cudaGetLastError();
-    return false;
-  }
-  return (a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged) &&
-         a.device == dev;
-}
-
 }  // namespace
 }  // namespace edp
 
@@ -478,38 +471,23 @@ extern "C" edp_status edp_update_priorities_td_static(
     edp_ctx *ctx, const int64_t *idx, const float *td, uint32_t n,
     double alpha, double eps, edp_stream stream) {
   using namespace edp;
-  if (!ctx) return EDP_ERR_INVALID;
-  if (!ctx->depth) {
-    ctx->err = "edp_update_priorities_td_static: context has no priorities";
-    return EDP_ERR_STATE;
-  }
-  if (n == 0) return EDP_OK;
-  if (n > kStaticMaxPairs) {
-    ctx->err = "edp_update_priorities_td_static: n exceeds the fixed maximum "
-               "of 16384 pairs (use edp_update_priorities_td)";
-    return EDP_ERR_INVALID;
-  }
-  if (!idx || !td || !is_device_ptr(idx, ctx->cfg.device) ||
-      !is_device_ptr(td, ctx->cfg.device)) {
-    ctx->err = "edp_update_priorities_td_static: idx and td must be device memory";
-    return EDP_ERR_INVALID;
-  }
-  if (!(alpha >= 0.0 && eps >= 0.0)) {
-    ctx->err = "edp_update_priorities_td_static: alpha, eps >= 0";
-    return EDP_ERR_INVALID;
-  }
-  if (ctx->cfg.device < 0 || ctx->cfg.device >= kMaxDevices) {
-    ctx->err = "edp_update_priorities_td_static: device ordinal out of range";
-    return EDP_ERR_INVALID;
-  }
-  cudaSetDevice(ctx->cfg.device);
+  static const char who[] = "edp_update_priorities_td_static";
+  if (ctx && n && !td) return fail(ctx, EDP_ERR_INVALID, "%s: td NULL", who);
+  const edp_status st = update_args(ctx, who, idx, nullptr, td, n, alpha, eps);
+  if (st != EDP_OK || n == 0) return st;
+  if (n > kStaticMaxPairs)
+    return fail(ctx, EDP_ERR_INVALID,
+                "%s: n exceeds the fixed maximum of 16384 pairs (use "
+                "edp_update_priorities_td)", who);
+  if (ctx->cfg.device < 0 || ctx->cfg.device >= kMaxDevices)
+    return fail(ctx, EDP_ERR_INVALID, "%s: device ordinal out of range", who);
+  DeviceGuard dg(ctx->cfg.device);
   uint32_t *qbuf = nullptr;
   cudaError_t e = static_qbuf(ctx->cfg.device, &qbuf);
   if (e != cudaSuccess) {
     cudaGetLastError();
-    ctx->err = std::string("edp_update_priorities_td_static: cudaGetSymbolAddress: ") +
-               cudaGetErrorString(e);
-    return EDP_ERR_CUDA;
+    return fail(ctx, EDP_ERR_CUDA, "%s: cudaGetSymbolAddress: %s", who,
+                cudaGetErrorString(e));
   }
   const uint64_t size = ctx->total < ctx->cap ? ctx->total : ctx->cap;
   const uint64_t oldest = (ctx->total - size) % ctx->cap;
@@ -520,8 +498,7 @@ extern "C" edp_status edp_update_priorities_td_static(
                  ctx->cap, oldest, size, ctx->defer, ctx->ctrl);
   if (e != cudaSuccess) {
     cudaGetLastError();
-    ctx->err = std::string("edp_update_priorities_td_static: ") + cudaGetErrorString(e);
-    return EDP_ERR_CUDA;
+    return fail(ctx, EDP_ERR_CUDA, "%s: %s", who, cudaGetErrorString(e));
   }
   return EDP_OK;
 }

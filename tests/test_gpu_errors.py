@@ -104,3 +104,72 @@ def test_failing_allocator(edp_lib, orc):
     assert np.array_equal(to_np(idx), orc.permutation(64, 5, 0))
     ring.close()
     assert not live  # everything libedp took went back through free
+
+
+def test_scratch_growth_refused_during_capture(edp_lib, orc):
+    """A call whose scratch would have to grow while its stream is being
+    captured returns EDP_ERR_STATE and enqueues nothing (the capture stays
+    usable); made once outside the capture, the same call then captures and
+    replays to the oracle's result."""
+    edp = edp_lib
+    cfg = edp.make_config(64, (3, 16, 16), edp.EDP_XFORM_HWC_CHW_BF16)
+    ring = edp.Ring(cfg, action=False, reward=False, done=False)
+    T, E = 8, 16
+    r = torch.randn(T, E, device="cuda")
+    v = torch.randn(T + 1, E, device="cuda")
+    d = torch.zeros(T, E, dtype=torch.uint8, device="cuda")
+    adv = torch.zeros(T, E, device="cuda")
+    ret = torch.zeros(T, E, device="cuda")
+    nrm = torch.zeros(T, E, device="cuda")
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, capture_error_mode="thread_local"):
+        with pytest.raises(edp.EdpError) as e:
+            edp.edp_gae(ring.ctx, r, v, d, T, E, 0.99, 0.95, adv, ret, nrm)
+    assert e.value.status == edp.EDP_ERR_STATE
+    assert "captur" in str(e.value)
+    edp.edp_gae(ring.ctx, r, v, d, T, E, 0.99, 0.95, adv, ret, nrm)  # grows here
+    edp.edp_sync(ring.ctx)
+    nrm.zero_()
+    g2 = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g2, capture_error_mode="thread_local"):
+        edp.edp_gae(ring.ctx, r, v, d, T, E, 0.99, 0.95, adv, ret, nrm)
+    g2.replay()
+    torch.cuda.synchronize()
+    edp.edp_sync(ring.ctx)
+    A, _ = orc.gae(to_np(r), to_np(v), to_np(d), 0.99, 0.95)
+    N, _, _ = orc.normalize(A)
+    assert np.abs(to_np(nrm) - N).max() <= 1e-5
+    ring.close()
+
+
+def test_calls_keep_the_callers_current_device(edp_lib, orc):
+    """Every call on a context of device 0 leaves the calling thread's
+    current device as it found it: device 0 here, and, where a second GPU
+    exists, the other device made current before the calls."""
+    edp = edp_lib
+    homes = [0] + ([1] if torch.cuda.device_count() > 1 else [])
+    m = MirroredDqn(100, prioritized=True)
+    frames, action, reward, done = fx.dqn_transitions(3, 60)
+    m.ingest(orc, frames, action, reward, done)
+    idx = torch.zeros(8, dtype=torch.int64, device="cuda:0")
+    q = torch.zeros(8, dtype=torch.int32, device="cuda:0")
+    td = torch.ones(8, dtype=torch.float32, device="cuda:0")
+    obs, nxt, act, rew, dn = dqn_outputs(8, 4, 7056)
+    s0 = torch.cuda.Stream(device=0)
+    for home in homes:
+        torch.cuda.set_device(home)
+        calls = [
+            lambda: edp.edp_sample(m.ring.ctx, edp.EDP_SAMPLE_PRIORITIZED, 8, 1, 0, idx, q,
+                                   stream=s0),
+            lambda: edp.edp_deliver(m.ring.ctx, idx, 8, edp.make_batch(obs, nxt, act, rew, dn),
+                                    stream=s0),
+            lambda: edp.edp_update_priorities_td(m.ring.ctx, idx, td, 8, 0.6, 1e-6, stream=s0),
+            lambda: edp.edp_update_priorities_td_static(m.ring.ctx, idx, td, 8, 0.6, 1e-6,
+                                                        stream=s0),
+            lambda: edp.edp_sync(m.ring.ctx, stream=s0),
+        ]
+        for call in calls:
+            call()
+            assert torch.cuda.current_device() == home
+    torch.cuda.set_device(0)

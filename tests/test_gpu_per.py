@@ -224,3 +224,46 @@ def test_prioritized_replay_full_size(edp_lib, orc):
         m.frames[need] = fx.content_bytes(seed, need, F)  # id == slot here
         _round(edp, orc, m, B, seed=7, rnd=rnd, td_seed=900 + rnd, subset=subset)
         check_tree(orc, m.ring, m.st)
+
+
+@pytest.mark.parametrize("path", ["u32", "td"])
+def test_updates_back_to_back_on_one_stream(edp_lib, orc, path):
+    """Two priority updates queued straight after each other on one stream,
+    with no synchronisation (and no other work) between them, over
+    overlapping slots.  The second launch may start while the first is
+    still applying its pairs, so neither may touch memory the other uses
+    before its wait on the preceding kernel.  Whole tree bit-exact against
+    the oracle applying both batches in order (for the TD-error path, with
+    the priorities the device's rule gives for the same TD errors)."""
+    edp = edp_lib
+    cap, n = 3000, 5000
+    frames, action, reward, done = fx.dqn_transitions(12, 2500, 84 * 4)
+    q = orc.priorities_from_td(fx.td_errors(12, 2500), ALPHA, EPS)
+    m = MirroredDqn(cap, prioritized=True, F=84 * 4)
+    m.ingest(orc, frames, action, reward, done, q=q)
+    rng = np.random.default_rng(41 + (path == "td"))
+    batches = []
+    for call in range(2):
+        idx = rng.integers(0, 2500, size=n).astype(np.int64)
+        idx[: n // 2] = rng.integers(0, 500, size=n // 2)  # slots both batches hit
+        idx[7] = m.total - 1  # the newest (deferred) transition
+        if path == "u32":
+            qu = rng.integers(0, 1 << 31, size=n).astype(np.uint32)
+            batches.append((cuda(idx), cuda(qu), idx, qu))
+        else:
+            td = (rng.standard_normal(n) * 3).astype(np.float32)
+            d_td = cuda(td)
+            qd = torch.zeros(n, dtype=torch.int32, device="cuda")
+            edp.edp_priorities_from_td(m.ring.ctx, d_td, n, ALPHA, EPS, qd)
+            edp.edp_sync(m.ring.ctx)
+            batches.append((cuda(idx), d_td, idx, u32(qd)))
+    torch.cuda.synchronize()
+    for d_idx, d_val, _, _ in batches:  # back to back, nothing between
+        if path == "u32":
+            edp.edp_update_priorities(m.ring.ctx, d_idx, d_val, n)
+        else:
+            edp.edp_update_priorities_td(m.ring.ctx, d_idx, d_val, n, ALPHA, EPS)
+    edp.edp_sync(m.ring.ctx)
+    for _, _, idx, qu in batches:
+        orc.update_leaves(m.st, m.total, idx, qu)
+    check_tree(orc, m.ring, m.st)

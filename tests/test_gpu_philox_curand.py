@@ -3,11 +3,10 @@ values: cuRAND's device generator of the same name, run through its public
 API (curand_init with a seed, a subsequence and an offset, then curand4),
 must give the same 128-bit blocks for counters whose four words are all in
 use (offset / 4 in words 0-1, the subsequence in words 2-3) and keys of
-every kind.  The probe is compiled here from tests/curand_philox_probe.cu."""
+every kind.  The probe, tests/curand_philox_probe.cu, is compiled by the
+package's build step (with the nvcc that builds libedp) or here, the same
+way, when that step has not made it."""
 import ctypes as C
-import os
-import shutil
-import subprocess
 
 import numpy as np
 import pytest
@@ -15,19 +14,11 @@ import torch
 
 pytestmark = pytest.mark.gpu
 
-HERE = os.path.dirname(os.path.abspath(__file__))
-
 
 @pytest.fixture(scope="module")
-def probe(tmp_path_factory):
-    nvcc = shutil.which("nvcc") or "/usr/local/cuda/bin/nvcc"
-    if not os.path.exists(nvcc):
-        pytest.skip("nvcc not found")
-    so = str(tmp_path_factory.mktemp("curand") / "probe.so")
-    subprocess.run([nvcc, "-gencode", "arch=compute_103a,code=sm_103a", "-O2", "-shared",
-                    "-Xcompiler", "-fPIC", os.path.join(HERE, "curand_philox_probe.cu"),
-                    "-o", so], check=True, capture_output=True)
-    lib = C.CDLL(so)
+def probe():
+    from paper_2609_24456_gb300 import build
+    lib = C.CDLL(build.build_curand_probe())
     lib.curand_philox_probe.argtypes = [C.c_void_p] * 3 + [C.c_uint, C.c_void_p]
     lib.curand_philox_probe.restype = C.c_int
     return lib

@@ -1,13 +1,16 @@
-"""The work-counter path of the frame-stack delivery.
+"""The work-word path of the frame-stack delivery.
 
 A batch with more work chunks than the delivery's persistent grid holds is
-handed out chunk by chunk from a per-launch counter (32 counter pairs per
-context, used round robin and reset by each launch's last CTA).  Here a
-batch of 1,024 stacks (about 2,900 chunks) is delivered many times: from two
-streams at once, so two launches with different counter pairs run
-concurrently, and more than 32 times in a row inside a CUDA graph, so every
-pair is reused.  Every delivery must equal the first bit for bit, and the
-first must equal the oracle on a strided sample of rows.
+handed out chunk by chunk from one of the context's 32 work words (chosen
+round robin at issue; a word is claimed by the launch's own grid id, and a
+CTA that finds another launch working from its word takes a fixed share of
+the chunks instead).  Here a batch of 1,024 stacks (about 2,900 chunks) is
+delivered many times: from two streams at once, and more than 32 times in a
+row inside a CUDA graph, so every word is reused; and 40 deliveries that may
+all run at once -- released together on eight streams, eagerly and from a
+graph replayed twice -- so that launches 32 apart share a word while both
+run.  Every delivery must equal the first bit for bit, and the first must
+equal the oracle on a strided sample of rows.
 """
 import numpy as np
 import pytest
@@ -95,3 +98,66 @@ def test_outputs_16_byte_aligned_only(edp_lib, orc, B):
     for x, y in zip(aligned, odd):
         assert np.array_equal(bits(x) if x.is_floating_point() else to_np(x),
                               bits(y) if y.is_floating_point() else to_np(y))
+
+
+def test_forty_deliveries_in_flight_at_once(edp_lib, orc):
+    """40 large deliveries with no order between them (8 streams, released
+    by one event; then the same as 40 independent nodes of one graph,
+    replayed twice with the outputs overwritten in between, so that a
+    replay that skipped its work would show), each into its own outputs."""
+    edp = edp_lib
+    B, n_out, n_streams = 256, 40, 8
+    frames, action, reward, done = fx.dqn_transitions(44, N_INGEST, done_p=0.05)
+    m = MirroredDqn(CAP)
+    m.ingest(orc, frames, action, reward, done)
+    idx = torch.empty(B, dtype=torch.int64, device="cuda")
+    edp.edp_sample(m.ring.ctx, edp.EDP_SAMPLE_UNIFORM, B, 45, 0, idx)
+    first = dqn_outputs(B, m.K, m.F)
+    edp.edp_deliver(m.ring.ctx, idx, B, edp.make_batch(*first))
+    edp.edp_sync(m.ring.ctx)
+    ref = [bits(t) if t.is_floating_point() else to_np(t) for t in first]
+    sel = np.arange(0, B, 5)
+    r_obs, r_nxt, r_act, r_rew, r_dn = orc.deliver_dqn(
+        m.frames, m.done, m.action, m.reward, m.cap, m.total, m.K, to_np(idx)[sel])
+    assert np.array_equal(ref[0][sel].reshape(r_obs.shape), r_obs.view(np.uint32))
+    assert np.array_equal(ref[1][sel].reshape(r_nxt.shape), r_nxt.view(np.uint32))
+    assert np.array_equal(ref[2][sel], r_act)
+    assert np.array_equal(ref[4][sel], r_dn)
+    outs = [dqn_outputs(B, m.K, m.F) for _ in range(n_out)]
+    batches = [edp.make_batch(*o) for o in outs]
+    streams = [torch.cuda.Stream() for _ in range(n_streams)]
+
+    def check(tag):
+        for i, o in enumerate(outs):
+            for j, (x, y) in enumerate(zip(ref, o)):
+                got = bits(y) if y.is_floating_point() else to_np(y)
+                assert np.array_equal(x, got), (tag, i, j)
+
+    torch.cuda.synchronize()
+    go = torch.cuda.Event()
+    go.record()
+    for i, b in enumerate(batches):
+        st = streams[i % n_streams]
+        st.wait_event(go)
+        edp.edp_deliver(m.ring.ctx, idx, B, b, stream=st)
+    torch.cuda.synchronize()
+    edp.edp_sync(m.ring.ctx)
+    check("eager")
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, capture_error_mode="thread_local"):
+        fork = torch.cuda.current_stream()
+        for i, b in enumerate(batches):
+            st = streams[i % n_streams]
+            st.wait_stream(fork)
+            edp.edp_deliver(m.ring.ctx, idx, B, b, stream=st)
+        for st in streams:
+            fork.wait_stream(st)
+    for rep in range(2):
+        for o in outs:
+            for t in o:
+                t.fill_(7)
+        torch.cuda.synchronize()
+        g.replay()
+        torch.cuda.synchronize()
+        edp.edp_sync(m.ring.ctx)
+        check("replay %d" % rep)

@@ -12,10 +12,9 @@ cases (hypothesis, derandomised so every run sees the same examples):
 import numpy as np
 import pytest
 
-hyp = pytest.importorskip("hypothesis")
-from hypothesis import given, settings, strategies as st  # noqa: E402
+from hypothesis import given, settings, strategies as st
 
-from oracle import llm  # noqa: E402
+from oracle import llm
 
 SETTINGS = settings(max_examples=60, derandomize=True, deadline=None)
 

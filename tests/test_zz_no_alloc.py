@@ -7,14 +7,16 @@ it keeps its per-pair scratch in a fixed per-device array instead of
 allocating it.  Its results must equal those of the allocating
 edp_update_priorities_td on the same arguments -- here compared on the whole
 priority tree (leaves, every internal sum, the deferred and the running
-maximum priority), bit for bit, after two calls in a row.  This file is
-collected last so that a failure here leaves every other test already run.
+maximum priority), bit for bit, after two calls in a row, and after two
+calls queued back to back on one stream; and against the oracle.  This
+file is collected last so that a failure here leaves every other test
+already run.
 """
 import numpy as np
 import pytest
 import torch
 
-from gpu_util import MirroredDqn, cuda, fx, tree_levels
+from gpu_util import MirroredDqn, check_tree, cuda, fx, tree_levels
 
 pytestmark = pytest.mark.gpu
 
@@ -57,6 +59,57 @@ def test_static_update_matches_allocating_update(edp_lib, orc):
         assert (pa, ma) == (pb, mb)
         # and the update did happen: the leaves of the updated slots moved
         assert not np.array_equal(la[:cap], b.st.leaves)
+    # then a pair of calls queued back to back on one stream, with nothing
+    # between them: stream order alone keeps them apart
+    pairs = []
+    for call in range(2):
+        n = 4000
+        idx = rng.integers(0, n_ingest, size=n).astype(np.int64)
+        idx[: n // 2] = rng.integers(0, 300, size=n // 2)  # slots both calls hit
+        pairs.append((cuda(idx), cuda(fx.td_errors(200 + call, n)), n))
+    torch.cuda.synchronize()
+    for d_idx, d_td, n in pairs:
+        edp.edp_update_priorities_td(a.ring.ctx, d_idx, d_td, n, ALPHA, EPS)
+    for d_idx, d_td, n in pairs:
+        edp.edp_update_priorities_td_static(b.ring.ctx, d_idx, d_td, n, ALPHA, EPS)
+    edp.edp_sync(a.ring.ctx)
+    edp.edp_sync(b.ring.ctx)
+    la, lva, pa, ma = tree_levels(a.ring)
+    lb, lvb, pb, mb = tree_levels(b.ring)
+    assert np.array_equal(la, lb)
+    for d, (x, y) in enumerate(zip(lva, lvb)):
+        assert np.array_equal(x, y), d
+    assert (pa, ma) == (pb, mb)
+
+
+def test_static_updates_back_to_back_match_oracle(edp_lib, orc):
+    """Two calls of the allocation-free update queued straight after each
+    other on one stream (no synchronisation, overlapping slots), then the
+    whole tree bit for bit against the oracle applying both batches in
+    order, with the priorities the device's rule gives for the same TD
+    errors."""
+    edp = edp_lib
+    cap, n_ingest = 3000, 2500
+    (m, _) = _twin_rings(orc, cap, n_ingest)
+    rng = np.random.default_rng(23)
+    calls = []
+    for call in range(2):
+        n = 5000
+        idx = rng.integers(0, n_ingest, size=n).astype(np.int64)
+        idx[: n // 2] = rng.integers(0, 400, size=n // 2)
+        idx[9] = n_ingest - 1  # the newest transition: deferred priority
+        d_td = cuda(fx.td_errors(300 + call, n))
+        qd = torch.zeros(n, dtype=torch.int32, device="cuda")
+        edp.edp_priorities_from_td(m.ring.ctx, d_td, n, ALPHA, EPS, qd)
+        edp.edp_sync(m.ring.ctx)
+        calls.append((cuda(idx), d_td, n, idx, qd.cpu().numpy().view(np.uint32)))
+    torch.cuda.synchronize()
+    for d_idx, d_td, n, _, _ in calls:
+        edp.edp_update_priorities_td_static(m.ring.ctx, d_idx, d_td, n, ALPHA, EPS)
+    edp.edp_sync(m.ring.ctx)
+    for _, _, _, idx, q in calls:
+        orc.update_leaves(m.st, m.total, idx, q)
+    check_tree(orc, m.ring, m.st)
 
 
 def test_static_update_rejects_sizes_above_its_maximum(edp_lib, orc):
