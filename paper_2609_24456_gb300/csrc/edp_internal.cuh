@@ -17,17 +17,12 @@ namespace edp {
 enum : uint32_t {
   DEVERR_INDEX = 1u,    // a slot index outside the sampleable range
   DEVERR_EMPTY = 2u,    // total priority 0 at sampling time
-  DEVERR_TIMEOUT = 4u,  // a bounded device-side wait expired (no kernel waits now)
+  DEVERR_TIMEOUT = 4u,  // a bounded device-side wait expired (staged delivery)
   DEVERR_TREE = 8u,     // a tree descent found no child holding its target
   DEVERR_OVERFLOW = 16u,  // packed output larger than its buffer (clipped)
 };
 
 // Small device-resident control block (one per context).
-// Work words of the dynamically scheduled frame-stack delivery: launch n of
-// a context starts at word n mod kWorkSlots (see k_deliver.cu for the claim
-// protocol, which stays correct whatever the number of launches in flight).
-constexpr int kWorkSlots = 32;
-
 struct Ctrl {
   uint32_t err;
   uint32_t pending_q;  // deferred priority of the newest transition
@@ -37,7 +32,6 @@ struct Ctrl {
   uint32_t pack_ticket;  // packed delivery: length CTAs done (calls are ordered)
   uint32_t pad;
   unsigned long long bad_index;  // first offending index (diagnostics)
-  unsigned long long work[kWorkSlots];
 };
 
 constexpr int kFanout = 32;
@@ -77,7 +71,6 @@ struct edp_ctx {
   float naff_a[4] = {}, naff_b[4] = {};
   int norm_affine = 0;
   int coop_sms = 0;
-  uint64_t work_seq = 0;  // frame-stack delivery launches so far (work words)
   std::string err;
 };
 
@@ -258,6 +251,71 @@ __device__ __forceinline__ void st_stream(uint4 *p, uint4 v, uint64_t pol) {
   asm volatile("st.global.L1::no_allocate.L2::cache_hint.v4.u32 [%0], {%1, %2, %3, %4}, %5;"
                :: "l"(p), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w), "l"(pol)
                : "memory");
+}
+
+// ---------------------------------------------------------------------------
+// Shared-memory staging: mbarriers and bulk asynchronous copies (sm_90+).
+// A bulk copy global -> shared moves a contiguous run of bytes (both
+// addresses 16-byte aligned, size a multiple of 16) on the copy engine of
+// the SM and signals its completion on an mbarrier as a transaction count.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_addr(const void *p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+__device__ __forceinline__ void mbar_init(unsigned long long *bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" :: "r"(smem_addr(bar)), "r"(count)
+               : "memory");
+}
+// Makes initialised mbarriers visible to the async proxy (the bulk copies)
+// and to the other threads once followed by a CTA barrier.
+__device__ __forceinline__ void mbar_init_fence() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_arrive(unsigned long long *bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" :: "r"(smem_addr(bar)) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_tx(unsigned long long *bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;"
+               :: "r"(smem_addr(bar)), "r"(bytes) : "memory");
+}
+// Raises the bytes the current phase of `bar` waits for, without arriving.
+__device__ __forceinline__ void mbar_expect_tx(unsigned long long *bar, uint32_t bytes) {
+  asm volatile("mbarrier.expect_tx.relaxed.cta.shared::cta.b64 [%0], %1;"
+               :: "r"(smem_addr(bar)), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ bool mbar_test(unsigned long long *bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile("{\n\t.reg .pred p;\n\t"
+               "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+               "selp.u32 %0, 1, 0, p;\n\t}"
+               : "=r"(ok) : "r"(smem_addr(bar)), "r"(parity) : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ uint64_t global_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+// Waits for the phase of `bar` with parity `parity` to complete; gives up
+// after about `limit_ns` nanoseconds (false), so that no wait can hang.
+__device__ __forceinline__ bool mbar_wait(unsigned long long *bar, uint32_t parity,
+                                          uint64_t limit_ns) {
+  if (mbar_test(bar, parity)) return true;
+  const uint64_t t0 = global_ns();
+  for (;;) {
+    for (int i = 0; i < 64; ++i)
+      if (mbar_test(bar, parity)) return true;
+    if (global_ns() - t0 > limit_ns) return false;
+  }
+}
+// bytes [src, src + n) -> shared [dst, dst + n), completion counted on bar;
+// `pol` is an L2 cache policy for the source.
+__device__ __forceinline__ void bulk_load(void *dst, const void *src, uint32_t n,
+                                          unsigned long long *bar, uint64_t pol) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1], %2, [%3], %4;"
+      :: "r"(smem_addr(dst)), "l"(src), "r"(n), "r"(smem_addr(bar)), "l"(pol) : "memory");
 }
 
 __device__ __forceinline__ void flag(Ctrl *c, uint32_t bits,

@@ -8,8 +8,9 @@
 // 32-bit word of a frame, an 8-pixel group, an 8-byte run of a plane), cut
 // into warp spans whose size is set from the work, not from the grid: a
 // warp runs a few iterations of its unrolled loop per span and the grid
-// holds as many CTAs as that takes (several waves), so the block scheduler,
-// or for the frame stack a work counter, balances the tail.  A warp walks
+// holds as many CTAs as that takes (several waves), so the block scheduler
+// balances the tail.  (A large frame-stack batch instead streams its frames
+// through shared memory: k_deliver_stack_staged below.)  A warp walks
 // its span segment by segment (a segment never crosses a frame or image),
 // resolving the sample's slot, episode-boundary mask and source pointer
 // once per segment.  Loads are the payload bytes a lane needs for one
@@ -36,8 +37,8 @@ constexpr int kWarps = kThreads / 32;
 constexpr int kNormUnroll = 8;
 
 // unrolled rows per warp iteration and iterations per warp (chunk span) of
-// each kernel; CTA slots per SM the frame-stack delivery leaves free
-constexpr int kStackUnroll = 4, kStackIters = 3, kStackHeadroom = 2;
+// each kernel
+constexpr int kStackUnroll = 4;
 constexpr int kStackMinBlocks = 6;  // __launch_bounds__: at most 40 registers
 constexpr int kHwcUnroll = 2, kHwcIters = 2;
 constexpr int kNormIters = 3;
@@ -58,8 +59,6 @@ struct Common {
   const float *gsrc0, *gsrc1;
   float *gdst0, *gdst1;
   Ctrl *ctrl;
-  unsigned long long *work;  // this launch's work word, or null (one chunk per CTA)
-  unsigned long long work_tag;
   float r1, r2;
   // fused uniform sampling: idx is then an output, sample k is drawn here
   int draw;
@@ -202,70 +201,6 @@ __device__ __forceinline__ float byte_f(uint32_t w, int i) {
 }
 
 // ---------------------------------------------------------------------------
-// Work claims of a persistent delivery grid.  The CTAs of a launch take
-// chunks in order from one 64-bit work word of the context, laid out as
-//   [63:28] owner tag   [27:0] chunks handed out;
-// tag 0 means free.  A launch's tag is 1 + its call number on the context
-// (host side: unique for every call, and for every node of a captured
-// graph).  A CTA claims from the word if its launch owns it, takes the word
-// over if it is free (claiming chunk 0), and otherwise -- another launch
-// still owns it -- takes a fixed share: chunks blockIdx.x, blockIdx.x +
-// gridDim.x, ...  A one-thread release kernel, queued after the delivery
-// on the same stream, frees the word once every CTA of the launch has
-// finished, so an owned word never changes hands while its owner runs, a
-// replayed graph finds its words free again, and no claim of one launch
-// can land on another's count.  Every chunk is processed: if any CTA of
-// the launch owns the word, the owning CTAs claim until the chunks run out;
-// if none does, the fixed shares cover them all; where both happen some
-// chunks are written twice, with the same bytes.  (Only the same captured
-// node running twice at once could meet its own tag on a live word; the
-// two share the claims and, having the same arguments, still write every
-// chunk of the one batch.)
-// ---------------------------------------------------------------------------
-constexpr int kWorkTagShift = 28;
-constexpr unsigned long long kWorkClaimMask = (1ull << kWorkTagShift) - 1;
-constexpr uint32_t kWorkMaxChunks = 1u << 27;  // chunks + grid stay below 2^28
-constexpr uint32_t kWorkFixed = 0xffffffffu;   // first claim: take the fixed share
-constexpr uint32_t kWorkDone = 0xfffffffeu;    // no chunk left for this launch
-
-// A chunk of the launch with tag `tag` (or kWorkDone).
-__device__ __forceinline__ uint32_t work_claim(unsigned long long *wd,
-                                               unsigned long long tag) {
-  const unsigned long long old = atomicAdd(wd, 1ull);
-  return (old >> kWorkTagShift) == tag ? (uint32_t)(old & kWorkClaimMask) : kWorkDone;
-}
-
-// A CTA's first claim: a chunk, or kWorkFixed when another launch owns the
-// word.
-__device__ __forceinline__ uint32_t work_first(unsigned long long *wd,
-                                               unsigned long long tag) {
-  unsigned long long w = *reinterpret_cast<volatile unsigned long long *>(wd);
-  for (int tries = 0; tries < 8; ++tries) {
-    const unsigned long long owner = w >> kWorkTagShift;
-    if (owner == tag) return work_claim(wd, tag);
-    if (owner != 0) return kWorkFixed;
-    const unsigned long long mine = (tag << kWorkTagShift) | 1ull;  // chunk 0 taken
-    const unsigned long long prev = atomicCAS(wd, w, mine);
-    if (prev == w) return 0;
-    w = prev;
-  }
-  return kWorkFixed;
-}
-
-// Frees the word of the launch with tag `tag`, after that launch (the
-// preceding kernel on the stream) has completed.
-__global__ void k_work_release(unsigned long long *wd, unsigned long long tag) {
-  pdl_wait();
-  pdl_launch();
-  unsigned long long w = *reinterpret_cast<volatile unsigned long long *>(wd);
-  for (int tries = 0; tries < 8 && (w >> kWorkTagShift) == tag; ++tries) {
-    const unsigned long long prev = atomicCAS(wd, w, 0ull);
-    if (prev == w) break;
-    w = prev;
-  }
-}
-
-// ---------------------------------------------------------------------------
 // Frame stack, float32 (DQN), on the load / store units.  A unit is one
 // 32-bit word of frame m in [0, U) of sample k -- the frame at logical
 // offset j = off - K + 1 + m, which is obs slot m (m < K) and next_obs slot
@@ -277,18 +212,10 @@ __global__ void k_work_release(unsigned long long *wd, unsigned long long tag) {
 // anchor" (zeroes the frame in obs and next_obs) and "at the anchor" (zeroes
 // it in next_obs only).
 //
-// Scheduling: the work is cut into chunks of kWarps spans.  A batch with
-// more chunks than the grid holds runs on a persistent grid that leaves
-// kStackHeadroom CTA slots of every SM free -- so the small sampling and
-// priority-update kernels of the next round find room beside a running
-// delivery (the overlapped timing of Sec. 6.1) -- and its CTAs claim chunks
-// from a work word (above) until the batch is done, which balances the
-// tail without relying on all CTAs being resident.  A smaller batch
-// runs one chunk per CTA with no counter, and one more CTA collates the
-// whole batch (collate_batch) so that no streaming warp waits on it; on the
-// persistent grid the head warp of each sample collates it before its span
-// (measured: a collate CTA there made the isolated launch faster, 29.1 ->
-// 25.6 us, but the overlapped replay round slower, 21.0 -> 23-24 us).
+// This direct form serves batches too small to fill the GPU with staged
+// pieces (below): one chunk per CTA, no work counter, and one more CTA
+// collates the whole batch (collate_batch) so that no streaming warp waits
+// on it.
 // ---------------------------------------------------------------------------
 struct StackArgs {
   const uint8_t *frames;
@@ -305,7 +232,7 @@ struct StackArgs {
 template <int UN>
 __device__ __forceinline__ void stack_span(const Common &c, const StackArgs &a,
                                            uint64_t f, uint64_t end, int lane,
-                                           uint64_t pol, bool head_collate) {
+                                           uint64_t pol) {
   const uint64_t per = (uint64_t)a.U * a.W;  // units per sample
   const float4 zero4 = make_float4(0.f, 0.f, 0.f, 0.f);
   while (f < end) {
@@ -315,10 +242,8 @@ __device__ __forceinline__ void stack_span(const Common &c, const StackArgs &a,
     const uint32_t w_lo = rem - m * a.W;
     const uint64_t seg_end = min(end, (uint64_t)k * per + (uint64_t)(m + 1) * a.W);
     const uint32_t w_hi = (uint32_t)(seg_end - (uint64_t)k * per - (uint64_t)m * a.W);
-    const bool head = head_collate && rem == 0;
     uint64_t slot = 0, off = 0;
-    const bool ok = sample_slot(c, k, &slot, &off, head && lane == 0);
-    if (head) collate(c, k, ok, slot, off, lane);
+    const bool ok = sample_slot(c, k, &slot, &off, false);
     const int64_t j = (int64_t)off - (int64_t)(a.K - 1) + (int64_t)m;
     const bool has_obs = m < a.K;
     const bool has_next = a.next && m >= 1;
@@ -384,46 +309,270 @@ __device__ __forceinline__ void stack_span(const Common &c, const StackArgs &a,
 template <int UN>
 __global__ void __launch_bounds__(kThreads, kStackMinBlocks)
 k_deliver_stack(Common c, StackArgs a) {
-  __shared__ uint32_t s_chunk[2];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const uint64_t pol = policy_stream();
   pdl_wait();
   pdl_launch();
-  const uint64_t total = (uint64_t)c.B * a.U * a.W;
-  const uint64_t per_chunk = (uint64_t)kWarps * a.span;
-  if (!c.work) {  // one chunk per CTA; CTA 0 collates the batch
-    if (blockIdx.x == 0) {
-      collate_batch(c);
-      return;
-    }
-    const uint64_t f = (uint64_t)(blockIdx.x - 1) * per_chunk + (uint64_t)warp * a.span;
-    if (f < total) stack_span<UN>(c, a, f, min(total, f + a.span), lane, pol, false);
+  if (blockIdx.x == 0) {  // CTA 0 collates the batch
+    collate_batch(c);
     return;
   }
-  // Thread 0 makes the CTA's first claim (or takes the fixed share), grabs
-  // the next chunk while the CTA works on the current one and publishes it
-  // in the other half of s_chunk before the one barrier per chunk; the half
-  // it overwrites was read before the previous barrier.
-  __shared__ uint32_t s_owned;
+  const uint64_t total = (uint64_t)c.B * a.U * a.W;
+  const uint64_t f = (uint64_t)(blockIdx.x - 1) * kWarps * a.span + (uint64_t)warp * a.span;
+  if (f < total) stack_span<UN>(c, a, f, min(total, f + a.span), lane, pol);
+}
+
+// ---------------------------------------------------------------------------
+// Frame stack, float32, staged through shared memory (batches that fill the
+// GPU).  A unit is one piece of one frame: piece p of frame m of sample k,
+// where frame m is the one at logical offset off - K + 1 + m (obs slot m for
+// m < K, next_obs slot m - 1 for m >= 1), and the npieces pieces of a frame
+// are equal runs of at most kPiece bytes.  Units are dealt to the CTAs round
+// robin (unit u to CTA u mod grid): equal units, so the split is balanced
+// without a work counter, and no state outlives the launch.  Per CTA:
+//  - warp 0 (producer) resolves 32 of its units at a time, a lane each:
+//    index -> slot and logical offset -> source address, and the done flags
+//    of the frame's window (offsets j .. off).  It issues the bulk copy of
+//    each unit's piece into a free stage as soon as the address is known,
+//    before the flags have arrived (a frame they then zero everywhere is
+//    copied for nothing), and publishes the unit -- which of its output
+//    copies are zero -- with its arrival on the stage once they have;
+//  - warp 1 collates this CTA's samples (k = blockIdx.x mod grid): action,
+//    reward, done, gathered scalars, the importance weight, and the index
+//    when the batch is drawn here;
+//  - warps 2 .. kStageWarps + 1 (consumers) wait for the stage, turn its
+//    bytes into floats and store them to obs and / or next_obs (zeros where
+//    the episode mask says so; each warp-wide store writes 512 contiguous
+//    bytes), then release the stage.
+// A stage's phase completes when the producer has arrived and the copy's
+// bytes have landed.  kStages stages keep several pieces in flight per CTA,
+// so the index -> flags chain is paid once per 32 units, beside the copies.
+// Every wait is bounded (kWaitNs): on expiry the warp records DEVERR_TIMEOUT
+// and stops, the producer after waiting (bounded again) for the copies it
+// has in flight.
+// ---------------------------------------------------------------------------
+constexpr int kStages = 6;
+constexpr uint32_t kPiece = 7168;  // bytes per stage, a multiple of 16
+constexpr int kStageWarps = 7;     // consumer warps
+constexpr int kStagedThreads = 32 * (kStageWarps + 2);
+constexpr int kStagedPerSm = 2;    // CTAs per SM in the grid
+constexpr int kStagedUnroll = 4;
+constexpr uint64_t kWaitNs = 1000000000ull;
+// unit flags (StageSmem::meta)
+constexpr uint32_t kZeroObs = 1u, kZeroNext = 2u, kLoaded = 4u;
+
+struct StageSmem {
+  alignas(128) uint8_t buf[kStages][kPiece];
+  unsigned long long full[kStages];   // producer -> consumers (bytes landed)
+  unsigned long long empty[kStages];  // consumers -> producer (stage free)
+  uint32_t meta[kStages];
+};
+
+// Collate of samples first, first + stride, ... (one warp): q_min over the
+// batch once, then one sample per lane.
+__device__ void collate_strided(const Common &c, uint32_t first, uint32_t stride, int lane) {
+  const uint32_t m = c.isw ? batch_qmin(c, lane) : 0u;
+  for (uint64_t k = first + (uint64_t)lane * stride; k < c.B; k += 32ull * stride) {
+    uint64_t slot = 0, off = 0;
+    const bool ok = sample_slot(c, (uint32_t)k, &slot, &off, true);
+    if (c.act_out) c.act_out[k] = ok ? c.action[slot] : 0;
+    if (c.rew_out) c.rew_out[k] = ok ? c.reward[slot] : 0.f;
+    if (c.done_out) c.done_out[k] = ok ? c.done[slot] : (uint8_t)0;
+    if (c.gdst0) c.gdst0[k] = ok ? c.gsrc0[off] : 0.f;
+    if (c.gdst1) c.gdst1[k] = ok ? c.gsrc1[off] : 0.f;
+    if (c.isw) c.isw[k] = is_weight(m, c.q[k], c.beta);
+  }
+}
+
+// Unit u -> (sample k, frame m, piece p).
+struct Unit {
+  uint32_t k, m, p;
+};
+__device__ __forceinline__ Unit unit_of(uint64_t u, uint32_t U, uint32_t npieces) {
+  const uint32_t per_k = U * npieces;
+  Unit r;
+  r.k = (uint32_t)(u / per_k);
+  const uint32_t rem = (uint32_t)(u - (uint64_t)r.k * per_k);
+  r.m = rem / npieces;
+  r.p = rem - r.m * npieces;
+  return r;
+}
+
+__device__ void stage_producer(const Common &c, const StackArgs &a, StageSmem &sm,
+                               uint32_t npieces, uint32_t piece, uint64_t nmine,
+                               int lane, uint64_t pol) {
+  for (uint64_t i0 = 0; i0 < nmine; i0 += 32) {
+    // lane l resolves unit i0 + l of this CTA: its source now, its episode
+    // flags in flight (used when the unit is published)
+    uint64_t src = 0;
+    bool valid = false, ok = false, has_obs = false, has_next = false;
+    int64_t span = 0;
+    uint32_t bits = 0;
+    if (i0 + lane < nmine) {
+      valid = true;
+      const Unit t = unit_of(blockIdx.x + (i0 + lane) * gridDim.x, a.U, npieces);
+      uint64_t slot = 0, off = 0;
+      ok = sample_slot(c, t.k, &slot, &off, false);
+      const int64_t j = (int64_t)off - (int64_t)(a.K - 1) + (int64_t)t.m;
+      has_obs = t.m < a.K;
+      has_next = a.next && t.m >= 1;
+      if (ok && j >= 0) {
+        uint64_t js = c.oldest + (uint64_t)j;
+        if (js >= c.cap) js -= c.cap;
+        src = (uint64_t)(a.frames + js * a.F + (uint64_t)t.p * piece);
+        span = (int64_t)off - j + 1;  // flags of offsets j .. off (<= K)
+      } else {
+        ok = false;  // zero in every copy
+      }
+      // bit i: done flag of offset j + i
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        if (i < span) {
+          uint64_t ps = c.oldest + (uint64_t)(off - (uint64_t)(span - 1)) + i;
+          if (ps >= c.cap) ps -= c.cap;
+          bits |= (c.done[ps] != 0 ? 1u : 0u) << i;
+        }
+      }
+    }
+    const uint32_t n = (uint32_t)min((uint64_t)32, nmine - i0);
+    uint32_t pub = 0;  // units of the group published so far
+    uint32_t good = 1;
+    // this lane's unit flags: an episode end before the anchor zeroes the
+    // frame in obs and next_obs; one at the anchor zeroes it in next_obs
+    // only (evaluated when the first unit is published: the flag loads are
+    // in flight until then)
+    uint32_t fl = 0;
+    bool fl_ready = false;
+#define EDP_PUBLISH()                                                            \
+    do {                                                                         \
+      if (!fl_ready) {                                                           \
+        const bool end_before = span > 1 && (bits & ((1u << (span - 1)) - 1u)) != 0; \
+        const bool end_at = span > 0 && ((bits >> (span - 1)) & 1u);             \
+        const bool zo = !ok || end_before, zn = zo || end_at;                    \
+        const bool load = (has_obs && !zo) || (has_next && !zn);                 \
+        fl = valid ? (zo ? kZeroObs : 0u) | (zn ? kZeroNext : 0u) | (load ? kLoaded : 0u) \
+                   : 0u;                                                         \
+        fl_ready = true;                                                         \
+      }                                                                          \
+      const uint32_t fl_t = __shfl_sync(kFull, fl, pub);                         \
+      if (lane == 0) {                                                           \
+        const int st_p = (int)((i0 + pub) % kStages);                            \
+        sm.meta[st_p] = fl_t;                                                    \
+        mbar_arrive(&sm.full[st_p]);                                             \
+      }                                                                          \
+      ++pub;                                                                     \
+    } while (0)
+    uint32_t t = 0;
+    for (; t < n; ++t) {
+      const uint64_t i = i0 + t;
+      const int st = (int)(i % kStages);
+      if (i >= kStages) {
+        // the stage's previous occupant (unit i - kStages) must have been
+        // published before the consumers can free the stage
+        while (pub + kStages <= t) EDP_PUBLISH();
+        if (lane == 0)
+          good = mbar_wait(&sm.empty[st], (uint32_t)((i / kStages) - 1) & 1u, kWaitNs);
+        good = __shfl_sync(kFull, good, 0);
+        if (!good) break;
+      }
+      const uint64_t src_t = __shfl_sync(kFull, src, t);
+      if (lane == 0 && src_t) {
+        mbar_expect_tx(&sm.full[st], piece);
+        bulk_load(sm.buf[st], reinterpret_cast<const void *>(src_t), piece, &sm.full[st], pol);
+      }
+    }
+    if (!good) {
+      // units i0 + pub .. i0 + t - 1 are issued but unpublished: publish
+      // them so their phases can complete, then wait (bounded) for the
+      // bytes of the last kStages issued copies, which land in this CTA's
+      // shared memory, before the CTA may exit
+      while (pub < t) EDP_PUBLISH();
+      if (lane == 0) {
+        const uint64_t end = i0 + t;
+        flag(c.ctrl, DEVERR_TIMEOUT, end);
+        for (uint64_t q = end > kStages ? end - kStages : 0; q < end; ++q)
+          mbar_wait(&sm.full[q % kStages], (uint32_t)(q / kStages) & 1u, kWaitNs);
+      }
+      return;
+    }
+    while (pub < n) EDP_PUBLISH();
+#undef EDP_PUBLISH
+  }
+}
+
+__device__ void stage_consumer(const Common &c, const StackArgs &a, StageSmem &sm,
+                               uint32_t npieces, uint32_t piece, uint64_t nmine,
+                               int cw, int lane, uint64_t pol) {
+  const float4 zero4 = make_float4(0.f, 0.f, 0.f, 0.f);
+  const uint32_t W = piece / 4;  // words of a piece
+  constexpr uint32_t kRow = 32 * kStageWarps;
+  for (uint64_t i = 0; i < nmine; ++i) {
+    const int st = (int)(i % kStages);
+    if (!mbar_wait(&sm.full[st], (uint32_t)(i / kStages) & 1u, kWaitNs)) {
+      if (lane == 0) flag(c.ctrl, DEVERR_TIMEOUT, i);
+      return;
+    }
+    const uint32_t fl = sm.meta[st];
+    const Unit t = unit_of(blockIdx.x + i * gridDim.x, a.U, npieces);
+    const bool zo = fl & kZeroObs, zn = fl & kZeroNext, loaded = fl & kLoaded;
+    const uint64_t pofs = (uint64_t)t.p * piece;
+    float4 *dobs = t.m < a.K ? reinterpret_cast<float4 *>(
+                                   a.obs + ((uint64_t)t.k * a.K + t.m) * a.F + pofs)
+                             : nullptr;
+    float4 *dnext = (a.next && t.m >= 1)
+                        ? reinterpret_cast<float4 *>(
+                              a.next + ((uint64_t)t.k * a.K + t.m - 1) * a.F + pofs)
+                        : nullptr;
+    const uint32_t *src = reinterpret_cast<const uint32_t *>(sm.buf[st]);
+    for (uint32_t w0 = cw * 32 + lane; w0 < W; w0 += kRow * kStagedUnroll) {
+      uint32_t v[kStagedUnroll];
+#pragma unroll
+      for (int u = 0; u < kStagedUnroll; ++u) {
+        const uint32_t w = w0 + u * kRow;
+        v[u] = (loaded && w < W) ? src[w] : 0u;
+      }
+#pragma unroll
+      for (int u = 0; u < kStagedUnroll; ++u) {
+        const uint32_t w = w0 + u * kRow;
+        if (w >= W) continue;
+        float4 fv;
+        fv.x = unit_f32(byte_f(v[u], 0), c.r1, c.r2);
+        fv.y = unit_f32(byte_f(v[u], 1), c.r1, c.r2);
+        fv.z = unit_f32(byte_f(v[u], 2), c.r1, c.r2);
+        fv.w = unit_f32(byte_f(v[u], 3), c.r1, c.r2);
+        if (dobs) st_stream(dobs + w, zo ? zero4 : fv, pol);
+        if (dnext) st_stream(dnext + w, zn ? zero4 : fv, pol);
+      }
+    }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&sm.empty[st]);
+  }
+}
+
+__global__ void __launch_bounds__(kStagedThreads)
+k_deliver_stack_staged(Common c, StackArgs a, uint32_t npieces, uint32_t piece) {
+  __shared__ StageSmem sm;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   if (threadIdx.x == 0) {
-    const uint32_t first = work_first(c.work, c.work_tag);
-    s_owned = first != kWorkFixed;
-    s_chunk[0] = first != kWorkFixed ? first : blockIdx.x;
+    for (int i = 0; i < kStages; ++i) {
+      mbar_init(&sm.full[i], 1);
+      mbar_init(&sm.empty[i], kStageWarps);
+    }
+    mbar_init_fence();
   }
   __syncthreads();
-  const bool owned = s_owned != 0;
-  uint32_t cur = s_chunk[0];
-  for (int p = 1;; p ^= 1) {
-    const uint64_t f0 = (uint64_t)cur * per_chunk;
-    if (f0 >= total) break;  // uniform across the CTA
-    uint32_t nxt = 0;
-    if (threadIdx.x == 0) nxt = owned ? work_claim(c.work, c.work_tag) : cur + gridDim.x;
-    const uint64_t f = f0 + (uint64_t)warp * a.span;
-    if (f < total) stack_span<UN>(c, a, f, min(total, f + a.span), lane, pol, true);
-    if (threadIdx.x == 0) s_chunk[p] = nxt;
-    __syncthreads();
-    cur = s_chunk[p];
-  }
+  const uint64_t pol = policy_stream();
+  pdl_wait();
+  pdl_launch();
+  const uint64_t units = (uint64_t)c.B * a.U * npieces;
+  const uint64_t nmine =
+      units > blockIdx.x ? (units - blockIdx.x + gridDim.x - 1) / gridDim.x : 0;
+  if (warp == 0)
+    stage_producer(c, a, sm, npieces, piece, nmine, lane, pol);
+  else if (warp == 1)
+    collate_strided(c, blockIdx.x, gridDim.x, lane);
+  else
+    stage_consumer(c, a, sm, npieces, piece, nmine, warp - 2, lane, pol);
 }
 
 // ---------------------------------------------------------------------------
@@ -669,35 +818,25 @@ cudaError_t launch_deliver(edp_ctx *ctx, const int64_t *idx, uint32_t B,
     a.obs = (float *)out->obs;
     a.next = (float *)out->next_obs;
     a.U = a.K + (a.next ? 1 : 0);
+    // equal pieces: the fewest that divide the frame's 16-byte runs and fit
+    // a stage
+    const uint32_t runs = a.F / 16;
+    uint32_t np = (a.F + kPiece - 1) / kPiece;
+    while (runs % np) ++np;
+    const uint64_t staged_units = (uint64_t)B * a.U * np;
+    const uint64_t staged_grid = (uint64_t)kStagedPerSm * sms;
+    if (staged_units >= 2 * staged_grid) {
+      return launch_pdl(k_deliver_stack_staged, dim3((unsigned)staged_grid),
+                        dim3(kStagedThreads), s, c, a, np, a.F / np);
+    }
+    // a small batch: one span of one unrolled iteration per warp, one chunk
+    // per CTA, and the collate CTA
+    a.span = 32 * kStackUnroll;
     const uint64_t units = (uint64_t)B * a.U * a.W;
-    auto kern = k_deliver_stack<kStackUnroll>;
-    static int per_sm = 0;
-    if (!per_sm) {
-      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, 0);
-      if (per_sm < 1) per_sm = 1;
-    }
-    const int resident = per_sm > kStackHeadroom ? per_sm - kStackHeadroom : 1;
-    uint64_t grid = (uint64_t)resident * sms;
-    auto n_chunks = [&](uint32_t span) {
-      return (units + (uint64_t)kWarps * span - 1) / ((uint64_t)kWarps * span);
-    };
-    a.span = 32 * kStackUnroll * kStackIters;
-    uint64_t chunks = n_chunks(a.span);
-    if (chunks < grid) {  // a small batch: one iteration per warp, more CTAs
-      a.span = 32 * kStackUnroll;
-      chunks = n_chunks(a.span);
-    }
-    if (grid >= chunks || chunks + grid >= kWorkMaxChunks) {
-      grid = chunks + 1;  // one chunk per CTA and the collate CTA, no work word
-      if (grid > 0x7FFFFFFFull) return cudaErrorInvalidValue;
-      return launch_pdl(kern, dim3((unsigned)grid), dim3(kThreads), s, c, a);
-    }
-    const uint64_t seq = ctx->work_seq++;
-    c.work = ctx->ctrl->work + (seq % kWorkSlots);
-    c.work_tag = seq % ((1ull << (64 - kWorkTagShift)) - 1) + 1;
-    cudaError_t e = launch_pdl(kern, dim3((unsigned)grid), dim3(kThreads), s, c, a);
-    if (e != cudaSuccess) return e;
-    return launch_pdl(k_work_release, dim3(1), dim3(32), s, c.work, c.work_tag);
+    const uint64_t chunks = (units + (uint64_t)kWarps * a.span - 1) / ((uint64_t)kWarps * a.span);
+    if (chunks + 1 > 0x7FFFFFFFull) return cudaErrorInvalidValue;
+    return launch_pdl(k_deliver_stack<kStackUnroll>, dim3((unsigned)(chunks + 1)),
+                      dim3(kThreads), s, c, a);
   } else if (cfg.transform == EDP_XFORM_HWC_CHW_BF16) {
     ChwArgs a{};
     a.obs = ctx->st.obs;

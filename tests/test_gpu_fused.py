@@ -2,7 +2,7 @@
 C ABI: the same indices as edp_sample(UNIFORM) with the same seed and round
 (and as the oracle's sampler), and outputs bit-identical to edp_deliver of
 those indices, for the three transforms -- frame stacks (one chunk per CTA
-and the work-counter path), HWC -> CHW bf16, and normalised bf16 over a
+and the staged path), HWC -> CHW bf16, and normalised bf16 over a
 two-tier ring; plus its argument errors."""
 import numpy as np
 import pytest

@@ -30,7 +30,7 @@ def test_frame_stack_per_into_host(edp_lib, orc):
     m = MirroredDqn(1200, prioritized=True)
     for sl in (slice(0, 700), slice(700, 1500)):  # wraps the ring
         m.ingest(orc, frames[sl], action[sl], reward[sl], done[sl], q=q[sl])
-    for B in (32, 700):  # one chunk per CTA, and the work-counter path
+    for B in (32, 700):  # one chunk per CTA, and the staged path
         idx = torch.empty(B, dtype=torch.int64, device="cuda")
         qs = torch.empty(B, dtype=torch.int32, device="cuda")
         edp.edp_sample(m.ring.ctx, edp.EDP_SAMPLE_PRIORITIZED, B, 5, B, idx, qs)

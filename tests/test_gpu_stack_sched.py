@@ -1,16 +1,13 @@
-"""The work-word path of the frame-stack delivery.
+"""The staged path of the frame-stack delivery, under concurrency.
 
-A batch with more work chunks than the delivery's persistent grid holds is
-handed out chunk by chunk from one of the context's 32 work words (chosen
-round robin at issue; a word is claimed by the launch's own grid id, and a
-CTA that finds another launch working from its word takes a fixed share of
-the chunks instead).  Here a batch of 1,024 stacks (about 2,900 chunks) is
-delivered many times: from two streams at once, and more than 32 times in a
-row inside a CUDA graph, so every word is reused; and 40 deliveries that may
-all run at once -- released together on eight streams, eagerly and from a
-graph replayed twice -- so that launches 32 apart share a word while both
-run.  Every delivery must equal the first bit for bit, and the first must
-equal the oracle on a strided sample of rows.
+A batch that fills the GPU (here 1,024 stacks, 5,120 frame pieces) is
+delivered by the staged kernel: pieces are dealt to the CTAs round robin,
+so a launch shares no state with any other and leaves none behind.  Here it
+is delivered many times: from two streams at once, 40 times in a row inside
+a CUDA graph, and 40 deliveries that may all run at once -- released
+together on eight streams, eagerly and from a graph replayed twice.  Every
+delivery must equal the first bit for bit, and the first must equal the
+oracle on a strided sample of rows.
 """
 import numpy as np
 import pytest
@@ -23,7 +20,7 @@ pytestmark = pytest.mark.gpu
 B, CAP, N_INGEST = 1024, 3000, 2900
 
 
-def test_concurrent_and_repeated_counter_deliveries(edp_lib, orc):
+def test_concurrent_and_repeated_staged_deliveries(edp_lib, orc):
     edp = edp_lib
     frames, action, reward, done = fx.dqn_transitions(40, N_INGEST, done_p=0.05)
     m = MirroredDqn(CAP)
@@ -57,7 +54,7 @@ def test_concurrent_and_repeated_counter_deliveries(edp_lib, orc):
     assert np.array_equal(ref[2][sel], r_act)
     assert np.array_equal(ref[3][sel], r_rew.view(np.uint32))
     assert np.array_equal(ref[4][sel], r_dn)
-    # 40 launches in one graph (every counter pair used at least once more),
+    # 40 launches in one graph,
     # alternating between two output sets; the last two must equal ref
     g = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g, capture_error_mode="thread_local"):
@@ -78,7 +75,7 @@ def test_concurrent_and_repeated_counter_deliveries(edp_lib, orc):
 def test_outputs_16_byte_aligned_only(edp_lib, orc, B):
     """Outputs 16 bytes past a 32-byte boundary (the alignment the ABI
     requires, and no more) give the same batches as aligned ones, on the
-    one-chunk-per-CTA and the counter paths."""
+    one-chunk-per-CTA and the staged paths."""
     edp = edp_lib
     frames, action, reward, done = fx.dqn_transitions(42, N_INGEST, done_p=0.05)
     m = MirroredDqn(CAP)
