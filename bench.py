@@ -1,16 +1,21 @@
 #!/usr/bin/env python3
 """Benchmark of the experience-path hot path on one GB300 (or N replicas).
 
-Default workload: prioritized replay over 1,000,000 uint8 84x84 frames
-(~7.06 GB in HBM), batch 512, frame stack 4, PER priorities from Exp(1) TD
-errors.  One step = one round of the hot path: stratified sampling through
-the sum-tree, fused frame-stack delivery of obs and next_obs as fp32 with
-collate and importance weights, and the priority update from fresh TD
-errors.  Other workloads (--workload) are for measurement by hand.
+Default workload (the largest HBM-resident configuration): multimodal
+replay over 200,000 transitions of a uint8 3x224x224 image, 512 int32
+tokens and a reward (~30.5 GB in HBM), uniform batch 1,024 delivered as
+per-channel normalised bf16 with collated tokens and rewards.  One step =
+one round of the hot path: the uniform draw and the fused gather +
+normalise + collate.  Other workloads (--workload): prioritized replay over
+1,000,000 84x84 frames (per1m: stratified sampling through the sum-tree,
+frame-stack delivery of obs and next_obs as fp32 with importance weights,
+priority update), the tiny DQN replay, the PPO iteration, the two-tier ring
+beyond HBM and the GRPO batch.
 
 Prints ONE JSON line (rank 0).  `value` = delivered GB/s (algorithmic bytes
 of the rounds / device time), `e2e` = the same through the C ABI with host
-buffers (TD errors copied in, the learner batch copied out every step).
+buffers (inputs copied in and the learner batch written to host memory
+every step).
 
 --impl reference times the CPU oracle (plain C, all host cores) on the same
 workload and metric; each step is one round of the same per-round work.
@@ -324,7 +329,7 @@ class PerReplay(Workload):
     512, frame stack 4, obs + next_obs fp32, PER alpha 0.6 / beta 0.4 with
     priorities from Exp(1) TD errors; step = sample, deliver, update."""
     name = "per-replay-1M-84x84-B512"
-    kernel = "k_deliver_stack"
+    kernel = "k_deliver_stack_staged"
     dtype = "u8->f32"
     launches_per_round = 3
 
@@ -1269,12 +1274,7 @@ class MmReplay(Workload):
         x = self.F + 4 * self.L
         ring_bytes = self.cap * x
         mem_gpu = bw["hbm_free"] + ring_bytes - 8e9  # this ring's HBM is the buffer's
-        avail = 0.0
-        with open("/proc/meminfo") as f:
-            for line in f:
-                if line.startswith("MemAvailable:"):
-                    avail = float(line.split()[1]) * 1024
-        mem_host = 0.8 * avail
+        mem_host = 0.8 * _mem_available()
         def best_of(fn, k=3):
             t = []
             for _ in range(k):
@@ -1402,14 +1402,29 @@ class MmReplay(Workload):
                     "predicted_ranking": [names[i] for i in sorted(range(4),
                                                                    key=lambda i: (t_pred[i], i))]}}
 
-    def cpu_setup(self, host_rows=16384):
+    def cpu_setup(self, host_rows=None):
+        """The oracle's host ring: by default at least 16 GB of images
+        (110,000 rows, 16.6 GB), so its gathers miss the host caches as the
+        GPU's miss L2; filled from one 256 MB random block (the timing does
+        not depend on the byte values).  Capped at the capacity and at a
+        quarter of the host's available memory."""
         import numpy as np
         import oracle as orc
         from paper_2609_24456_gb300 import fixtures as fx
         self.orc = orc
-        self.hrows = min(host_rows, self.cap)
+        if host_rows is None:
+            host_rows = 110_000
+            avail = _mem_available()
+            if avail:
+                host_rows = min(host_rows, int(avail // 4 // self.F))
+        self.hrows = max(1, min(host_rows, self.cap))
         rng = np.random.default_rng(self.seed)
-        self.h_obs = rng.integers(0, 256, size=(self.hrows, self.F), dtype=np.uint8)
+        block = rng.integers(0, 256, size=(min(self.hrows, max(1, (256 << 20) // self.F)),
+                                           self.F), dtype=np.uint8)
+        self.h_obs = np.empty((self.hrows, self.F), dtype=np.uint8)
+        for lo in range(0, self.hrows, len(block)):
+            n = min(len(block), self.hrows - lo)
+            self.h_obs[lo:lo + n] = block[:n]
         self.h_tok, self.h_rew = fx.mm_metadata(self.seed, self.hrows, tokens=self.L)
         if self.ingest:
             self.h_stage = rng.integers(0, 256, size=(self.ingest, self.F), dtype=np.uint8)
@@ -1590,6 +1605,18 @@ WORKLOADS = {
 
 
 # ----------------------------------------------------------------------------
+def _mem_available():
+    """MemAvailable of this host in bytes (0 if unknown)."""
+    try:
+        with open("/proc/meminfo") as f:
+            for line in f:
+                if line.startswith("MemAvailable:"):
+                    return float(line.split()[1]) * 1024
+    except OSError:
+        pass
+    return 0.0
+
+
 def time_cpu(wl, budget_s, min_rounds=3):
     wl.cpu_round(0)
     n, t0 = 0, time.perf_counter()
@@ -1819,7 +1846,9 @@ def main():
     ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", default="edp", choices=["edp", "reference"])
-    ap.add_argument("--workload", default="per1m", choices=sorted(WORKLOADS))
+    # default: the largest HBM-resident configuration (200,000 multimodal
+    # transitions, ~30 GB), whose metric is the fraction of HBM bandwidth
+    ap.add_argument("--workload", default="mm200k", choices=sorted(WORKLOADS))
     ap.add_argument("--capacity", type=int, default=0,
                     help="override the ring capacity (profiling small cases)")
     ap.add_argument("--no-graph", action="store_true")
