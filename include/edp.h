@@ -13,6 +13,9 @@
  *   delivery   -> edp_sample            (uniform, prioritized, shuffle)
  *                 edp_deliver           (gather + transform + collate)
  *   callback   -> edp_update_priorities / edp_update_priorities_td
+ *   sharding   -> edp_tree_total, edp_route_prioritized, edp_sample_targets,
+ *                 edp_batch_qmin, edp_is_weights, edp_gae_stats,
+ *                 edp_gae_normalize (a buffer split across GPUs, Sec. 5.1)
  *
  * Conventions shared by every call
  * --------------------------------
@@ -355,6 +358,101 @@ EDP_API edp_status edp_gae(edp_ctx *ctx, const float *r, const float *v,
                    const uint8_t *d, uint32_t T, uint32_t E, double gamma,
                    double lambda, float *adv, float *ret, float *adv_norm,
                    edp_stream stream);
+
+/* ---------------------------------------------------------------------------
+ * Sharded buffer (Sec. 5.1, the shared-GPU placement: a node's GPUs each hold
+ * a share of the ring's slots and every learner samples the whole buffer, so
+ * most of a batch is fetched from other GPUs).  G ranks each hold one
+ * context (a shard).  The global prioritized distribution is that of one
+ * buffer whose leaves are the shards' leaves in shard-major order (all of
+ * shard 0's physical slots, then shard 1's, ...), so a shard holds a
+ * contiguous block of the global inverse CDF.  One round, for a global batch
+ * of B split into consecutive strata per learner:
+ *   1. edp_tree_total on every shard; the caller all-gathers the G totals;
+ *   2. each learner: edp_route_prioritized over its strata -> local targets,
+ *      grouped by owning shard, and per-shard counts; the caller exchanges
+ *      the counts and then the targets (all-to-all);
+ *   3. each owner: edp_sample_targets on the targets it received, in source
+ *      rank order, then edp_deliver of those slots; the caller sends the rows
+ *      (and slots and priorities) back with the reverse all-to-all -- they
+ *      arrive at each learner in stratum order;
+ *   4. each learner: edp_batch_qmin, a minimum over ranks by the caller, and
+ *      edp_is_weights with that global minimum;
+ *   5. priority updates travel to the owners in the same grouping and are
+ *      applied with edp_update_priorities* (source rank order = global batch
+ *      order, so the last occurrence of a slot still wins).
+ * The indices, priorities, weights and rows equal those of a single buffer
+ * holding all shards' leaves.  For on-policy rollouts sharded by
+ * environment, edp_gae_stats gives each rank's (n, sum A, sum A^2); the
+ * caller sums them over the ranks and edp_gae_normalize normalises with the
+ * totals.  These calls never communicate: the exchanges are the caller's
+ * (e.g. NCCL through torch.distributed).
+ * ------------------------------------------------------------------------- */
+
+/* Total priority S of this context's tree (device uint64 [1]).
+ * EDP_ERR_STATE for a context without priorities; EDP_ERR_INVALID when
+ * d_total is not device memory. */
+EDP_API edp_status edp_tree_total(edp_ctx *ctx, uint64_t *d_total, edp_stream stream);
+
+/* Stratified targets of strata k0 .. k0+n-1 of a global batch of `batch`
+ * over G shard totals (device uint64 [G], shard order), as edp_sample
+ * (PRIORITIZED) draws them over a single buffer (same seed, round and Philox
+ * stream), each routed to the shard whose prefix range holds it:
+ * d_local_t[i] (device uint64 [n]) = target - (totals of the shards before
+ * the owner), in stratum order -- which groups them by owner, ascending --
+ * and d_counts[s] (device int64 [G]) = strata owned by shard s.  The
+ * context only names the GPU and receives device-side flags: an all-zero
+ * total (DEVERR_EMPTY, edp_sync -> EDP_ERR_EMPTY) or a sum of totals beyond
+ * 64 bits (DEVERR_OVERFLOW) routes nothing (counts 0, targets 2^64-1).
+ * EDP_ERR_INVALID when G is 0 or above 1024, batch is 0, k0 + n > batch, or
+ * a pointer is not device memory. */
+EDP_API edp_status edp_route_prioritized(edp_ctx *ctx, const uint64_t *d_totals, uint32_t G,
+                                         uint32_t batch, uint32_t k0, uint32_t n,
+                                         uint64_t seed, uint64_t round, uint64_t *d_local_t,
+                                         int64_t *d_counts, edp_stream stream);
+
+/* Tree descent of n given targets (device uint64 [n], each below this
+ * shard's total): d_idx (device int64 [n]) = the physical slot whose
+ * prefix range holds the target, d_q (device uint32 [n] or NULL) = its
+ * priority.  A target at or above the total gives idx -1, q 0 and a device
+ * flag (edp_sync -> EDP_ERR_INVALID).  EDP_ERR_STATE without priorities;
+ * EDP_ERR_INVALID for pointers outside device memory.  n == 0 does nothing. */
+EDP_API edp_status edp_sample_targets(edp_ctx *ctx, const uint64_t *d_targets, uint32_t n,
+                                      int64_t *d_idx, uint32_t *d_q, edp_stream stream);
+
+/* Minimum of d_q[0..n) (device uint32) into d_qmin (device int64 [1]);
+ * 2^32 - 1 for n == 0.  EDP_ERR_INVALID for pointers outside device memory. */
+EDP_API edp_status edp_batch_qmin(edp_ctx *ctx, const uint32_t *d_q, uint32_t n,
+                                  int64_t *d_qmin, edp_stream stream);
+
+/* Importance weights of a batch whose priority minimum is given:
+ * d_w[k] = (q_min / d_q[k])^beta in fp64, rounded once to fp32, with q_min =
+ * *d_qmin (device int64, e.g. the minimum over every rank's share of a global
+ * batch) -- the weights edp_deliver computes with q_min over its own batch.
+ * EDP_ERR_INVALID for beta < 0 or pointers outside device memory.  n == 0
+ * does nothing. */
+EDP_API edp_status edp_is_weights(edp_ctx *ctx, const uint32_t *d_q, uint32_t n,
+                                  const int64_t *d_qmin, double beta, float *d_w,
+                                  edp_stream stream);
+
+/* edp_gae without the normalisation, for environments sharded over ranks:
+ * writes adv (required) and ret (or NULL) as edp_gae does, and d_stats
+ * (device double [3]) = (T*E, sum of A, sum of A^2) over this rank's
+ * values.  Errors as edp_gae, and EDP_ERR_INVALID when adv or d_stats is
+ * NULL. */
+EDP_API edp_status edp_gae_stats(edp_ctx *ctx, const float *r, const float *v,
+                                 const uint8_t *d, uint32_t T, uint32_t E, double gamma,
+                                 double lambda, float *adv, float *ret, double *d_stats,
+                                 edp_stream stream);
+
+/* adv_norm[i] = (adv[i] - mean) / (std + 1e-8) for i < n, with mean and the
+ * unbiased std from d_stats = (N, sum A, sum A^2) (device double [3]: the
+ * sums of every rank's edp_gae_stats); N == 1 gives 0.  adv and adv_norm
+ * device float [n] (they may be the same array).  EDP_ERR_INVALID for n == 0,
+ * n >= 2^31 or pointers outside device memory. */
+EDP_API edp_status edp_gae_normalize(edp_ctx *ctx, const float *adv, uint64_t n,
+                                     const double *d_stats, float *adv_norm,
+                                     edp_stream stream);
 
 /* ---------------------------------------------------------------------------
  * LLM post-training (Appendix A, Table "Verl map"): advantage computation is

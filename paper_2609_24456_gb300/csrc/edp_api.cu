@@ -7,6 +7,7 @@
 #include <cstdio>
 #include <cstdlib>
 #include <cstring>
+#include <initializer_list>
 #include <new>
 
 #include "edp_internal.cuh"
@@ -1013,6 +1014,119 @@ edp_status edp_gae(edp_ctx *ctx, const float *r, const float *v,
   return EDP_OK;
 }
 
+// ---- sharded buffer -------------------------------------------------------
+
+// true when every non-NULL pointer is device memory of the context's GPU
+static bool all_device(const edp_ctx *ctx, std::initializer_list<const void *> ps) {
+  const void *p;
+  for (const void *o : ps)
+    if (o && !device_view(ctx, o, &p, false)) return false;
+  return true;
+}
+
+edp_status edp_tree_total(edp_ctx *ctx, uint64_t *d_total, edp_stream stream) {
+  if (!ctx) return EDP_ERR_INVALID;
+  if (!ctx->depth) return fail(ctx, EDP_ERR_STATE, "edp_tree_total: context has no priorities");
+  if (!d_total || !all_device(ctx, {d_total}))
+    return fail(ctx, EDP_ERR_INVALID, "edp_tree_total: d_total must be device memory");
+  DeviceGuard dg(ctx->cfg.device);
+  cudaError_t e = launch_tree_total(ctx, d_total, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_tree_total");
+  return EDP_OK;
+}
+
+edp_status edp_route_prioritized(edp_ctx *ctx, const uint64_t *d_totals, uint32_t G,
+                                 uint32_t batch, uint32_t k0, uint32_t n, uint64_t seed,
+                                 uint64_t round, uint64_t *d_local_t, int64_t *d_counts,
+                                 edp_stream stream) {
+  if (!ctx) return EDP_ERR_INVALID;
+  if (G == 0 || G > 1024)
+    return fail(ctx, EDP_ERR_INVALID, "edp_route_prioritized: G must be in [1, 1024]");
+  if (batch == 0) return fail(ctx, EDP_ERR_INVALID, "edp_route_prioritized: batch == 0");
+  if ((uint64_t)k0 + n > batch)
+    return fail(ctx, EDP_ERR_INVALID, "edp_route_prioritized: k0 + n > batch");
+  if (!d_totals || !d_counts || (n && !d_local_t) ||
+      !all_device(ctx, {d_totals, d_counts, d_local_t}))
+    return fail(ctx, EDP_ERR_INVALID,
+                "edp_route_prioritized: totals, local targets and counts must be device memory");
+  DeviceGuard dg(ctx->cfg.device);
+  cudaError_t e = launch_route_prioritized(ctx, d_totals, G, batch, k0, n, seed, round,
+                                           d_local_t, d_counts, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_route_prioritized");
+  return EDP_OK;
+}
+
+edp_status edp_sample_targets(edp_ctx *ctx, const uint64_t *d_targets, uint32_t n,
+                              int64_t *d_idx, uint32_t *d_q, edp_stream stream) {
+  if (!ctx) return EDP_ERR_INVALID;
+  if (!ctx->depth)
+    return fail(ctx, EDP_ERR_STATE, "edp_sample_targets: context has no priorities");
+  if (n == 0) return EDP_OK;
+  if (!d_targets || !d_idx || !all_device(ctx, {d_targets, d_idx, d_q}))
+    return fail(ctx, EDP_ERR_INVALID,
+                "edp_sample_targets: targets, idx and q must be device memory");
+  DeviceGuard dg(ctx->cfg.device);
+  cudaError_t e = launch_sample_targets(ctx, d_targets, n, d_idx, d_q, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_sample_targets");
+  return EDP_OK;
+}
+
+edp_status edp_batch_qmin(edp_ctx *ctx, const uint32_t *d_q, uint32_t n, int64_t *d_qmin,
+                          edp_stream stream) {
+  if (!ctx) return EDP_ERR_INVALID;
+  if (!d_qmin || (n && !d_q) || !all_device(ctx, {d_q, d_qmin}))
+    return fail(ctx, EDP_ERR_INVALID, "edp_batch_qmin: q and qmin must be device memory");
+  DeviceGuard dg(ctx->cfg.device);
+  cudaError_t e = launch_batch_qmin(ctx, d_q, n, d_qmin, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_batch_qmin");
+  return EDP_OK;
+}
+
+edp_status edp_is_weights(edp_ctx *ctx, const uint32_t *d_q, uint32_t n,
+                          const int64_t *d_qmin, double beta, float *d_w, edp_stream stream) {
+  if (!ctx) return EDP_ERR_INVALID;
+  if (!(beta >= 0.0)) return fail(ctx, EDP_ERR_INVALID, "edp_is_weights: beta must be >= 0");
+  if (n == 0) return EDP_OK;
+  if (!d_q || !d_qmin || !d_w || !all_device(ctx, {d_q, d_qmin, d_w}))
+    return fail(ctx, EDP_ERR_INVALID, "edp_is_weights: q, qmin and w must be device memory");
+  DeviceGuard dg(ctx->cfg.device);
+  cudaError_t e = launch_is_weights(ctx, d_q, n, d_qmin, beta, d_w, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_is_weights");
+  return EDP_OK;
+}
+
+edp_status edp_gae_stats(edp_ctx *ctx, const float *r, const float *v, const uint8_t *d,
+                         uint32_t T, uint32_t E, double gamma, double lambda, float *adv,
+                         float *ret, double *d_stats, edp_stream stream) {
+  if (!ctx) return EDP_ERR_INVALID;
+  if (!r || !v || !d) return fail(ctx, EDP_ERR_INVALID, "edp_gae_stats: r/v/d NULL");
+  if (!adv || !d_stats) return fail(ctx, EDP_ERR_INVALID, "edp_gae_stats: adv/stats NULL");
+  if (T == 0 || E == 0 || (uint64_t)T * E > 0x7FFFFFFFull)
+    return fail(ctx, EDP_ERR_INVALID, "edp_gae_stats: need T, E >= 1 and T*E < 2^31");
+  if (!std::isfinite(gamma) || !std::isfinite(lambda))
+    return fail(ctx, EDP_ERR_INVALID, "edp_gae_stats: gamma/lambda not finite");
+  if (!all_device(ctx, {r, v, d, adv, ret, d_stats}))
+    return fail(ctx, EDP_ERR_INVALID, "edp_gae_stats: arrays must be device memory");
+  DeviceGuard dg(ctx->cfg.device);
+  cudaError_t e = launch_gae_stats(ctx, r, v, d, T, E, gamma, lambda, adv, ret, d_stats,
+                                   (cudaStream_t)stream);
+  if (e != cudaSuccess) return launch_fail(ctx, e, "edp_gae_stats");
+  return EDP_OK;
+}
+
+edp_status edp_gae_normalize(edp_ctx *ctx, const float *adv, uint64_t n, const double *d_stats,
+                             float *adv_norm, edp_stream stream) {
+  if (!ctx) return EDP_ERR_INVALID;
+  if (n == 0 || n > 0x7FFFFFFFull)
+    return fail(ctx, EDP_ERR_INVALID, "edp_gae_normalize: need 1 <= n < 2^31");
+  if (!adv || !d_stats || !adv_norm || !all_device(ctx, {adv, d_stats, adv_norm}))
+    return fail(ctx, EDP_ERR_INVALID, "edp_gae_normalize: arrays must be device memory");
+  DeviceGuard dg(ctx->cfg.device);
+  cudaError_t e = launch_gae_normalize(ctx, adv, n, d_stats, adv_norm, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_gae_normalize");
+  return EDP_OK;
+}
+
 edp_status edp_grpo_advantage(edp_ctx *ctx, const float *r, const uint64_t *group_off,
                               uint32_t n_groups, float eps, float *adv, edp_stream stream) {
   if (!ctx) return EDP_ERR_INVALID;
@@ -1123,8 +1237,8 @@ edp_status edp_sync(edp_ctx *ctx, edp_stream stream) {
     return fail(ctx, EDP_ERR_STATE, "device: inconsistent priority tree (flags 0x%x)", h.err);
   if (h.err & DEVERR_OVERFLOW)
     return fail(ctx, EDP_ERR_INVALID,
-                "device: packed output exceeds its capacity (needed %llu, flags 0x%x)", bi,
-                h.err);
+                "device: a packed output or a sum of shard totals exceeds its capacity "
+                "(%llu, flags 0x%x)", bi, h.err);
   return fail(ctx, EDP_ERR_INVALID,
               "device: index out of range (first offender %llu, flags 0x%x)", bi, h.err);
 }

@@ -113,6 +113,20 @@ __device__ __forceinline__ uint64_t mulhi64(uint64_t a, uint64_t n) {
   return __umul64hi(a, n);
 }
 
+// Target of stratum k of B over a total S (stratified proportional
+// sampling): the stratum is [lo, hi) = [floor(kS/B), floor((k+1)S/B)),
+// computed as floor(kS/B) = ak + floor(bk/B) with S = aB + b (every term
+// below 2^64), and t = lo + mulhi64(u, hi - lo) with u the Philox draw k of
+// (seed, round, stream 1).  Targets never decrease with k.
+__device__ __forceinline__ uint64_t stratum_target(uint64_t S, uint32_t B, uint32_t k,
+                                                   uint64_t seed, uint64_t round) {
+  const uint64_t a = S / B, b = S % B;
+  const uint64_t lo = a * k + (b * k) / B;
+  const uint64_t hi = a * (k + 1) + (b * (k + 1)) / B;
+  const uint64_t u = philox_u64(seed, k, round, 1);
+  return lo + mulhi64(u, hi - lo);
+}
+
 // fl32(b/255) for an integer-valued x = b in [0, 255]: r1 + r2 is 1/255 to
 // ~2^-48 relative, and b/255 never lies that close to a rounding boundary
 // of binary32, so one fused multiply-add rounds to the correctly rounded
@@ -204,6 +218,19 @@ __device__ __forceinline__ double pow_pos(double x, double a) {
   q = fma(q, r, 1.0);
   const long long ni = (long long)n;
   return q * __longlong_as_double((ni + 1023) << 52);
+}
+
+// Importance weight (q_min / q_k)^beta in fp64, one rounding to fp32 (PER:
+// (N P(i))^-beta over its batch maximum, in which N and the total cancel).
+__device__ __forceinline__ float is_weight(uint32_t m, uint32_t qk, double beta) {
+  if (qk == m) return 1.f;
+  if (!qk) return 0.f;
+  // m / qk with an fp32 seed and two Newton steps (no fp64 divide)
+  const double d = (double)qk;
+  double y = (double)(1.0f / (float)qk);
+  y = fma(y, fma(-d, y, 1.0), y);
+  y = fma(y, fma(-d, y, 1.0), y);
+  return (float)pow_pos<false>((double)m * y, beta);
 }
 
 // L2 residency hints: payload streams through (an evict_first policy) so
@@ -409,6 +436,24 @@ cudaError_t launch_sample_uniform(edp_ctx *ctx, uint32_t B, uint64_t seed,
 cudaError_t launch_sample_prioritized(edp_ctx *ctx, uint32_t B, uint64_t seed,
                                       uint64_t round, int64_t *idx,
                                       uint32_t *q, cudaStream_t s);
+// Sharded buffer (k_tree.cu, k_shard.cu)
+cudaError_t launch_sample_targets(edp_ctx *ctx, const uint64_t *targets, uint32_t n,
+                                  int64_t *idx, uint32_t *q, cudaStream_t s);
+cudaError_t launch_tree_total(edp_ctx *ctx, uint64_t *total, cudaStream_t s);
+cudaError_t launch_route_prioritized(edp_ctx *ctx, const uint64_t *totals, uint32_t G,
+                                     uint32_t B, uint32_t k0, uint32_t n, uint64_t seed,
+                                     uint64_t round, uint64_t *local_t, int64_t *counts,
+                                     cudaStream_t s);
+cudaError_t launch_batch_qmin(edp_ctx *ctx, const uint32_t *q, uint32_t n, int64_t *qmin,
+                              cudaStream_t s);
+cudaError_t launch_is_weights(edp_ctx *ctx, const uint32_t *q, uint32_t n,
+                              const int64_t *qmin, double beta, float *w, cudaStream_t s);
+cudaError_t launch_gae_stats(edp_ctx *ctx, const float *r, const float *v,
+                             const uint8_t *d, uint32_t T, uint32_t E, double gamma,
+                             double lambda, float *adv, float *ret, double *stats,
+                             cudaStream_t s);
+cudaError_t launch_gae_normalize(edp_ctx *ctx, const float *adv, uint64_t n,
+                                 const double *stats, float *adv_norm, cudaStream_t s);
 cudaError_t launch_permute(edp_ctx *ctx, uint32_t n, uint64_t seed,
                            uint64_t round, int64_t *idx, cudaStream_t s);
 cudaError_t launch_update(edp_ctx *ctx, const int64_t *idx, const uint32_t *q,

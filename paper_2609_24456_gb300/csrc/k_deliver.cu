@@ -115,18 +115,6 @@ __device__ __forceinline__ uint32_t batch_qmin(const Common &c, int lane) {
   return m;
 }
 
-// Importance weight (q_min / q_k)^beta in fp64, one rounding to fp32.
-__device__ __forceinline__ float is_weight(uint32_t m, uint32_t qk, double beta) {
-  if (qk == m) return 1.f;
-  if (!qk) return 0.f;
-  // m / qk with an fp32 seed and two Newton steps (no fp64 divide)
-  const double d = (double)qk;
-  double y = (double)(1.0f / (float)qk);
-  y = fma(y, fma(-d, y, 1.0), y);
-  y = fma(y, fma(-d, y, 1.0), y);
-  return (float)pow_pos<false>((double)m * y, beta);
-}
-
 // Per-sample collate, importance weight and scalar gathers (one warp).  The
 // head warp of each sample runs this before its payload span, so the fp64
 // chain of the weight overlaps the other warps' streaming.

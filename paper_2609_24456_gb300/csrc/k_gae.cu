@@ -26,7 +26,10 @@
 // the returns and per-CTA fp64 sums of A and A^2; the normalisation kernel
 // forms mean and the unbiased standard deviation (every CTA reduces the
 // partials in the same fixed order, so all agree bit for bit) and writes
-// the normalised values, one thread per element.
+// the normalised values, one thread per element.  With the environments
+// sharded over several ranks, the scan's sums are reduced to this rank's
+// (n, sum A, sum A^2) instead (k_gae_stats), the caller sums those over the
+// ranks, and the normalisation reads the totals.
 #include "edp_internal.cuh"
 
 namespace edp {
@@ -205,19 +208,11 @@ k_gae_scan(const float *__restrict__ r, const float *__restrict__ v,
   }
 }
 
-// Normalisation: every CTA reduces the per-CTA partials of the scan in the
-// same fixed order, then one thread per element writes (A - mean) * inv_std.
-// A is read from A_src (the caller's adv, or adv_norm itself).
-__global__ void __launch_bounds__(kNormThreads)
-k_gae_norm(const float *A_src, float *adv_norm, uint64_t n, const double *partial,
-           uint32_t nparts) {
-  __shared__ double r1[kNormThreads], r2[kNormThreads];
-  __shared__ double stat[2];
-  pdl_wait();
-  pdl_launch();
-  // this thread's first element, loaded beside the partial sums
-  const uint64_t i0 = blockIdx.x * (uint64_t)kNormThreads + threadIdx.x;
-  const float a0 = i0 < n ? __ldcg(&A_src[i0]) : 0.f;
+// Sum of the per-CTA partials (sum A, sum A^2) in a fixed order: strided
+// per-thread sums, then a shared-memory tree; the totals end in r1[0],
+// r2[0].  Every CTA that calls it gets the same bits.
+__device__ __forceinline__ void reduce_partials(const double *partial, uint32_t nparts,
+                                                double *r1, double *r2) {
   double t1 = 0.0, t2 = 0.0;
   for (unsigned i = threadIdx.x; i < nparts; i += kNormThreads) {
     t1 += __ldcg(&partial[2 * i]);
@@ -233,16 +228,58 @@ k_gae_norm(const float *A_src, float *adv_norm, uint64_t n, const double *partia
     }
     __syncthreads();
   }
+}
+
+// This rank's statistics of A for a normalisation over several ranks:
+// stats = (n, sum A, sum A^2), reduced from the scan's partials in the same
+// order as k_gae_norm reduces them (one CTA).
+__global__ void __launch_bounds__(kNormThreads)
+k_gae_stats(const double *partial, uint32_t nparts, uint64_t n, double *stats) {
+  __shared__ double r1[kNormThreads], r2[kNormThreads];
+  pdl_wait();
+  pdl_launch();
+  reduce_partials(partial, nparts, r1, r2);
   if (threadIdx.x == 0) {
-    const double nn = (double)n;
-    const double mean = r1[0] / nn;
-    double var = n > 1 ? (r2[0] - r1[0] * mean) / (nn - 1.0) : 0.0;
+    stats[0] = (double)n;
+    stats[1] = r1[0];
+    stats[2] = r2[0];
+  }
+}
+
+// Normalisation: every CTA reduces the per-CTA partials of the scan in the
+// same fixed order (or reads the statistics (n, sum A, sum A^2) of all ranks
+// when `stats` is given), then one thread per element writes
+// (A - mean) * inv_std.  A is read from A_src (the caller's adv, or adv_norm
+// itself); n is the number of elements here.
+__global__ void __launch_bounds__(kNormThreads)
+k_gae_norm(const float *A_src, float *adv_norm, uint64_t n, const double *partial,
+           uint32_t nparts, const double *stats) {
+  __shared__ double r1[kNormThreads], r2[kNormThreads];
+  __shared__ double stat[2];
+  pdl_wait();
+  pdl_launch();
+  // this thread's first element, loaded beside the partial sums
+  const uint64_t i0 = blockIdx.x * (uint64_t)kNormThreads + threadIdx.x;
+  const float a0 = i0 < n ? __ldcg(&A_src[i0]) : 0.f;
+  double nn = (double)n, s1, s2;
+  if (stats) {
+    nn = __ldcg(&stats[0]);
+    s1 = __ldcg(&stats[1]);
+    s2 = __ldcg(&stats[2]);
+  } else {
+    reduce_partials(partial, nparts, r1, r2);
+    s1 = r1[0];
+    s2 = r2[0];
+  }
+  if (threadIdx.x == 0) {
+    const double mean = s1 / nn;
+    double var = nn > 1.0 ? (s2 - s1 * mean) / (nn - 1.0) : 0.0;
     if (var < 0.0) var = 0.0;
     stat[0] = mean;
     // a single value equals its mean and normalises to exactly 0; the scale
     // is 0 so that the fp32 rounding of the stored A (A - mean ~ 2^-24 |A|
     // here) is not multiplied by 1 / 1e-8
-    stat[1] = n > 1 ? 1.0 / (sqrt(var) + 1e-8) : 0.0;
+    stat[1] = nn > 1.0 ? 1.0 / (sqrt(var) + 1e-8) : 0.0;
   }
   __syncthreads();
   const double mean = stat[0], inv = stat[1];
@@ -277,7 +314,31 @@ cudaError_t launch_gae(edp_ctx *c, const float *r, const float *v,
   if (ng > 4ull * c->coop_sms) ng = 4ull * c->coop_sms;
   return launch_pdl(k_gae_norm, dim3((unsigned)ng), dim3(kNormThreads), s,
                     (const float *)A_out, adv_norm, n, (const double *)partial,
-                    (uint32_t)grid);
+                    (uint32_t)grid, (const double *)nullptr);
+}
+
+cudaError_t launch_gae_stats(edp_ctx *c, const float *r, const float *v,
+                             const uint8_t *d, uint32_t T, uint32_t E, double gamma,
+                             double lambda, float *adv, float *ret, double *stats,
+                             cudaStream_t s) {
+  const uint64_t grid = (E + kGaeWarps - 1) / kGaeWarps;
+  void *blk = nullptr;
+  cudaError_t e = ctx_scratch(c, grid * 2 * sizeof(double), s, &blk);
+  if (e != cudaSuccess) return e;
+  double *partial = (double *)blk;
+  e = launch_pdl(k_gae_scan, dim3((unsigned)grid), dim3(kGaeThreads), s, r, v, d, T, E,
+                 gamma, lambda, adv, ret, partial);
+  if (e != cudaSuccess) return e;
+  return launch_pdl(k_gae_stats, dim3(1), dim3(kNormThreads), s, (const double *)partial,
+                    (uint32_t)grid, (uint64_t)T * E, stats);
+}
+
+cudaError_t launch_gae_normalize(edp_ctx *c, const float *adv, uint64_t n,
+                                 const double *stats, float *adv_norm, cudaStream_t s) {
+  uint64_t ng = (n + kNormThreads - 1) / kNormThreads;
+  if (ng > 4ull * c->coop_sms) ng = 4ull * c->coop_sms;
+  return launch_pdl(k_gae_norm, dim3((unsigned)ng), dim3(kNormThreads), s, adv, adv_norm, n,
+                    (const double *)nullptr, 0u, stats);
 }
 
 }  // namespace edp

@@ -67,6 +67,60 @@ __global__ void k_tree_level(uint64_t *__restrict__ out,
 constexpr int kSmemLevels = 2;
 constexpr int kSmemNodes = 32 + 1024;
 
+// Copies levels 1 .. cached of the tree into top (all loads issued before
+// any use); returns the number of cached levels.
+__device__ __forceinline__ uint32_t cache_top(const TreeView &t, uint64_t *top,
+                                              uint64_t keep) {
+  const uint32_t cached = t.depth - 1 < (uint32_t)kSmemLevels ? t.depth - 1 : kSmemLevels;
+  const uint32_t ncached = cached == 0 ? 0 : (cached == 1 ? 32 : 32 + 1024);
+  uint64_t v5[5];
+#pragma unroll
+  for (int u = 0; u < 5; ++u) {
+    const uint32_t i = threadIdx.x + u * 256;
+    v5[u] = i < ncached ? ld_keep(t.nodes + 1 + i, keep) : 0ull;
+  }
+#pragma unroll
+  for (int u = 0; u < 5; ++u) {
+    const uint32_t i = threadIdx.x + u * 256;
+    if (i < ncached) top[i] = v5[u];
+  }
+  return cached;
+}
+
+// Descent of one target (one warp): the leaf whose prefix range [prefix(i),
+// prefix(i) + q_i) holds `target`, for target < S.  Per level: the 32
+// children, an inclusive warp prefix sum and a ballot.  *ok is cleared if
+// the sums disagree with the children (the leaf then stays in range).
+__device__ __forceinline__ uint64_t descend(const TreeView &t, const uint64_t *top,
+                                            uint32_t cached, uint64_t target, int lane,
+                                            uint64_t keep, bool *ok) {
+  uint64_t node = 0;
+  for (uint32_t d = 1; d <= t.depth; ++d) {
+    const uint64_t c = node * kFanout + lane;
+    uint64_t v;
+    if (d <= cached)
+      v = top[(d == 1 ? 0 : 32) + c];
+    else
+      v = d < t.depth ? ld_keep(t.lvl(d) + c, keep) : (uint64_t)ld_keep(t.leaves + c, keep);
+    uint64_t incl = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint64_t y = __shfl_up_sync(kFull, incl, o);
+      if (lane >= o) incl += y;
+    }
+    unsigned m = __ballot_sync(kFull, target < incl);
+    if (m == 0) {  // sums disagree with children: report, stay in range
+      *ok = false;
+      m = 1u << 31;
+    }
+    const int f = __ffs(m) - 1;
+    const uint64_t excl = __shfl_sync(kFull, incl - v, f);
+    target = target >= excl ? target - excl : 0;
+    node = node * kFanout + f;
+  }
+  return node;
+}
+
 __global__ void __launch_bounds__(256)
 k_sample_prio(TreeView t, uint32_t B, uint64_t seed, uint64_t round,
               int64_t *__restrict__ idx, uint32_t *__restrict__ qout,
@@ -76,21 +130,8 @@ k_sample_prio(TreeView t, uint32_t B, uint64_t seed, uint64_t round,
   const uint64_t keep = policy_keep();
   pdl_wait();
   pdl_launch();
-  const uint32_t cached = t.depth - 1 < (uint32_t)kSmemLevels ? t.depth - 1 : kSmemLevels;
-  const uint32_t ncached = cached == 0 ? 0 : (cached == 1 ? 32 : 32 + 1024);
-  // levels 1.. start right after the root; all loads issued before any use
-  uint64_t v5[5];
-#pragma unroll
-  for (int u = 0; u < 5; ++u) {
-    const uint32_t i = threadIdx.x + u * 256;
-    v5[u] = i < ncached ? ld_keep(t.nodes + 1 + i, keep) : 0ull;
-  }
-  const uint64_t S = t.nodes[0];
-#pragma unroll
-  for (int u = 0; u < 5; ++u) {
-    const uint32_t i = threadIdx.x + u * 256;
-    if (i < ncached) top[i] = v5[u];
-  }
+  const uint64_t S = t.nodes[0];  // issued beside the loads of the top levels
+  const uint32_t cached = cache_top(t, top, keep);
   __syncthreads();
   const uint32_t warps = (gridDim.x * blockDim.x) >> 5;
   for (uint32_t k = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; k < B;
@@ -103,38 +144,45 @@ k_sample_prio(TreeView t, uint32_t B, uint64_t seed, uint64_t round,
       }
       continue;
     }
-    // stratum [lo, hi) = [floor(kS/B), floor((k+1)S/B)); with S = aB + b,
-    // floor(kS/B) = ak + floor(bk/B), every term below 2^64.
-    const uint64_t a = S / B, b = S % B;
-    const uint64_t lo = a * k + (b * k) / B;
-    const uint64_t hi = a * (k + 1) + (b * (k + 1)) / B;
-    const uint64_t u = philox_u64(seed, k, round, 1);
-    uint64_t target = lo + mulhi64(u, hi - lo);
-    uint64_t node = 0;
+    const uint64_t target = stratum_target(S, B, k, seed, round);
     bool ok = true;
-    for (uint32_t d = 1; d <= t.depth; ++d) {
-      const uint64_t c = node * kFanout + lane;
-      uint64_t v;
-      if (d <= cached)
-        v = top[(d == 1 ? 0 : 32) + c];
-      else
-        v = d < t.depth ? ld_keep(t.lvl(d) + c, keep) : (uint64_t)ld_keep(t.leaves + c, keep);
-      uint64_t incl = v;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const uint64_t y = __shfl_up_sync(kFull, incl, o);
-        if (lane >= o) incl += y;
-      }
-      unsigned m = __ballot_sync(kFull, target < incl);
-      if (m == 0) {  // sums disagree with children: report, stay in range
-        ok = false;
-        m = 1u << 31;
-      }
-      const int f = __ffs(m) - 1;
-      const uint64_t excl = __shfl_sync(kFull, incl - v, f);
-      target = target >= excl ? target - excl : 0;
-      node = node * kFanout + f;
+    const uint64_t node = descend(t, top, cached, target, lane, keep, &ok);
+    if (lane == 0) {
+      if (!ok) flag(ctrl, DEVERR_TREE, k);
+      idx[k] = (int64_t)node;
+      if (qout) qout[k] = t.leaves[node];
     }
+  }
+}
+
+// Descent of given targets (the shard side of a sharded buffer: targets
+// routed here by edp_route_prioritized, each below this tree's total):
+// one warp per target.  A target >= S is reported (DEVERR_INDEX) and
+// gives idx -1, q 0.
+__global__ void __launch_bounds__(256)
+k_sample_targets(TreeView t, const uint64_t *__restrict__ targets, uint32_t n,
+                 int64_t *__restrict__ idx, uint32_t *__restrict__ qout, Ctrl *ctrl) {
+  __shared__ uint64_t top[kSmemNodes];
+  const int lane = threadIdx.x & 31;
+  const uint64_t keep = policy_keep();
+  pdl_wait();
+  pdl_launch();
+  const uint64_t S = t.nodes[0];  // issued beside the loads of the top levels
+  const uint32_t cached = cache_top(t, top, keep);
+  __syncthreads();
+  const uint32_t warps = (gridDim.x * blockDim.x) >> 5;
+  for (uint32_t k = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; k < n; k += warps) {
+    const uint64_t target = targets[k];
+    if (target >= S) {
+      if (lane == 0) {
+        idx[k] = -1;
+        if (qout) qout[k] = 0;
+        flag(ctrl, DEVERR_INDEX, target);
+      }
+      continue;
+    }
+    bool ok = true;
+    const uint64_t node = descend(t, top, cached, target, lane, keep, &ok);
     if (lane == 0) {
       if (!ok) flag(ctrl, DEVERR_TREE, k);
       idx[k] = (int64_t)node;
@@ -383,6 +431,15 @@ cudaError_t launch_tree_refresh(edp_ctx *c, uint64_t first, uint64_t count,
 
 cudaError_t launch_tree_build_all(edp_ctx *c, cudaStream_t s) {
   return launch_tree_refresh(c, 0, c->cap, s);
+}
+
+cudaError_t launch_sample_targets(edp_ctx *c, const uint64_t *targets, uint32_t n,
+                                  int64_t *idx, uint32_t *q, cudaStream_t s) {
+  const unsigned warps_per_block = 8;
+  uint64_t blocks = (n + warps_per_block - 1) / warps_per_block;
+  if (blocks > 8u * (unsigned)c->coop_sms) blocks = 8u * (unsigned)c->coop_sms;
+  return launch_pdl(k_sample_targets, dim3((unsigned)blocks), dim3(warps_per_block * 32),
+                    s, view(c), targets, n, idx, q, c->ctrl);
 }
 
 cudaError_t launch_sample_prioritized(edp_ctx *c, uint32_t B, uint64_t seed,

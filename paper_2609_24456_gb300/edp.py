@@ -115,6 +115,15 @@ SIGNATURES = {
     "edp_priorities_from_td": (C.c_int, [_VP, _VP, _U32, _D, _D, _VP, _VP]),
     "edp_gae": (C.c_int, [_VP, _VP, _VP, _VP, _U32, _U32, _D, _D, _VP, _VP,
                           _VP, _VP]),
+    "edp_tree_total": (C.c_int, [_VP, _VP, _VP]),
+    "edp_route_prioritized": (C.c_int, [_VP, _VP, _U32, _U32, _U32, _U32, _U64, _U64,
+                                        _VP, _VP, _VP]),
+    "edp_sample_targets": (C.c_int, [_VP, _VP, _U32, _VP, _VP, _VP]),
+    "edp_batch_qmin": (C.c_int, [_VP, _VP, _U32, _VP, _VP]),
+    "edp_is_weights": (C.c_int, [_VP, _VP, _U32, _VP, _D, _VP, _VP]),
+    "edp_gae_stats": (C.c_int, [_VP, _VP, _VP, _VP, _U32, _U32, _D, _D, _VP, _VP, _VP,
+                                _VP]),
+    "edp_gae_normalize": (C.c_int, [_VP, _VP, _U64, _VP, _VP, _VP]),
     "edp_sync": (C.c_int, [_VP, _VP]),
     "edp_last_error": (C.c_char_p, [_VP]),
     "edp_get_info": (C.c_int, [_VP, C.POINTER(edp_info)]),
@@ -269,6 +278,45 @@ def edp_gae(ctx, r, v, d, T, E, gamma, lam, adv=None, ret=None, adv_norm=None,
     return _check(ctx, lib().edp_gae(ctx, ptr(r), ptr(v), ptr(d), T, E, gamma,
                                      lam, ptr(adv), ptr(ret), ptr(adv_norm),
                                      stream_handle(stream)), "edp_gae")
+
+
+# --- sharded buffer (include/edp.h, "Sharded buffer") ---------------------------
+def edp_tree_total(ctx, total, stream=None):
+    return _check(ctx, lib().edp_tree_total(ctx, ptr(total), stream_handle(stream)),
+                  "edp_tree_total")
+
+
+def edp_route_prioritized(ctx, totals, G, batch, k0, n, seed, round_, local_t, counts,
+                          stream=None):
+    return _check(ctx, lib().edp_route_prioritized(
+        ctx, ptr(totals), G, batch, k0, n, seed, round_, ptr(local_t), ptr(counts),
+        stream_handle(stream)), "edp_route_prioritized")
+
+
+def edp_sample_targets(ctx, targets, n, idx, q=None, stream=None):
+    return _check(ctx, lib().edp_sample_targets(ctx, ptr(targets), n, ptr(idx), ptr(q),
+                                                stream_handle(stream)), "edp_sample_targets")
+
+
+def edp_batch_qmin(ctx, q, n, qmin, stream=None):
+    return _check(ctx, lib().edp_batch_qmin(ctx, ptr(q), n, ptr(qmin),
+                                            stream_handle(stream)), "edp_batch_qmin")
+
+
+def edp_is_weights(ctx, q, n, qmin, beta, w, stream=None):
+    return _check(ctx, lib().edp_is_weights(ctx, ptr(q), n, ptr(qmin), beta, ptr(w),
+                                            stream_handle(stream)), "edp_is_weights")
+
+
+def edp_gae_stats(ctx, r, v, d, T, E, gamma, lam, adv, stats, ret=None, stream=None):
+    return _check(ctx, lib().edp_gae_stats(ctx, ptr(r), ptr(v), ptr(d), T, E, gamma, lam,
+                                           ptr(adv), ptr(ret), ptr(stats),
+                                           stream_handle(stream)), "edp_gae_stats")
+
+
+def edp_gae_normalize(ctx, adv, n, stats, adv_norm, stream=None):
+    return _check(ctx, lib().edp_gae_normalize(ctx, ptr(adv), n, ptr(stats), ptr(adv_norm),
+                                               stream_handle(stream)), "edp_gae_normalize")
 
 
 def edp_sync(ctx, stream=None):
