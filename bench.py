@@ -1591,6 +1591,127 @@ class LlmBatch(Workload):
         self.llm.pack(self.h_tok, self.h_off, self.h_perms[r % self.n_perm], adv)
 
 
+class ShardedPerReplay(PerReplay):
+    """The prioritized replay sharded over the ranks (N > 1, Sec. 5.1's
+    shared-GPU placement): every rank holds a 1,000,000-frame shard (its own
+    content) and a learner that receives 512 samples of each global batch of
+    512 N, drawn from the distribution over all shards' leaves.  Step = one
+    sharded round (paper_2609_24456_gb300.shard.ShardedPer): shard totals
+    all-gathered, targets routed to their owners, the owners' descents and
+    deliveries, rows back to the learners, importance weights against the
+    global minimum, TD-error updates back to the owners.  Rounds run eagerly:
+    each waits on the host for its routing counts, which size the
+    all-to-alls."""
+
+    def __init__(self, rank=0, **kw):
+        super().__init__(**kw)
+        self.sample_seed = self.seed
+        self.seed = self.seed + 7919 * rank  # this shard's content and TD errors
+
+    def setup(self, device):
+        from paper_2609_24456_gb300.shard import ShardComm, ShardedPer
+        super().setup(device)
+        self.sp = ShardedPer(self.ring, ShardComm(), self.B, beta=BETA, alpha=ALPHA, eps=EPS)
+
+    def config(self):
+        c = super().config()
+        c.update(workload=self.name + "-sharded", batch_per_rank=self.B,
+                 exchange="all-gather of shard totals, all-to-all of counts, targets, "
+                          "rows and TD errors, min-reduce of the batch minimum")
+        return c
+
+    def round(self, r):
+        self.sp.sample_deliver(self.sample_seed, r)
+        self.sp.update(td=self.td[r % self.td_rounds])
+
+    def schedules(self):
+        return [("sharded", self.round, "sharded round, eager (host-sized exchanges)")]
+
+    def time_latency(self, n, mk, stream):
+        import torch
+        out = []
+        for r in range(n):
+            e0, e1 = mk(), mk()
+            e0.record(stream)
+            self.sp.sample_deliver(self.sample_seed, 100000 + r)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            out.append(e0.elapsed_time(e1) * 1e3)
+        return out
+
+    def e2e_setup(self, device):
+        import torch
+        lo = self.sp.out
+        self.h_out = {k: torch.empty(lo[k].shape, dtype=lo[k].dtype, pin_memory=True)
+                      for k in ("obs", "nxt", "isw", "idx")}
+        self.h2d = 0
+        self.d2h = sum(t.numel() * t.element_size() for t in self.h_out.values())
+
+    def e2e_round(self, r):
+        self.sp.sample_deliver(self.sample_seed, r)
+        for k, t in self.h_out.items():
+            t.copy_(self.sp.out[k], non_blocking=True)
+        self.sp.update(td=self.td[r % self.td_rounds])
+
+
+class ShardedPpoIteration(PpoIteration):
+    """The on-policy iteration with environments sharded over the ranks
+    (N > 1): every rank holds 256 environments x 128 steps; GAE per rank,
+    the advantage normalisation over every rank's values (one fp64
+    all-reduce of (n, sum A, sum A^2)), then the rank's shuffle and its 8
+    mini-batches delivered in one call.  Eager."""
+
+    def __init__(self, rank=0, **kw):
+        super().__init__(**kw)
+        self.seed = self.seed + 7919 * rank
+
+    def setup(self, device):
+        import torch
+        from paper_2609_24456_gb300.shard import ShardComm
+        self.comm = ShardComm()
+        self.stats = torch.zeros(3, dtype=torch.float64, device=device)
+        super().setup(device)
+
+    def config(self):
+        c = super().config()
+        c.update(workload=self.name + "-sharded",
+                 exchange="all-reduce of (n, sum A, sum A^2) in fp64")
+        return c
+
+    def _gae(self):
+        from paper_2609_24456_gb300.shard import sharded_gae
+        sharded_gae(self.ring.ctx, self.comm, self.r, self.v, self.d, self.T, self.E,
+                    0.99, 0.95, self.adv, self.ret, self.nrm, self.stats)
+
+    def round(self, r):
+        self._gae()
+        self.edp.edp_sample(self.ring.ctx, self.edp.EDP_SAMPLE_PERMUTE, self.n,
+                            self.seed, r, self.idx)
+        self._deliver_all(1)
+
+    def schedules(self):
+        return [("sharded", self.round, "sharded GAE normalisation, shuffle, one delivery "
+                                        "call, eager")]
+
+    def time_latency(self, n, mk, stream):
+        import torch
+        out = []
+        for r in range(n):
+            e0, e1 = mk(), mk()
+            e0.record(stream)
+            self.latency_step(100000 + r, e1)
+            torch.cuda.synchronize()
+            out.append(e0.elapsed_time(e1) * 1e3)
+        return out
+
+    def extra(self, device, mk, stream, deliver_us):
+        return {}
+
+
+# with N > 1 ranks these workloads run sharded (one exchange per step);
+# the others run N independent replicas
+SHARDED = {"per1m": ShardedPerReplay, "ppo": ShardedPpoIteration}
+
 WORKLOADS = {
     "per1m": PerReplay,
     "dqn10k": DqnTiny,
@@ -1660,7 +1781,8 @@ def job_ms(ms, dist, device):
     if dist is None:
         return ms
     import torch
-    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    on = device if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([ms], dtype=torch.float64, device=on)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
 
@@ -1679,7 +1801,10 @@ def run_edp(args):
     dist = None
     if world > 1:
         import torch.distributed as dist
-        dist.init_process_group("nccl")
+        dist.init_process_group(args.dist_backend)
+    # one rank per GPU; with fewer GPUs than ranks (gloo, host-staged
+    # exchanges) ranks share them
+    local = local % max(1, torch.cuda.device_count())
     torch.cuda.set_device(local)
     device = torch.device("cuda", local)
     from paper_2609_24456_gb300 import build
@@ -1690,9 +1815,15 @@ def run_edp(args):
         dist.barrier()
     build.build()  # up to date by now: only checks
 
-    wl = WORKLOADS[args.workload](**({"capacity": args.capacity} if args.capacity else {}))
     if args.workload == "ppo" and args.capacity:
         raise SystemExit("--capacity does not apply to the ppo workload")
+    kw = {"capacity": args.capacity} if args.capacity else {}
+    sharded = world > 1 and args.workload in SHARDED
+    if sharded:
+        wl = SHARDED[args.workload](rank=rank, **kw)
+        args.no_graph = True  # every round sizes its exchanges on the host
+    else:
+        wl = WORKLOADS[args.workload](**kw)
     wl.setup(device)
     K, W = args.steps, args.warmup
     mk = lambda: torch.cuda.Event(enable_timing=True, external=True)
@@ -1818,7 +1949,8 @@ def run_edp(args):
                 "ms_per_step": ms_step, "higher_is_better": True,
                 "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype,
                 "data": "synthetic", "config": dict(wl.config(),
-                                                    parallelism="replicas%d" % world,
+                                                    parallelism=("sharded%d" if sharded
+                                                                 else "replicas%d") % world,
                                                     graph=use_graph,
                                                     schedule="%s: %s" % scheds[0][::2]),
                 "pct_hbm_peak": 100.0 * value / peak,
@@ -1846,6 +1978,9 @@ def main():
     ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", default="edp", choices=["edp", "reference"])
+    ap.add_argument("--dist-backend", default="nccl", choices=["nccl", "gloo"],
+                    help="process-group backend for N > 1 (gloo stages the sharded "
+                         "exchanges through host memory, so several ranks may share a GPU)")
     # default: the largest HBM-resident configuration (200,000 multimodal
     # transitions, ~30 GB), whose metric is the fraction of HBM bandwidth
     ap.add_argument("--workload", default="mm200k", choices=sorted(WORKLOADS))

@@ -16,9 +16,13 @@ METHODS = ["config", "setup", "schedules", "deliver_once", "latency_step",
            "e2e_setup", "e2e_round", "cpu_setup", "cpu_round"]
 
 
-@pytest.mark.parametrize("name", sorted(bench.WORKLOADS))
+@pytest.mark.parametrize("name", sorted(bench.WORKLOADS) + ["sharded-" + n for n in
+                                                            sorted(bench.SHARDED)])
 def test_workload_has_every_leg(name):
-    wl = bench.WORKLOADS[name]()
+    if name.startswith("sharded-"):
+        wl = bench.SHARDED[name[len("sharded-"):]](rank=1)
+    else:
+        wl = bench.WORKLOADS[name]()
     for m in METHODS:
         assert callable(getattr(wl, m, None)), (name, m)
     for attr in ("kernel", "dtype", "deliver_bytes", "round_bytes", "launches_per_round"):
