@@ -801,16 +801,10 @@ edp_status edp_ingest(edp_ctx *ctx, const edp_fields *src, uint64_t n,
     }
     if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_ingest(host tier)");
   }
-  const uint64_t skip = new_hbm_lo - T, nh = Tn - new_hbm_lo;
-  if (!swapped) {
-    e = launch_copy_rows(ctx->st.obs, ctx->cap_h, new_hbm_lo % ctx->cap_h,
-                         f.obs + skip * ctx->obs_bytes, nh, ctx->obs_bytes, s);
-    if (e == cudaSuccess && ctx->tok_bytes)
-      e = launch_copy_rows((uint8_t *)ctx->st.tokens, ctx->cap_h,
-                           new_hbm_lo % ctx->cap_h,
-                           (const uint8_t *)f.tokens + skip * ctx->tok_bytes, nh,
-                           ctx->tok_bytes, s);
-  }
+  // metadata and leaves, then the tree above them, then the payload rows:
+  // the row copy starts behind the (waiting) metadata and tree kernels and
+  // overlaps them, since neither reads the rows
+  const bool meta = ctx->st.action || ctx->st.reward || ctx->st.done || ctx->leaves;
   if (e == cudaSuccess) e = launch_ingest_meta(ctx, &f, n, q, s);
   if (e == cudaSuccess && ctx->depth) {
     uint64_t first = ctx->total % ctx->cap, count = n;
@@ -820,6 +814,16 @@ edp_status edp_ingest(edp_ctx *ctx, const edp_fields *src, uint64_t n,
     }
     if (count > ctx->cap) count = ctx->cap;
     e = launch_tree_refresh(ctx, first, count, s);
+  }
+  const uint64_t skip = new_hbm_lo - T, nh = Tn - new_hbm_lo;
+  if (e == cudaSuccess && !swapped) {
+    e = launch_copy_rows(ctx->st.obs, ctx->cap_h, new_hbm_lo % ctx->cap_h,
+                         f.obs + skip * ctx->obs_bytes, nh, ctx->obs_bytes, s, !meta);
+    if (e == cudaSuccess && ctx->tok_bytes)
+      e = launch_copy_rows((uint8_t *)ctx->st.tokens, ctx->cap_h,
+                           new_hbm_lo % ctx->cap_h,
+                           (const uint8_t *)f.tokens + skip * ctx->tok_bytes, nh,
+                           ctx->tok_bytes, s, false);  // behind the row copy
   }
   if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_ingest");
   ctx->total += n;

@@ -384,9 +384,13 @@ cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block,
 // ---------------------------------------------------------------------------
 // Launchers (host).  Each returns cudaGetLastError() after its launches.
 // ---------------------------------------------------------------------------
+// Rows of an ingest source into the ring at first, first + 1, ... (mod
+// dst_cap).  wait_first: wait for the preceding kernel before touching
+// memory; false only right behind a kernel of the same call that waited on
+// its own predecessor (the copy then overlaps it, and waits at its end).
 cudaError_t launch_copy_rows(uint8_t *dst, uint64_t dst_cap, uint64_t first,
                              const uint8_t *src, uint64_t n, uint64_t row_bytes,
-                             cudaStream_t s);
+                             cudaStream_t s, bool wait_first);
 cudaError_t launch_ingest_meta(edp_ctx *ctx, const edp_fields *src, uint64_t n,
                                const uint32_t *q, cudaStream_t s);
 cudaError_t launch_demote(edp_ctx *ctx, uint64_t first_id, uint64_t n,

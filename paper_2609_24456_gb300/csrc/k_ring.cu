@@ -14,35 +14,57 @@ namespace {
 constexpr int kCopyThreads = 256;
 constexpr int kCopyUnroll = 4;
 
-// Copy n rows of cpr 16-byte chunks: src row (src_first + j) mod src_cap ->
-// dst row (dst_first + j) mod dst_cap.  Grid: x tiles the chunks of a row,
-// y strides over rows.  src may be page-locked host memory (mapped).
+// Copy of up to three contiguous runs of 16-byte words (a range of ring
+// rows splits where the source or the destination wraps): a flat
+// grid-stride loop, kCopyFlat words in flight per thread, so the copy is
+// one stream of full 16-byte accesses whatever the row size.  src may be
+// page-locked host memory (mapped).  With wait_first the kernel waits for
+// the preceding kernel before it reads or writes anything; otherwise it
+// starts at once -- allowed only right behind a kernel of the same call that
+// waited on its own predecessor, so the rows it overwrites are no longer
+// read -- and waits at its end, so it never completes before that kernel.
+constexpr int kCopyFlat = 8;
+constexpr int kCopyCtasPerSm = 64;
+struct CopyRuns {
+  const uint4 *src[3];
+  uint4 *dst[3];
+  uint64_t end[3];  // cumulative word counts; unused runs repeat the total
+};
+
 __global__ void __launch_bounds__(kCopyThreads)
-k_copy_rows(uint8_t *__restrict__ dst, uint64_t dst_cap, uint64_t dst_first,
-            const uint8_t *__restrict__ src, uint64_t src_cap,
-            uint64_t src_first, uint64_t n, uint32_t cpr) {
-  const uint64_t row_bytes = (uint64_t)cpr * 16u;
-  for (uint64_t j = blockIdx.y; j < n; j += gridDim.y) {
-    const uint64_t ds = (dst_first + j) % dst_cap;
-    const uint64_t ss = (src_first + j) % src_cap;
-    const uint4 *s = reinterpret_cast<const uint4 *>(src + ss * row_bytes);
-    uint4 *d = reinterpret_cast<uint4 *>(dst + ds * row_bytes);
-    const uint32_t step = gridDim.x * kCopyThreads * kCopyUnroll;
-    for (uint32_t w0 = blockIdx.x * kCopyThreads * kCopyUnroll + threadIdx.x;
-         w0 < cpr; w0 += step) {
-      uint4 v[kCopyUnroll];
+k_copy_flat(CopyRuns r, int wait_first) {
+  if (wait_first) pdl_wait();
+  pdl_launch();
+  const uint64_t total = r.end[2];  // unused runs repeat the last end
+  constexpr uint64_t kTile = (uint64_t)kCopyThreads * kCopyFlat;  // words per tile
+  const uint64_t tiles = (total + kTile - 1) / kTile;
+  // a CTA moves whole tiles: kCopyFlat warp-wide accesses of 512 contiguous
+  // bytes each per warp, the CTA's loads covering one contiguous tile
+  for (uint64_t t = blockIdx.x; t < tiles; t += gridDim.x) {
+    const uint64_t i0 = t * kTile + threadIdx.x;
+    uint4 v[kCopyFlat];
 #pragma unroll
-      for (int u = 0; u < kCopyUnroll; ++u) {
-        const uint32_t w = w0 + u * kCopyThreads;
-        if (w < cpr) v[u] = s[w];
+    for (int u = 0; u < kCopyFlat; ++u) {
+      const uint64_t i = i0 + (uint64_t)u * kCopyThreads;
+      if (i < total) {
+        // run of word i, selected without indexing the parameter array
+        // (which would place it in local memory)
+        const bool g1 = i >= r.end[0], g2 = i >= r.end[1];
+        const uint64_t o = g2 ? i - r.end[1] : (g1 ? i - r.end[0] : i);
+        v[u] = (g2 ? r.src[2] : (g1 ? r.src[1] : r.src[0]))[o];
       }
+    }
 #pragma unroll
-      for (int u = 0; u < kCopyUnroll; ++u) {
-        const uint32_t w = w0 + u * kCopyThreads;
-        if (w < cpr) d[w] = v[u];
+    for (int u = 0; u < kCopyFlat; ++u) {
+      const uint64_t i = i0 + (uint64_t)u * kCopyThreads;
+      if (i < total) {
+        const bool g1 = i >= r.end[0], g2 = i >= r.end[1];
+        const uint64_t o = g2 ? i - r.end[1] : (g1 ? i - r.end[0] : i);
+        (g2 ? r.dst[2] : (g1 ? r.dst[1] : r.dst[0]))[o] = v[u];
       }
     }
   }
+  if (!wait_first) pdl_wait();
 }
 
 // Swap rows through HBM: HBM row (first + j) mod hbm_cap moves to host row
@@ -97,17 +119,36 @@ cudaError_t swap_rows(uint8_t *hbm, uint64_t hbm_cap, uint8_t *host, uint64_t ho
   return cudaGetLastError();
 }
 
+// Rows (src_first + j) mod src_cap -> (dst_first + j) mod dst_cap for
+// j < n, as the contiguous runs between the wrap points of either side.
 cudaError_t copy_rows(uint8_t *dst, uint64_t dst_cap, uint64_t dst_first,
                       const uint8_t *src, uint64_t src_cap, uint64_t src_first,
-                      uint64_t n, uint64_t row_bytes, cudaStream_t s) {
+                      uint64_t n, uint64_t row_bytes, cudaStream_t s, bool wait_first) {
   if (!n) return cudaSuccess;
-  const uint32_t cpr = (uint32_t)(row_bytes / 16);
-  uint32_t gx = (cpr + kCopyThreads * kCopyUnroll - 1) / (kCopyThreads * kCopyUnroll);
-  if (gx > 64) gx = 64;
-  const uint32_t gy = n < 65535 ? (uint32_t)n : 65535u;
-  k_copy_rows<<<dim3(gx, gy), kCopyThreads, 0, s>>>(dst, dst_cap, dst_first, src,
-                                                   src_cap, src_first, n, cpr);
-  return cudaGetLastError();
+  uint64_t cut[4] = {0, n, n, n};
+  int nc = 1;
+  const uint64_t jd = dst_cap - dst_first, js = src_cap - src_first;
+  for (uint64_t j : {jd < js ? jd : js, jd < js ? js : jd})
+    if (j > cut[nc - 1] && j < n) cut[nc++] = j;
+  cut[nc] = n;
+  CopyRuns r{};
+  uint64_t acc = 0;
+  for (int g = 0; g < nc; ++g) {
+    const uint64_t j0 = cut[g];
+    r.src[g] = reinterpret_cast<const uint4 *>(src + ((src_first + j0) % src_cap) * row_bytes);
+    r.dst[g] = reinterpret_cast<uint4 *>(dst + ((dst_first + j0) % dst_cap) * row_bytes);
+    acc += (cut[g + 1] - j0) * (row_bytes / 16);
+    r.end[g] = acc;
+  }
+  for (int g = nc; g < 3; ++g) r.end[g] = acc;
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  uint64_t blocks = (acc + (uint64_t)kCopyThreads * kCopyFlat - 1) / ((uint64_t)kCopyThreads * kCopyFlat);
+  const uint64_t most = (uint64_t)kCopyCtasPerSm * (sms > 0 ? sms : 1);
+  if (blocks > most) blocks = most;
+  return launch_pdl(k_copy_flat, dim3((unsigned)blocks), dim3(kCopyThreads), s, r,
+                    wait_first ? 1 : 0);
 }
 
 // Metadata of n new transitions at logical ids total.. and, for PER, their
@@ -124,6 +165,8 @@ __global__ void k_ingest_meta(int32_t *__restrict__ action,
                               const uint32_t *__restrict__ q, Ctrl *ctrl,
                               uint64_t cap, uint64_t total, uint64_t n,
                               int defer) {
+  pdl_wait();
+  pdl_launch();
   uint32_t qdefault = 0;
   if (leaves && !q) qdefault = ctrl->max_q;
   uint32_t qmax_local = 0;  // one atomic per warp, not per transition
@@ -188,8 +231,8 @@ __global__ void k_probe_read(const uint4 *__restrict__ src, uint64_t n16,
 
 cudaError_t launch_copy_rows(uint8_t *dst, uint64_t dst_cap, uint64_t first,
                              const uint8_t *src, uint64_t n, uint64_t row_bytes,
-                             cudaStream_t s) {
-  return copy_rows(dst, dst_cap, first, src, ~0ull, 0, n, row_bytes, s);
+                             cudaStream_t s, bool wait_first) {
+  return copy_rows(dst, dst_cap, first, src, ~0ull, 0, n, row_bytes, s, wait_first);
 }
 
 cudaError_t launch_ingest_meta(edp_ctx *c, const edp_fields *f, uint64_t n,
@@ -199,10 +242,9 @@ cudaError_t launch_ingest_meta(edp_ctx *c, const edp_fields *f, uint64_t n,
   const int threads = 256;
   uint64_t blocks = (n + threads - 1) / threads;
   if (blocks > 4096) blocks = 4096;
-  k_ingest_meta<<<(unsigned)blocks, threads, 0, s>>>(
-      c->st.action, c->st.reward, c->st.done, f->action, f->reward, f->done,
-      c->leaves, q, c->ctrl, c->cap, c->total, n, c->defer);
-  return cudaGetLastError();
+  return launch_pdl(k_ingest_meta, dim3((unsigned)blocks), dim3(threads), s,
+                    c->st.action, c->st.reward, c->st.done, f->action, f->reward, f->done,
+                    c->leaves, q, c->ctrl, c->cap, c->total, n, c->defer);
 }
 
 // Two-tier demotion: payload of ids [first_id, first_id+n) moves from HBM
@@ -212,11 +254,11 @@ cudaError_t launch_demote(edp_ctx *c, uint64_t first_id, uint64_t n,
                           cudaStream_t s) {
   cudaError_t e = copy_rows(c->st.host_obs, c->cap_c, first_id % c->cap_c,
                             c->st.obs, c->cap_h, first_id % c->cap_h, n,
-                            c->obs_bytes, s);
+                            c->obs_bytes, s, true);
   if (e == cudaSuccess && c->tok_bytes)
     e = copy_rows((uint8_t *)c->st.host_tokens, c->cap_c, first_id % c->cap_c,
                   (const uint8_t *)c->st.tokens, c->cap_h, first_id % c->cap_h,
-                  n, c->tok_bytes, s);
+                  n, c->tok_bytes, s, true);
   return e;
 }
 
@@ -332,11 +374,11 @@ cudaError_t launch_copy_rows_to_host(edp_ctx *c, const uint8_t *obs,
                                      cudaStream_t s) {
   cudaError_t e = copy_rows(c->st.host_obs, c->cap_c, first_id % c->cap_c,
                             obs + src_row * c->obs_bytes, ~0ull, 0, n,
-                            c->obs_bytes, s);
+                            c->obs_bytes, s, true);
   if (e == cudaSuccess && c->tok_bytes)
     e = copy_rows((uint8_t *)c->st.host_tokens, c->cap_c, first_id % c->cap_c,
                   (const uint8_t *)tokens + src_row * c->tok_bytes, ~0ull, 0, n,
-                  c->tok_bytes, s);
+                  c->tok_bytes, s, true);
   return e;
 }
 

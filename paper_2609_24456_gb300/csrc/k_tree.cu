@@ -50,6 +50,8 @@ __global__ void k_tree_level(uint64_t *__restrict__ out,
                              const uint64_t *__restrict__ child64,
                              const uint32_t *__restrict__ child32, uint64_t a0,
                              uint64_t n0, uint64_t a1, uint64_t n1) {
+  pdl_wait();
+  pdl_launch();
   const uint64_t w = (blockIdx.x * (uint64_t)blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (w >= n0 + n1) return;
@@ -419,11 +421,12 @@ cudaError_t launch_tree_refresh(edp_ctx *c, uint64_t first, uint64_t count,
     const uint64_t threads = nodes * 32;
     const unsigned blocks = (unsigned)((threads + 255) / 256);
     const bool leaves_below = (uint32_t)(d + 1) == c->depth;
-    k_tree_level<<<blocks, 256, 0, s>>>(c->level[d],
-                                        leaves_below ? nullptr : c->level[d + 1],
-                                        leaves_below ? c->leaves : nullptr, x0,
-                                        y0 - x0, x1, y1 - x1);
-    cudaError_t e = cudaGetLastError();
+    cudaError_t e = launch_pdl(k_tree_level, dim3(blocks), dim3(256), s, c->level[d],
+                               leaves_below ? (const uint64_t *)nullptr
+                                            : (const uint64_t *)c->level[d + 1],
+                               leaves_below ? (const uint32_t *)c->leaves
+                                            : (const uint32_t *)nullptr,
+                               x0, y0 - x0, x1, y1 - x1);
     if (e != cudaSuccess) return e;
   }
   return cudaSuccess;
