@@ -212,6 +212,8 @@ class Workload:
     name = kernel = ""
     dtype = ""
     launches_per_round = 0
+    # launches per round of schedules that differ from launches_per_round
+    launches_by_schedule = {}
     h2d = d2h = 0
 
     def config(self):
@@ -552,6 +554,7 @@ class DqnTiny(Workload):
     kernel = "k_deliver_stack"
     dtype = "u8->f32"
     launches_per_round = 2
+    launches_by_schedule = {"fused": 1}
 
     def __init__(self, capacity=10_000, batch=32, K=4, seed=1234, out_sets=32):
         self.cap, self.B, self.K, self.seed, self.R = capacity, batch, K, seed, out_sets
@@ -1067,6 +1070,7 @@ class MmReplay(Workload):
         self.round_bytes = self.deliver_bytes + batch * 8 + self.ingest_bytes + \
             (self.demote_bytes if self.tiered else 0)
         self.launches_per_round = 2 + (3 if ingest else 0)  # + swap obs, swap tokens, metadata
+        self.launches_by_schedule = {"fused overlapped": 1}  # one fused launch per step
 
     def split_bytes(self):
         """Per-step bytes by where they move (two-tier only): over HBM, and
@@ -1603,6 +1607,9 @@ class ShardedPerReplay(PerReplay):
     each waits on the host for its routing counts, which size the
     all-to-alls."""
 
+    # total, routing, descent, delivery, batch minimum, weights, update
+    launches_per_round = 7
+
     def __init__(self, rank=0, **kw):
         super().__init__(**kw)
         self.sample_seed = self.seed
@@ -1664,6 +1671,8 @@ class ShardedPpoIteration(PpoIteration):
     def __init__(self, rank=0, **kw):
         super().__init__(**kw)
         self.seed = self.seed + 7919 * rank
+        # scan, statistics, normalisation, shuffle (3), delivery
+        self.launches_per_round = 7
 
     def setup(self, device):
         import torch
@@ -1957,7 +1966,8 @@ def run_edp(args):
                 "batches_per_s": K * world / (ms / 1e3),
                 "p50_sample_to_batch_us": p50,
                 "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
-                "gpu_launches": wl.launches_per_round * K,
+                "gpu_launches": wl.launches_by_schedule.get(scheds[0][0],
+                                                            wl.launches_per_round) * K,
                 "clocks": clk}
         if others:
             line["other_schedules"] = others
