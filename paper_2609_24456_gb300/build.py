@@ -102,6 +102,27 @@ def build_curand_probe(force: bool = False) -> str:
     return PROBE_LIB
 
 
+WAIT_PROBE_SRC = os.path.join(ROOT, "tests", "mbar_wait_probe.cu")
+WAIT_PROBE_LIB = os.path.join(ROOT, "tests", "_build", "mbar_wait_probe.so")
+
+
+def build_wait_probe(force: bool = False) -> str:
+    """Compile the tests' bounded-wait probe (test infrastructure, not part
+    of libedp): libedp's mbarrier wait helper run on its own."""
+    deps = [WAIT_PROBE_SRC, os.path.join(CSRC, "edp_internal.cuh"), os.path.abspath(__file__)]
+    if not force and not _stale(WAIT_PROBE_LIB, deps):
+        return WAIT_PROBE_LIB
+    os.makedirs(os.path.dirname(WAIT_PROBE_LIB), exist_ok=True)
+    tmp = WAIT_PROBE_LIB + ".tmp.%d" % os.getpid()
+    cmd = [nvcc()] + ARCH + ["-O2", "-std=c++17", "-shared", "-Xcompiler", "-fPIC",
+                             "-I", INCLUDE, "-I", CSRC, WAIT_PROBE_SRC, "-o", tmp]
+    p = subprocess.run(cmd, capture_output=True, text=True)
+    if p.returncode != 0:
+        raise RuntimeError("nvcc failed for %s:\n%s%s" % (WAIT_PROBE_SRC, p.stdout, p.stderr))
+    os.replace(tmp, WAIT_PROBE_LIB)
+    return WAIT_PROBE_LIB
+
+
 if __name__ == "__main__":
     print(build(force="--force" in sys.argv, verbose=True,
                 ptxas_v="--ptxas-v" in sys.argv))

@@ -330,7 +330,7 @@ __device__ __forceinline__ bool mbar_wait(unsigned long long *bar, uint32_t pari
   if (mbar_test(bar, parity)) return true;
   const uint64_t t0 = global_ns();
   for (;;) {
-    for (int i = 0; i < 64; ++i)
+    for (int i = 0; i < 8; ++i)  // a try_wait may itself suspend the thread
       if (mbar_test(bar, parity)) return true;
     if (global_ns() - t0 > limit_ns) return false;
   }

@@ -107,3 +107,43 @@ def test_dqn_host_pinned_ingest_source(edp_lib, orc):
         orc.ring_write(arr, cap, 0, np.ascontiguousarray(src))
     m.total = 100
     _deliver_and_check(edp, orc, m, 50, seed=1, rnd=2)
+
+
+@pytest.mark.parametrize("fw", [112, 560])
+def test_staged_stack_multi_piece_frames_and_bad_indices(edp_lib, orc, fw):
+    """Frames larger than one shared-memory stage (84 x 112 = 9,408 B in two
+    pieces, 84 x 560 = 47,040 B in seven) through the staged delivery (a
+    batch of 300 stacks fills the GPU), with episode ends and a wrapped ring;
+    slots outside the sampleable range (-1, capacity, the newest slot, whose
+    successor does not exist) give zero rows and a device flag, and every
+    other row equals the oracle's."""
+    edp = edp_lib
+    cap, n, B = 700, 900, 300
+    F = 84 * fw
+    frames, action, reward, done = fx.dqn_transitions(11, n, frame_bytes=F, done_p=0.1)
+    m = MirroredDqn(cap, F=F)
+    m.ingest(orc, frames[:500], action[:500], reward[:500], done[:500])
+    m.ingest(orc, frames[500:], action[500:], reward[500:], done[500:])
+    idx = torch.empty(B, dtype=torch.int64, device="cuda")
+    edp.edp_sample(m.ring.ctx, edp.EDP_SAMPLE_UNIFORM, B, 4, 0, idx)
+    newest = (m.total - 1) % cap
+    bad = {7: -1, 100: cap, 211: newest}
+    for k, v in bad.items():
+        idx[k] = v
+    obs, nxt, act, rew, dn = dqn_outputs(B, m.K, m.F)
+    edp.edp_deliver(m.ring.ctx, idx, B, edp.make_batch(obs, nxt, act, rew, dn))
+    st, msg = edp.edp_sync_status(m.ring.ctx)
+    assert st == edp.EDP_ERR_INVALID, msg
+    got = to_np(idx)
+    good = np.array([k for k in range(B) if k not in bad])
+    r_obs, r_nxt, r_act, r_rew, r_dn = orc.deliver_dqn(
+        m.frames, m.done, m.action, m.reward, m.cap, m.total, m.K, got[good])
+    o, x = bits(obs).reshape(B, -1), bits(nxt).reshape(B, -1)
+    assert np.array_equal(o[good], r_obs.reshape(len(good), -1).view(np.uint32))
+    assert np.array_equal(x[good], r_nxt.reshape(len(good), -1).view(np.uint32))
+    assert np.array_equal(to_np(act)[good], r_act)
+    assert np.array_equal(bits(rew)[good], r_rew.view(np.uint32))
+    assert np.array_equal(to_np(dn)[good], r_dn)
+    for k in bad:
+        assert not o[k].any() and not x[k].any(), k
+        assert to_np(act)[k] == 0 and bits(rew)[k] == 0 and to_np(dn)[k] == 0, k
