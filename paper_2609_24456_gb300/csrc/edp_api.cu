@@ -801,20 +801,27 @@ edp_status edp_ingest(edp_ctx *ctx, const edp_fields *src, uint64_t n,
     }
     if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_ingest(host tier)");
   }
+  // leaves whose tree sums change: the new ones and, with next_obs, the
+  // previous newest (its deferred priority lands now)
+  uint64_t tfirst = ctx->total % ctx->cap, tcount = n;
+  if (ctx->defer && ctx->total >= 1) {
+    tfirst = (ctx->total - 1) % ctx->cap;
+    tcount = n + 1;
+  }
+  if (tcount > ctx->cap) tcount = ctx->cap;
+  if (e == cudaSuccess && ingest_fusable(ctx, n)) {
+    // single tier, a moderate n: the whole insertion in one launch
+    e = launch_ingest_fused(ctx, &f, n, q, tfirst, ctx->depth ? tcount : 0, s);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_ingest");
+    ctx->total += n;
+    return EDP_OK;
+  }
   // metadata and leaves, then the tree above them, then the payload rows:
   // the row copy starts behind the (waiting) metadata and tree kernels and
-  // overlaps them, since neither reads the rows
+  // overlaps the last of them, since neither reads the rows
   const bool meta = ctx->st.action || ctx->st.reward || ctx->st.done || ctx->leaves;
   if (e == cudaSuccess) e = launch_ingest_meta(ctx, &f, n, q, s);
-  if (e == cudaSuccess && ctx->depth) {
-    uint64_t first = ctx->total % ctx->cap, count = n;
-    if (ctx->defer && ctx->total >= 1) {
-      first = (ctx->total - 1) % ctx->cap;
-      count = n + 1;
-    }
-    if (count > ctx->cap) count = ctx->cap;
-    e = launch_tree_refresh(ctx, first, count, s);
-  }
+  if (e == cudaSuccess && ctx->depth) e = launch_tree_refresh(ctx, tfirst, tcount, s);
   const uint64_t skip = new_hbm_lo - T, nh = Tn - new_hbm_lo;
   if (e == cudaSuccess && !swapped) {
     e = launch_copy_rows(ctx->st.obs, ctx->cap_h, new_hbm_lo % ctx->cap_h,

@@ -434,6 +434,20 @@ cudaError_t launch_grpo_pack(edp_ctx *ctx, const float *r, const uint64_t *goff,
                              uint64_t cap, cudaStream_t s);
 cudaError_t launch_tree_refresh(edp_ctx *ctx, uint64_t first_leaf,
                                 uint64_t count, cudaStream_t s);
+// Nodes of each level d that cover leaves [first, first + count) (mod the
+// capacity): [a0, a0 + n0) and, on a wrap, [a1, a1 + n1).
+struct TreeRanges {
+  uint64_t a0[kMaxDepth], n0[kMaxDepth], a1[kMaxDepth], n1[kMaxDepth];
+};
+void tree_ranges(const edp_ctx *ctx, uint64_t first, uint64_t count, TreeRanges *out);
+// A whole insertion in one launch (single-tier rings, n small enough):
+// metadata, leaves and the refresh of the tree above leaves
+// [tree_first, tree_first + tree_count) by one CTA, the payload rows by
+// the others.
+bool ingest_fusable(const edp_ctx *ctx, uint64_t n);
+cudaError_t launch_ingest_fused(edp_ctx *ctx, const edp_fields *f, uint64_t n,
+                                const uint32_t *q, uint64_t tree_first,
+                                uint64_t tree_count, cudaStream_t s);
 cudaError_t launch_tree_build_all(edp_ctx *ctx, cudaStream_t s);
 cudaError_t launch_sample_uniform(edp_ctx *ctx, uint32_t B, uint64_t seed,
                                   uint64_t round, int64_t *idx, cudaStream_t s);

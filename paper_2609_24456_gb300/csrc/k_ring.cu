@@ -31,21 +31,20 @@ struct CopyRuns {
   uint64_t end[3];  // cumulative word counts; unused runs repeat the total
 };
 
-__global__ void __launch_bounds__(kCopyThreads)
-k_copy_flat(CopyRuns r, int wait_first) {
-  if (wait_first) pdl_wait();
-  pdl_launch();
+// Tiles of kThr * kCopyFlat words of the runs, CTA `cta` of `ncta`: each
+// warp-wide access moves 512 contiguous bytes, a CTA's loads cover one
+// contiguous tile.
+template <int kThr>
+__device__ __forceinline__ void copy_tiles(const CopyRuns &r, uint64_t cta, uint64_t ncta) {
   const uint64_t total = r.end[2];  // unused runs repeat the last end
-  constexpr uint64_t kTile = (uint64_t)kCopyThreads * kCopyFlat;  // words per tile
+  constexpr uint64_t kTile = (uint64_t)kThr * kCopyFlat;  // words per tile
   const uint64_t tiles = (total + kTile - 1) / kTile;
-  // a CTA moves whole tiles: kCopyFlat warp-wide accesses of 512 contiguous
-  // bytes each per warp, the CTA's loads covering one contiguous tile
-  for (uint64_t t = blockIdx.x; t < tiles; t += gridDim.x) {
+  for (uint64_t t = cta; t < tiles; t += ncta) {
     const uint64_t i0 = t * kTile + threadIdx.x;
     uint4 v[kCopyFlat];
 #pragma unroll
     for (int u = 0; u < kCopyFlat; ++u) {
-      const uint64_t i = i0 + (uint64_t)u * kCopyThreads;
+      const uint64_t i = i0 + (uint64_t)u * kThr;
       if (i < total) {
         // run of word i, selected without indexing the parameter array
         // (which would place it in local memory)
@@ -56,7 +55,7 @@ k_copy_flat(CopyRuns r, int wait_first) {
     }
 #pragma unroll
     for (int u = 0; u < kCopyFlat; ++u) {
-      const uint64_t i = i0 + (uint64_t)u * kCopyThreads;
+      const uint64_t i = i0 + (uint64_t)u * kThr;
       if (i < total) {
         const bool g1 = i >= r.end[0], g2 = i >= r.end[1];
         const uint64_t o = g2 ? i - r.end[1] : (g1 ? i - r.end[0] : i);
@@ -64,7 +63,44 @@ k_copy_flat(CopyRuns r, int wait_first) {
       }
     }
   }
+}
+
+__global__ void __launch_bounds__(kCopyThreads)
+k_copy_flat(CopyRuns r, int wait_first) {
+  if (wait_first) pdl_wait();
+  pdl_launch();
+  copy_tiles<kCopyThreads>(r, blockIdx.x, gridDim.x);
   if (!wait_first) pdl_wait();
+}
+
+// The runs of rows (src_first + j) mod src_cap -> (dst_first + j) mod
+// dst_cap, j < n: contiguous between the wrap points of either side.
+CopyRuns row_runs(uint8_t *dst, uint64_t dst_cap, uint64_t dst_first, const uint8_t *src,
+                  uint64_t src_cap, uint64_t src_first, uint64_t n, uint64_t row_bytes) {
+  uint64_t cut[4] = {0, n, n, n};
+  int nc = 1;
+  const uint64_t jd = dst_cap - dst_first, js = src_cap - src_first;
+  for (uint64_t j : {jd < js ? jd : js, jd < js ? js : jd})
+    if (j > cut[nc - 1] && j < n) cut[nc++] = j;
+  cut[nc] = n;
+  CopyRuns r{};
+  uint64_t acc = 0;
+  for (int g = 0; g < nc; ++g) {
+    const uint64_t j0 = cut[g];
+    r.src[g] = reinterpret_cast<const uint4 *>(src + ((src_first + j0) % src_cap) * row_bytes);
+    r.dst[g] = reinterpret_cast<uint4 *>(dst + ((dst_first + j0) % dst_cap) * row_bytes);
+    acc += (cut[g + 1] - j0) * (row_bytes / 16);
+    r.end[g] = acc;
+  }
+  for (int g = nc; g < 3; ++g) r.end[g] = acc;
+  return r;
+}
+
+int sm_count() {
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  return sms > 0 ? sms : 1;
 }
 
 // Swap rows through HBM: HBM row (first + j) mod hbm_cap moves to host row
@@ -125,27 +161,10 @@ cudaError_t copy_rows(uint8_t *dst, uint64_t dst_cap, uint64_t dst_first,
                       const uint8_t *src, uint64_t src_cap, uint64_t src_first,
                       uint64_t n, uint64_t row_bytes, cudaStream_t s, bool wait_first) {
   if (!n) return cudaSuccess;
-  uint64_t cut[4] = {0, n, n, n};
-  int nc = 1;
-  const uint64_t jd = dst_cap - dst_first, js = src_cap - src_first;
-  for (uint64_t j : {jd < js ? jd : js, jd < js ? js : jd})
-    if (j > cut[nc - 1] && j < n) cut[nc++] = j;
-  cut[nc] = n;
-  CopyRuns r{};
-  uint64_t acc = 0;
-  for (int g = 0; g < nc; ++g) {
-    const uint64_t j0 = cut[g];
-    r.src[g] = reinterpret_cast<const uint4 *>(src + ((src_first + j0) % src_cap) * row_bytes);
-    r.dst[g] = reinterpret_cast<uint4 *>(dst + ((dst_first + j0) % dst_cap) * row_bytes);
-    acc += (cut[g + 1] - j0) * (row_bytes / 16);
-    r.end[g] = acc;
-  }
-  for (int g = nc; g < 3; ++g) r.end[g] = acc;
-  int dev = 0, sms = 0;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const CopyRuns r = row_runs(dst, dst_cap, dst_first, src, src_cap, src_first, n, row_bytes);
+  const uint64_t acc = r.end[2];
   uint64_t blocks = (acc + (uint64_t)kCopyThreads * kCopyFlat - 1) / ((uint64_t)kCopyThreads * kCopyFlat);
-  const uint64_t most = (uint64_t)kCopyCtasPerSm * (sms > 0 ? sms : 1);
+  const uint64_t most = (uint64_t)kCopyCtasPerSm * sm_count();
   if (blocks > most) blocks = most;
   return launch_pdl(k_copy_flat, dim3((unsigned)blocks), dim3(kCopyThreads), s, r,
                     wait_first ? 1 : 0);
@@ -155,47 +174,106 @@ cudaError_t copy_rows(uint8_t *dst, uint64_t dst_cap, uint64_t dst_first,
 // leaves.  With `defer` the newest transition's leaf stays 0 and its
 // priority waits in ctrl->pending_q; the previous newest (id total-1) gets
 // its pending priority now -- unless this insertion overwrites its slot.
-__global__ void k_ingest_meta(int32_t *__restrict__ action,
-                              float *__restrict__ reward,
-                              uint8_t *__restrict__ done,
-                              const int32_t *__restrict__ s_action,
-                              const float *__restrict__ s_reward,
-                              const uint8_t *__restrict__ s_done,
-                              uint32_t *__restrict__ leaves,
-                              const uint32_t *__restrict__ q, Ctrl *ctrl,
-                              uint64_t cap, uint64_t total, uint64_t n,
-                              int defer) {
-  pdl_wait();
-  pdl_launch();
+struct MetaArgs {
+  int32_t *action;
+  float *reward;
+  uint8_t *done;
+  const int32_t *s_action;
+  const float *s_reward;
+  const uint8_t *s_done;
+  uint32_t *leaves;
+  const uint32_t *q;
+  Ctrl *ctrl;
+  uint64_t cap, total, n;
+  int defer;
+};
+
+// Transitions j = j0, j0 + stride, ... of the insertion.
+__device__ __forceinline__ void ingest_meta_range(const MetaArgs &a, uint64_t j0,
+                                                  uint64_t stride) {
   uint32_t qdefault = 0;
-  if (leaves && !q) qdefault = ctrl->max_q;
+  if (a.leaves && !a.q) qdefault = a.ctrl->max_q;
   uint32_t qmax_local = 0;  // one atomic per warp, not per transition
-  for (uint64_t j = blockIdx.x * (uint64_t)blockDim.x + threadIdx.x; j < n;
-       j += (uint64_t)gridDim.x * blockDim.x) {
-    const uint64_t m = (total + j) % cap;
-    if (action) action[m] = s_action ? s_action[j] : 0;
-    if (reward) reward[m] = s_reward ? s_reward[j] : 0.f;
-    if (done) done[m] = s_done ? s_done[j] : (uint8_t)0;
-    if (leaves) {
-      const uint32_t qj = q ? q[j] : qdefault;
-      if (q) qmax_local = max(qmax_local, qj);
-      if (defer) {
-        leaves[m] = (j == n - 1) ? 0u : qj;
+  for (uint64_t j = j0; j < a.n; j += stride) {
+    const uint64_t m = (a.total + j) % a.cap;
+    if (a.action) a.action[m] = a.s_action ? a.s_action[j] : 0;
+    if (a.reward) a.reward[m] = a.s_reward ? a.s_reward[j] : 0.f;
+    if (a.done) a.done[m] = a.s_done ? a.s_done[j] : (uint8_t)0;
+    if (a.leaves) {
+      const uint32_t qj = a.q ? a.q[j] : qdefault;
+      if (a.q) qmax_local = max(qmax_local, qj);
+      if (a.defer) {
+        a.leaves[m] = (j == a.n - 1) ? 0u : qj;
         if (j == 0) {
           // only this thread touches pending_q and the previous newest leaf
-          if (total >= 1 && n < cap) leaves[(total - 1) % cap] = ctrl->pending_q;
-          ctrl->pending_q = q ? q[n - 1] : qdefault;
+          if (a.total >= 1 && a.n < a.cap)
+            a.leaves[(a.total - 1) % a.cap] = a.ctrl->pending_q;
+          a.ctrl->pending_q = a.q ? a.q[a.n - 1] : qdefault;
         }
       } else {
-        leaves[m] = qj;
+        a.leaves[m] = qj;
       }
     }
   }
-  if (leaves && q) {
+  if (a.leaves && a.q) {
 #pragma unroll
     for (int o = 16; o; o >>= 1)
       qmax_local = max(qmax_local, __shfl_xor_sync(0xffffffffu, qmax_local, o));
-    if ((threadIdx.x & 31) == 0 && qmax_local) atomicMax(&ctrl->max_q, qmax_local);
+    if ((threadIdx.x & 31) == 0 && qmax_local) atomicMax(&a.ctrl->max_q, qmax_local);
+  }
+}
+
+__global__ void k_ingest_meta(MetaArgs a) {
+  pdl_wait();
+  pdl_launch();
+  ingest_meta_range(a, blockIdx.x * (uint64_t)blockDim.x + threadIdx.x,
+                    (uint64_t)gridDim.x * blockDim.x);
+}
+
+// One insertion in one launch (replay rings: a single HBM tier, at most
+// kFusedMaxRows rows).  CTA 0 writes the metadata and leaves, then refreshes
+// the tree above them level by level (a CTA barrier between levels, so each
+// level reads the sums written below it); the other CTAs copy the payload
+// rows (obs, then tokens).  Nothing of the two parts reads what the other
+// writes, so the metadata chain runs beside the copy.
+constexpr int kFusedThreads = 1024;
+constexpr uint64_t kFusedMaxRows = 16384;
+
+struct TreeRefresh {
+  uint64_t *level[kMaxDepth];  // level d: 32^d sums
+  uint32_t *leaves;
+  uint32_t depth;
+  // nodes of level d to recompute: [a0, a0 + n0) and [a1, a1 + n1)
+  uint64_t a0[kMaxDepth], n0[kMaxDepth], a1[kMaxDepth], n1[kMaxDepth];
+};
+
+__global__ void __launch_bounds__(kFusedThreads, 1)
+k_ingest_fused(CopyRuns obs, CopyRuns tok, MetaArgs meta, TreeRefresh t) {
+  pdl_wait();
+  pdl_launch();
+  if (blockIdx.x != 0) {
+    copy_tiles<kFusedThreads>(obs, blockIdx.x - 1, gridDim.x - 1);
+    copy_tiles<kFusedThreads>(tok, blockIdx.x - 1, gridDim.x - 1);
+    return;
+  }
+  ingest_meta_range(meta, threadIdx.x, kFusedThreads);
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  constexpr int kWarps = kFusedThreads / 32;
+#pragma unroll
+  for (int d = kMaxDepth - 1; d >= 0; --d) {  // constant indices into t
+    if ((uint32_t)d >= t.depth) continue;
+    __syncthreads();  // the level below (or the leaves) is written
+    const bool leaves_below = (uint32_t)d + 1 == t.depth;
+    const uint64_t n = t.n0[d] + t.n1[d];
+    for (uint64_t w = warp; w < n; w += kWarps) {
+      const uint64_t node = w < t.n0[d] ? t.a0[d] + w : t.a1[d] + (w - t.n0[d]);
+      const uint64_t c = node * kFanout + lane;
+      uint64_t v = leaves_below ? (uint64_t)__ldcg(t.leaves + c)
+                                : __ldcg(t.level[d + 1 < kMaxDepth ? d + 1 : d] + c);
+#pragma unroll
+      for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+      if (lane == 0) t.level[d][node] = v;
+    }
   }
 }
 
@@ -235,6 +313,26 @@ cudaError_t launch_copy_rows(uint8_t *dst, uint64_t dst_cap, uint64_t first,
   return copy_rows(dst, dst_cap, first, src, ~0ull, 0, n, row_bytes, s, wait_first);
 }
 
+namespace {
+MetaArgs meta_args(edp_ctx *c, const edp_fields *f, uint64_t n, const uint32_t *q) {
+  MetaArgs a{};
+  a.action = c->st.action;
+  a.reward = c->st.reward;
+  a.done = c->st.done;
+  a.s_action = f->action;
+  a.s_reward = f->reward;
+  a.s_done = f->done;
+  a.leaves = c->leaves;
+  a.q = q;
+  a.ctrl = c->ctrl;
+  a.cap = c->cap;
+  a.total = c->total;
+  a.n = n;
+  a.defer = c->defer;
+  return a;
+}
+}  // namespace
+
 cudaError_t launch_ingest_meta(edp_ctx *c, const edp_fields *f, uint64_t n,
                                const uint32_t *q, cudaStream_t s) {
   if (!c->st.action && !c->st.reward && !c->st.done && !c->leaves)
@@ -243,8 +341,43 @@ cudaError_t launch_ingest_meta(edp_ctx *c, const edp_fields *f, uint64_t n,
   uint64_t blocks = (n + threads - 1) / threads;
   if (blocks > 4096) blocks = 4096;
   return launch_pdl(k_ingest_meta, dim3((unsigned)blocks), dim3(threads), s,
-                    c->st.action, c->st.reward, c->st.done, f->action, f->reward, f->done,
-                    c->leaves, q, c->ctrl, c->cap, c->total, n, c->defer);
+                    meta_args(c, f, n, q));
+}
+
+bool ingest_fusable(const edp_ctx *c, uint64_t n) {
+  return c->cap_c == 0 && n <= kFusedMaxRows;
+}
+
+cudaError_t launch_ingest_fused(edp_ctx *c, const edp_fields *f, uint64_t n,
+                                const uint32_t *q, uint64_t tree_first, uint64_t tree_count,
+                                cudaStream_t s) {
+  const uint64_t first = c->total % c->cap_h;
+  const CopyRuns obs = row_runs(c->st.obs, c->cap_h, first, f->obs, ~0ull, 0, n, c->obs_bytes);
+  CopyRuns tok{};
+  if (c->tok_bytes)
+    tok = row_runs((uint8_t *)c->st.tokens, c->cap_h, first, (const uint8_t *)f->tokens, ~0ull,
+                   0, n, c->tok_bytes);
+  TreeRefresh t{};
+  if (c->depth && tree_count) {
+    TreeRanges tr;
+    tree_ranges(c, tree_first, tree_count, &tr);
+    t.depth = c->depth;
+    t.leaves = c->leaves;
+    for (uint32_t d = 0; d < c->depth; ++d) {
+      t.level[d] = c->level[d];
+      t.a0[d] = tr.a0[d];
+      t.n0[d] = tr.n0[d];
+      t.a1[d] = tr.a1[d];
+      t.n1[d] = tr.n1[d];
+    }
+  }
+  const uint64_t words = obs.end[2] + tok.end[2];
+  uint64_t blocks = (words + (uint64_t)kFusedThreads * kCopyFlat - 1) /
+                    ((uint64_t)kFusedThreads * kCopyFlat);
+  const uint64_t most = 2ull * sm_count();
+  if (blocks > most) blocks = most;
+  return launch_pdl(k_ingest_fused, dim3((unsigned)(blocks + 1)), dim3(kFusedThreads), s, obs,
+                    tok, meta_args(c, f, n, q), t);
 }
 
 // Two-tier demotion: payload of ids [first_id, first_id+n) moves from HBM

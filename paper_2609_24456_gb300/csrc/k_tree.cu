@@ -395,9 +395,7 @@ k_update(TreeView t, const int64_t *__restrict__ idx,
 
 }  // namespace
 
-cudaError_t launch_tree_refresh(edp_ctx *c, uint64_t first, uint64_t count,
-                                cudaStream_t s) {
-  if (!c->depth || !count) return cudaSuccess;
+void tree_ranges(const edp_ctx *c, uint64_t first, uint64_t count, TreeRanges *out) {
   // leaf ranges [a0, b0) and [a1, b1) (the second only on ring wrap)
   uint64_t a0 = first, b0 = first + count, a1 = 0, b1 = 0;
   if (b0 > c->cap) {
@@ -417,7 +415,20 @@ cudaError_t launch_tree_refresh(edp_ctx *c, uint64_t first, uint64_t count,
         x1 = y1 = 0;
       }
     }
-    const uint64_t nodes = (y0 - x0) + (y1 - x1);
+    out->a0[d] = x0;
+    out->n0[d] = y0 - x0;
+    out->a1[d] = x1;
+    out->n1[d] = y1 - x1;
+  }
+}
+
+cudaError_t launch_tree_refresh(edp_ctx *c, uint64_t first, uint64_t count,
+                                cudaStream_t s) {
+  if (!c->depth || !count) return cudaSuccess;
+  TreeRanges r;
+  tree_ranges(c, first, count, &r);
+  for (int d = (int)c->depth - 1; d >= 0; --d) {
+    const uint64_t nodes = r.n0[d] + r.n1[d];
     const uint64_t threads = nodes * 32;
     const unsigned blocks = (unsigned)((threads + 255) / 256);
     const bool leaves_below = (uint32_t)(d + 1) == c->depth;
@@ -426,7 +437,7 @@ cudaError_t launch_tree_refresh(edp_ctx *c, uint64_t first, uint64_t count,
                                             : (const uint64_t *)c->level[d + 1],
                                leaves_below ? (const uint32_t *)c->leaves
                                             : (const uint32_t *)nullptr,
-                               x0, y0 - x0, x1, y1 - x1);
+                               r.a0[d], r.n0[d], r.a1[d], r.n1[d]);
     if (e != cudaSuccess) return e;
   }
   return cudaSuccess;

@@ -51,6 +51,9 @@ class ShardComm:
         """[world * n] from every rank's [n] (rank order)."""
         import torch
         src = self._out(t.contiguous())
+        if out is not None and not self.host:
+            self.dist.all_gather_into_tensor(out, src, group=self.group)
+            return out
         res = torch.empty(self.world * src.numel(), dtype=src.dtype, device=src.device)
         self.dist.all_gather_into_tensor(res, src, group=self.group)
         return self._back(t, res, out)
@@ -61,13 +64,17 @@ class ShardComm:
         arrive in rank order."""
         import torch
         src = self._out(t.contiguous())
-        res = torch.empty((sum(recv_counts),) + tuple(src.shape[1:]), dtype=src.dtype,
-                          device=src.device)
+        n = sum(recv_counts)
+        if out is not None and not self.host:
+            res = out[:n]  # received in place (a leading slice is contiguous)
+        else:
+            res = torch.empty((n,) + tuple(src.shape[1:]), dtype=src.dtype, device=src.device)
         self.dist.all_to_all_single(res, src, output_split_sizes=list(recv_counts),
                                     input_split_sizes=list(send_counts), group=self.group)
         if out is not None:
-            out[:res.shape[0]].copy_(res)
-            return out[:res.shape[0]]
+            if res.data_ptr() != out.data_ptr() or res.device != out.device:
+                out[:n].copy_(res)
+            return out[:n]
         return self._back(t, res)
 
     def all_reduce(self, t, op):
