@@ -565,6 +565,33 @@ EDP_API edp_status edp_load(edp_ctx *ctx, const char *path, edp_stream stream);
  * for a NULL argument. */
 EDP_API edp_status edp_get_info(const edp_ctx *ctx, edp_info *out);
 
+/* Per-context traffic counters (no counterpart in the paper, whose metrics
+ * are latencies).  Counts accumulate from context creation or the last
+ * edp_reset_counters, at enqueue time, for every call that enqueued work.
+ * Byte counts are algorithmic, the bytes the path must move: the payload
+ * rows and metadata an insertion reads from its source and writes to the
+ * ring (demotions included), the source bytes a delivery reads and the
+ * outputs it writes, and the index / priority arrays of sampling and
+ * updates.  Every count is split by where the bytes live: device memory
+ * (hbm_*) or page-locked host memory reached over the host link (link_*).
+ * The tier of a two-tier delivery's rows depends on the sampled slots, so
+ * its kernel counts its host-tier rows on the device; edp_get_counters
+ * reads that count, which is exact once the deliveries have completed
+ * (e.g. after edp_sync).  Not counted: a packed delivery's tokens, whose
+ * number is only known on the device, and traffic inside the priority tree.
+ * EDP_ERR_INVALID for a NULL argument; EDP_ERR_CUDA when the device count
+ * cannot be read. */
+typedef struct {
+  uint64_t calls;       /* calls that enqueued work */
+  uint64_t ingested;    /* transitions inserted */
+  uint64_t sampled;     /* indices drawn (sampling, fused sampling) */
+  uint64_t delivered;   /* batch entries delivered */
+  uint64_t hbm_read, hbm_write;    /* bytes read from / written to device memory */
+  uint64_t link_read, link_write;  /* bytes read from / written to host memory */
+} edp_counters;
+EDP_API edp_status edp_get_counters(edp_ctx *ctx, edp_counters *out);
+EDP_API edp_status edp_reset_counters(edp_ctx *ctx);
+
 /* Host-link probe: streams `bytes` (a multiple of 16) of page-locked host
  * memory through the GPU with 16-byte loads, xor-folding them into
  * *d_fold (device uint64).  Used to measure achievable host-link read

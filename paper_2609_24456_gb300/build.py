@@ -75,7 +75,7 @@ def build(force: bool = False, verbose: bool = False, ptxas_v: bool = False) -> 
                 print(log)
     objs = [o for o, _ in results]
     tmp = LIB + ".tmp.%d" % os.getpid()
-    cmd = [cc] + ARCH + ["-shared", "-cudart", "static", "-o", tmp] + objs
+    cmd = [cc] + ARCH + ["-shared", "-cudart", "static", "-o", tmp] + objs + ["-ldl"]
     p = subprocess.run(cmd, capture_output=True, text=True)
     if p.returncode != 0:
         raise RuntimeError("link failed:\n%s%s" % (p.stdout, p.stderr))

@@ -186,6 +186,32 @@ bool edp::device_view(const edp_ctx *c, const void *p, const void **out,
   return false;
 }
 
+bool edp::host_memory(const void *p) {
+  if (!p) return false;
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return a.type == cudaMemoryTypeHost;
+}
+
+namespace {
+// Traffic counters: bytes at p (device or page-locked host memory).
+void count_read(edp_ctx *c, const void *p, uint64_t bytes) {
+  if (p && bytes) (host_memory(p) ? c->cnt.link_read : c->cnt.hbm_read) += bytes;
+}
+void count_write(edp_ctx *c, const void *p, uint64_t bytes) {
+  if (p && bytes) (host_memory(p) ? c->cnt.link_write : c->cnt.hbm_write) += bytes;
+}
+// Device-resident arrays of a call (index, priority and scalar arrays).
+void count_hbm(edp_ctx *c, uint64_t read, uint64_t write) {
+  c->cnt.hbm_read += read;
+  c->cnt.hbm_write += write;
+  ++c->cnt.calls;
+}
+}  // namespace
+
 edp_status edp::launch_fail(edp_ctx *c, cudaError_t e, const char *where) {
   if (e == cudaErrorMemoryAllocation)
     return fail(c, EDP_ERR_OOM, "%s: scratch allocation failed", where);
@@ -329,6 +355,7 @@ edp_status edp_create(const edp_config *cfg, const edp_storage *st,
     return bad("no CUDA device %d", cfg->device);
   }
   DeviceGuard dg(cfg->device);
+  EDP_TRACE(__func__);
   if (!dg.ok()) return bad("cudaSetDevice failed");
   c->cap = cfg->capacity;
   c->cap_h = cfg->hbm_capacity;
@@ -435,6 +462,7 @@ edp_status edp_create(const edp_config *cfg, const edp_storage *st,
 edp_status edp_destroy(edp_ctx *ctx) {
   if (!ctx) return EDP_ERR_INVALID;
   DeviceGuard dg(ctx->cfg.device);
+  EDP_TRACE(__func__);
   cudaDeviceSynchronize();
   free_all(ctx);
   delete ctx;
@@ -457,6 +485,7 @@ edp_status edp_migrate(const edp_ctx *src, edp_ctx *dst, edp_stream stream) {
       (src->st.done != nullptr) != (dst->st.done != nullptr))
     return fail(dst, EDP_ERR_STATE, "edp_migrate: metadata arrays differ");
   DeviceGuard dg(b.device);
+  EDP_TRACE(__func__);
   cudaStream_t s = (cudaStream_t)stream;
   const uint64_t size = ring_size(src);
   const uint64_t n = size < dst->cap ? size : dst->cap;
@@ -552,6 +581,7 @@ edp_status edp_save(edp_ctx *ctx, const char *path, edp_stream stream) {
   if (!ctx) return EDP_ERR_INVALID;
   if (!path) return fail(ctx, EDP_ERR_INVALID, "edp_save: path is NULL");
   DeviceGuard dg(ctx->cfg.device);
+  EDP_TRACE(__func__);
   cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_save");
   CkptHeader h{};
@@ -643,6 +673,7 @@ edp_status edp_load(edp_ctx *ctx, const char *path, edp_stream stream) {
                 have, (unsigned long long)want);
   }
   DeviceGuard dg(ctx->cfg.device);
+  EDP_TRACE(__func__);
   const uint64_t n = h.n < ctx->cap ? h.n : ctx->cap;  // the newest n are kept
   const uint64_t skip = h.n - n;
   uint8_t *stage = (uint8_t *)std::malloc(kStage);
@@ -735,6 +766,7 @@ edp_status edp_ingest(edp_ctx *ctx, const edp_fields *src, uint64_t n,
                 (unsigned long long)n);
   if (n == 0) return EDP_OK;
   DeviceGuard dg(ctx->cfg.device);
+  EDP_TRACE(__func__);
   cudaStream_t s = (cudaStream_t)stream;
   edp_fields f{};
   const void *p;
@@ -775,6 +807,7 @@ edp_status edp_ingest(edp_ctx *ctx, const edp_fields *src, uint64_t n,
   const uint64_t keep = Tn < ctx->cap ? Tn : ctx->cap;
   uint64_t new_hbm_lo = T;
   bool swapped = false;
+  uint64_t demoted = 0, to_host = 0;  // rows moved into the host tier
   if (ctx->cap_c) {
     const uint64_t in_hbm = T < ctx->cap_h ? T : ctx->cap_h;
     uint64_t lo = T - in_hbm;
@@ -789,6 +822,8 @@ edp_status edp_ingest(edp_ctx *ctx, const edp_fields *src, uint64_t n,
     // directions at once
     swapped = hi > lo && dhi <= dlo && hi - lo == Tn - new_hbm_lo &&
               lo + ctx->cap_h == new_hbm_lo;
+    demoted = hi > lo ? hi - lo : 0;
+    to_host = dhi > dlo ? dhi - dlo : 0;
     if (swapped) {
       const uint64_t skip = new_hbm_lo - T;
       e = launch_swap(ctx, lo, f.obs + skip * ctx->obs_bytes,
@@ -809,10 +844,30 @@ edp_status edp_ingest(edp_ctx *ctx, const edp_fields *src, uint64_t n,
     tcount = n + 1;
   }
   if (tcount > ctx->cap) tcount = ctx->cap;
+  // traffic: source rows and metadata read; ring rows written to their
+  // tier (demoted rows read from HBM and written to the host); metadata
+  // and leaves written to HBM
+  auto count_ingest = [&]() {
+    const uint64_t R = ctx->obs_bytes + ctx->tok_bytes;
+    count_read(ctx, src->obs, n * ctx->obs_bytes);
+    count_read(ctx, src->tokens, n * ctx->tok_bytes);
+    count_read(ctx, src->action, 4 * n);
+    count_read(ctx, src->reward, 4 * n);
+    count_read(ctx, src->done, n);
+    count_read(ctx, q, 4 * n);
+    ctx->cnt.hbm_write += (n - to_host) * R;
+    ctx->cnt.link_write += (to_host + demoted) * R;
+    ctx->cnt.hbm_read += demoted * R;
+    ctx->cnt.hbm_write += n * (4 * (ctx->st.action != nullptr) + 4 * (ctx->st.reward != nullptr) +
+                               (ctx->st.done != nullptr) + 4 * (ctx->leaves != nullptr));
+    ctx->cnt.ingested += n;
+    ++ctx->cnt.calls;
+  };
   if (e == cudaSuccess && ingest_fusable(ctx, n)) {
     // single tier, a moderate n: the whole insertion in one launch
     e = launch_ingest_fused(ctx, &f, n, q, tfirst, ctx->depth ? tcount : 0, s);
     if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_ingest");
+    count_ingest();
     ctx->total += n;
     return EDP_OK;
   }
@@ -833,6 +888,7 @@ edp_status edp_ingest(edp_ctx *ctx, const edp_fields *src, uint64_t n,
                            ctx->tok_bytes, s, false);  // behind the row copy
   }
   if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_ingest");
+  count_ingest();
   ctx->total += n;
   return EDP_OK;
 }
@@ -847,6 +903,7 @@ edp_status edp_sample(edp_ctx *ctx, edp_sample_mode mode, uint32_t batch,
   if (!device_view(ctx, idx, &p, false) || (q && !device_view(ctx, q, &p, false)))
     return fail(ctx, EDP_ERR_INVALID, "edp_sample: outputs must be device memory");
   DeviceGuard dg(ctx->cfg.device);
+  EDP_TRACE(__func__);
   cudaStream_t s = (cudaStream_t)stream;
   cudaError_t e;
   switch (mode) {
@@ -875,6 +932,8 @@ edp_status edp_sample(edp_ctx *ctx, edp_sample_mode mode, uint32_t batch,
       return fail(ctx, EDP_ERR_INVALID, "edp_sample: unknown mode %d", (int)mode);
   }
   if (e != cudaSuccess) return launch_fail(ctx, e, "edp_sample");
+  count_hbm(ctx, 0, 8ull * batch + (q && mode == EDP_SAMPLE_PRIORITIZED ? 4ull * batch : 0));
+  ctx->cnt.sampled += batch;
   return EDP_OK;
 }
 
@@ -931,6 +990,39 @@ static edp_status deliver_checks(edp_ctx *ctx, const int64_t *idx, uint32_t batc
   return EDP_OK;
 }
 
+// Traffic of a delivery of B entries into `out` (the caller's pointers):
+// per entry the unique source bytes (the K or K + 1 frames of a stack, the
+// image and tokens otherwise) and the scalars read, and every output
+// written to its memory.  A two-tier ring's host rows are counted on the
+// device and moved to link_read by edp_get_counters.
+static void count_deliver(edp_ctx *ctx, uint32_t B, const edp_batch *out) {
+  const auto &cfg = ctx->cfg;
+  const uint64_t F = ctx->obs_bytes;
+  uint64_t per = F, obs_out = 0;
+  if (cfg.transform == EDP_XFORM_STACK_F32) {
+    per = F * (cfg.frame_stack + (out->next_obs ? 1 : 0));
+    obs_out = F * cfg.frame_stack * 4;
+  } else {
+    per = F + (out->tokens ? ctx->tok_bytes : 0);
+    obs_out = F * 2;
+  }
+  const uint64_t scalars = 8 + 4 * (out->action != nullptr) + 4 * (out->reward != nullptr) +
+                           (out->done != nullptr) + 4 * (out->q != nullptr) +
+                           4 * (out->gather_src[0] != nullptr) + 4 * (out->gather_src[1] != nullptr);
+  ctx->cnt.hbm_read += B * (per + scalars);
+  count_write(ctx, out->obs, B * obs_out);
+  count_write(ctx, out->next_obs, B * obs_out);
+  count_write(ctx, out->tokens, B * ctx->tok_bytes);
+  count_write(ctx, out->action, 4ull * B);
+  count_write(ctx, out->reward, 4ull * B);
+  count_write(ctx, out->done, 1ull * B);
+  count_write(ctx, out->isw, 4ull * B);
+  count_write(ctx, out->gather_dst[0], 4ull * B);
+  count_write(ctx, out->gather_dst[1], 4ull * B);
+  ctx->cnt.delivered += B;
+  ++ctx->cnt.calls;
+}
+
 edp_status edp_deliver(edp_ctx *ctx, const int64_t *idx, uint32_t batch,
                        const edp_batch *out, edp_stream stream) {
   if (!ctx) return EDP_ERR_INVALID;
@@ -938,8 +1030,10 @@ edp_status edp_deliver(edp_ctx *ctx, const int64_t *idx, uint32_t batch,
   const edp_status st = deliver_checks(ctx, idx, batch, out, &res);
   if (st != EDP_OK) return st;
   DeviceGuard dg(ctx->cfg.device);
+  EDP_TRACE(__func__);
   cudaError_t e = launch_deliver(ctx, idx, batch, &res, (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_deliver");
+  count_deliver(ctx, batch, out);
   return EDP_OK;
 }
 
@@ -955,9 +1049,14 @@ edp_status edp_sample_deliver(edp_ctx *ctx, uint32_t batch, uint64_t seed, uint6
   const edp_status st = deliver_checks(ctx, idx, batch, out, &res);
   if (st != EDP_OK) return st;
   DeviceGuard dg(ctx->cfg.device);
+  EDP_TRACE(__func__);
   DrawUniform d{seed, round, idx};
   cudaError_t e = launch_deliver(ctx, idx, batch, &res, (cudaStream_t)stream, &d);
   if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_sample_deliver");
+  count_deliver(ctx, batch, out);  // the drawn indices are written, not read:
+  ctx->cnt.hbm_read -= 8ull * batch;  // the index bytes count once, as a write
+  ctx->cnt.hbm_write += 8ull * batch;
+  ctx->cnt.sampled += batch;
   return EDP_OK;
 }
 
@@ -967,8 +1066,10 @@ static edp_status update_common(edp_ctx *ctx, const char *who, const int64_t *id
   const edp_status st = update_args(ctx, who, idx, q, td, n, alpha, eps);
   if (st != EDP_OK || n == 0) return st;
   DeviceGuard dg(ctx->cfg.device);
+  EDP_TRACE(who);
   cudaError_t e = launch_update(ctx, idx, q, td, alpha, eps, n, (cudaStream_t)stream);
   if (e != cudaSuccess) return launch_fail(ctx, e, who);
+  count_hbm(ctx, 12ull * n, 4ull * n);  // pairs read, leaves written
   return EDP_OK;
 }
 
@@ -998,8 +1099,10 @@ edp_status edp_priorities_from_td(edp_ctx *ctx, const float *td, uint32_t n,
   if (!(alpha >= 0.0 && eps >= 0.0))
     return fail(ctx, EDP_ERR_INVALID, "edp_priorities_from_td: alpha, eps >= 0");
   DeviceGuard dg(ctx->cfg.device);
+  EDP_TRACE(__func__);
   cudaError_t e = launch_prio_from_td(td, n, alpha, eps, q, (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_priorities_from_td");
+  count_hbm(ctx, 4ull * n, 4ull * n);
   return EDP_OK;
 }
 
@@ -1019,9 +1122,13 @@ edp_status edp_gae(edp_ctx *ctx, const float *r, const float *v,
     if (o && !device_view(ctx, o, &p, false))
       return fail(ctx, EDP_ERR_INVALID, "edp_gae: arrays must be device memory");
   DeviceGuard dg(ctx->cfg.device);
+  EDP_TRACE(__func__);
   cudaError_t e = launch_gae(ctx, r, v, d, T, E, gamma, lambda, adv, ret, adv_norm,
                              (cudaStream_t)stream);
   if (e != cudaSuccess) return launch_fail(ctx, e, "edp_gae");
+  const uint64_t te = (uint64_t)T * E;
+  count_hbm(ctx, 9 * te + 4ull * E,
+            4 * te * ((adv != nullptr) + (ret != nullptr) + (adv_norm != nullptr)));
   return EDP_OK;
 }
 
@@ -1041,8 +1148,10 @@ edp_status edp_tree_total(edp_ctx *ctx, uint64_t *d_total, edp_stream stream) {
   if (!d_total || !all_device(ctx, {d_total}))
     return fail(ctx, EDP_ERR_INVALID, "edp_tree_total: d_total must be device memory");
   DeviceGuard dg(ctx->cfg.device);
+  EDP_TRACE(__func__);
   cudaError_t e = launch_tree_total(ctx, d_total, (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_tree_total");
+  count_hbm(ctx, 8, 8);
   return EDP_OK;
 }
 
@@ -1061,9 +1170,11 @@ edp_status edp_route_prioritized(edp_ctx *ctx, const uint64_t *d_totals, uint32_
     return fail(ctx, EDP_ERR_INVALID,
                 "edp_route_prioritized: totals, local targets and counts must be device memory");
   DeviceGuard dg(ctx->cfg.device);
+  EDP_TRACE(__func__);
   cudaError_t e = launch_route_prioritized(ctx, d_totals, G, batch, k0, n, seed, round,
                                            d_local_t, d_counts, (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_route_prioritized");
+  count_hbm(ctx, 8ull * G, 8ull * n + 8ull * G);
   return EDP_OK;
 }
 
@@ -1077,8 +1188,11 @@ edp_status edp_sample_targets(edp_ctx *ctx, const uint64_t *d_targets, uint32_t 
     return fail(ctx, EDP_ERR_INVALID,
                 "edp_sample_targets: targets, idx and q must be device memory");
   DeviceGuard dg(ctx->cfg.device);
+  EDP_TRACE(__func__);
   cudaError_t e = launch_sample_targets(ctx, d_targets, n, d_idx, d_q, (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_sample_targets");
+  count_hbm(ctx, 8ull * n, (d_q ? 12ull : 8ull) * n);
+  ctx->cnt.sampled += n;
   return EDP_OK;
 }
 
@@ -1088,8 +1202,10 @@ edp_status edp_batch_qmin(edp_ctx *ctx, const uint32_t *d_q, uint32_t n, int64_t
   if (!d_qmin || (n && !d_q) || !all_device(ctx, {d_q, d_qmin}))
     return fail(ctx, EDP_ERR_INVALID, "edp_batch_qmin: q and qmin must be device memory");
   DeviceGuard dg(ctx->cfg.device);
+  EDP_TRACE(__func__);
   cudaError_t e = launch_batch_qmin(ctx, d_q, n, d_qmin, (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_batch_qmin");
+  count_hbm(ctx, 4ull * n, 8);
   return EDP_OK;
 }
 
@@ -1101,8 +1217,10 @@ edp_status edp_is_weights(edp_ctx *ctx, const uint32_t *d_q, uint32_t n,
   if (!d_q || !d_qmin || !d_w || !all_device(ctx, {d_q, d_qmin, d_w}))
     return fail(ctx, EDP_ERR_INVALID, "edp_is_weights: q, qmin and w must be device memory");
   DeviceGuard dg(ctx->cfg.device);
+  EDP_TRACE(__func__);
   cudaError_t e = launch_is_weights(ctx, d_q, n, d_qmin, beta, d_w, (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_is_weights");
+  count_hbm(ctx, 4ull * n + 8, 4ull * n);
   return EDP_OK;
 }
 
@@ -1119,9 +1237,12 @@ edp_status edp_gae_stats(edp_ctx *ctx, const float *r, const float *v, const uin
   if (!all_device(ctx, {r, v, d, adv, ret, d_stats}))
     return fail(ctx, EDP_ERR_INVALID, "edp_gae_stats: arrays must be device memory");
   DeviceGuard dg(ctx->cfg.device);
+  EDP_TRACE(__func__);
   cudaError_t e = launch_gae_stats(ctx, r, v, d, T, E, gamma, lambda, adv, ret, d_stats,
                                    (cudaStream_t)stream);
   if (e != cudaSuccess) return launch_fail(ctx, e, "edp_gae_stats");
+  const uint64_t te = (uint64_t)T * E;
+  count_hbm(ctx, 9 * te + 4ull * E, 4 * te * (1 + (ret != nullptr)) + 24);
   return EDP_OK;
 }
 
@@ -1133,8 +1254,10 @@ edp_status edp_gae_normalize(edp_ctx *ctx, const float *adv, uint64_t n, const d
   if (!adv || !d_stats || !adv_norm || !all_device(ctx, {adv, d_stats, adv_norm}))
     return fail(ctx, EDP_ERR_INVALID, "edp_gae_normalize: arrays must be device memory");
   DeviceGuard dg(ctx->cfg.device);
+  EDP_TRACE(__func__);
   cudaError_t e = launch_gae_normalize(ctx, adv, n, d_stats, adv_norm, (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_gae_normalize");
+  count_hbm(ctx, 4 * n + 24, 4 * n);
   return EDP_OK;
 }
 
@@ -1151,8 +1274,10 @@ edp_status edp_grpo_advantage(edp_ctx *ctx, const float *r, const uint64_t *grou
     if (!device_view(ctx, o, &p, false))
       return fail(ctx, EDP_ERR_INVALID, "edp_grpo_advantage: arrays must be device memory");
   DeviceGuard dg(ctx->cfg.device);
+  EDP_TRACE(__func__);
   cudaError_t e = launch_grpo(ctx, r, group_off, n_groups, eps, adv, (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_grpo_advantage");
+  count_hbm(ctx, 8ull * (n_groups + 1), 0);  // the reward count is known on the device only
   return EDP_OK;
 }
 
@@ -1182,10 +1307,14 @@ edp_status edp_pack_deliver(edp_ctx *ctx, const int32_t *tokens, const uint64_t 
     o = const_cast<void *>(p);
   }
   DeviceGuard dg(ctx->cfg.device);
+  EDP_TRACE(__func__);
   cudaError_t e = launch_pack(ctx, tokens, seq_off, n_seq, idx, batch, seq_value,
                               (int32_t *)outs[0], (uint64_t *)outs[1], (float *)outs[2],
                               out_cap, (cudaStream_t)stream);
   if (e != cudaSuccess) return launch_fail(ctx, e, "edp_pack_deliver");
+  count_hbm(ctx, 24ull * batch, 0);  // indices and sequence offsets; tokens not counted
+  count_write(ctx, out_off, 8ull * (batch + 1));
+  ctx->cnt.delivered += batch;
   return EDP_OK;
 }
 
@@ -1219,16 +1348,52 @@ edp_status edp_grpo_pack_deliver(edp_ctx *ctx, const float *r, const uint64_t *g
     o = const_cast<void *>(p);
   }
   DeviceGuard dg(ctx->cfg.device);
+  EDP_TRACE(__func__);
   cudaError_t e = launch_grpo_pack(ctx, r, group_off, n_groups, eps, adv, tokens, seq_off,
                                    n_seq, idx, batch, (int32_t *)outs[0], (uint64_t *)outs[1],
                                    (float *)outs[2], out_cap, (cudaStream_t)stream);
   if (e != cudaSuccess) return launch_fail(ctx, e, "edp_grpo_pack_deliver");
+  count_hbm(ctx, 8ull * (n_groups + 1) + 24ull * batch, 0);
+  count_write(ctx, out_off, 8ull * (batch + 1));
+  ctx->cnt.delivered += batch;
+  return EDP_OK;
+}
+
+edp_status edp_get_counters(edp_ctx *ctx, edp_counters *out) {
+  if (!ctx || !out) return EDP_ERR_INVALID;
+  *out = ctx->cnt;
+  if (ctx->cap_c) {  // two-tier: the host-tier bytes the deliveries counted
+    DeviceGuard dg(ctx->cfg.device);
+    unsigned long long hb = 0;
+    const cudaError_t e = cudaMemcpy(&hb, &ctx->ctrl->host_bytes, sizeof hb,
+                                     cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_get_counters");
+    uint64_t d = hb - ctx->host_bytes_base;
+    if (d > out->hbm_read) d = out->hbm_read;
+    out->hbm_read -= d;
+    out->link_read += d;
+  }
+  return EDP_OK;
+}
+
+edp_status edp_reset_counters(edp_ctx *ctx) {
+  if (!ctx) return EDP_ERR_INVALID;
+  ctx->cnt = edp_counters{};
+  if (ctx->cap_c) {
+    DeviceGuard dg(ctx->cfg.device);
+    unsigned long long hb = 0;
+    const cudaError_t e = cudaMemcpy(&hb, &ctx->ctrl->host_bytes, sizeof hb,
+                                     cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_reset_counters");
+    ctx->host_bytes_base = hb;
+  }
   return EDP_OK;
 }
 
 edp_status edp_sync(edp_ctx *ctx, edp_stream stream) {
   if (!ctx) return EDP_ERR_INVALID;
   DeviceGuard dg(ctx->cfg.device);
+  EDP_TRACE(__func__);
   cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
   if (e == cudaSuccess) e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(ctx, e, "edp_sync");

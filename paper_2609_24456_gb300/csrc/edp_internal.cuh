@@ -8,6 +8,8 @@
 
 #include <string>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "edp.h"
 
 namespace edp {
@@ -32,6 +34,7 @@ struct Ctrl {
   uint32_t pack_ticket;  // packed delivery: length CTAs done (calls are ordered)
   uint32_t pad;
   unsigned long long bad_index;  // first offending index (diagnostics)
+  unsigned long long host_bytes;  // two-tier deliveries: bytes read from the host tier
 };
 
 constexpr int kFanout = 32;
@@ -71,6 +74,8 @@ struct edp_ctx {
   float naff_a[4] = {}, naff_b[4] = {};
   int norm_affine = 0;
   int coop_sms = 0;
+  edp_counters cnt{};  // host-side traffic counters (edp_get_counters)
+  uint64_t host_bytes_base = 0;  // the device's host-tier byte count at the last reset
   std::string err;
 };
 
@@ -533,11 +538,39 @@ class DeviceGuard {
   bool switched_ = false;
 };
 
+// Host-side NVTX range (domain "libedp") spanning an entry point's enqueue
+// work, so a timeline tool shows each call beside the kernels it launched.
+// The NVTX calls are no-ops unless a tool is attached.
+class TraceRange {
+ public:
+  explicit TraceRange(const char *name) {
+    nvtxEventAttributes_t a = {};
+    a.version = NVTX_VERSION;
+    a.size = NVTX_EVENT_ATTRIB_STRUCT_SIZE;
+    a.messageType = NVTX_MESSAGE_TYPE_ASCII;
+    a.message.ascii = name;
+    nvtxDomainRangePushEx(domain(), &a);
+  }
+  ~TraceRange() { nvtxDomainRangePop(domain()); }
+  TraceRange(const TraceRange &) = delete;
+  TraceRange &operator=(const TraceRange &) = delete;
+
+ private:
+  static nvtxDomainHandle_t domain() {
+    static const nvtxDomainHandle_t d = nvtxDomainCreateA("libedp");
+    return d;
+  }
+};
+#define EDP_TRACE(name) ::edp::TraceRange edp_trace_range_(name)
+
 // Resolve a caller pointer to a device-usable address.  Device memory of the
 // context's GPU passes through; page-locked host memory is translated to its
 // mapped device address when allow_host; pageable or foreign memory is
 // rejected (false).
 bool device_view(const edp_ctx *c, const void *p, const void **out, bool allow_host);
+
+// true for page-locked host memory (reached over the host link)
+bool host_memory(const void *p);
 
 // Record a printf-style message as the context's last error; returns s.
 edp_status fail(edp_ctx *c, edp_status s, const char *fmt, ...);

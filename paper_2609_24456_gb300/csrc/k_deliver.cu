@@ -727,6 +727,10 @@ k_deliver_norm(Common c, NormArgs a) {
       }
     }
     if (head) {
+      // a two-tier row read over the host link (edp_get_counters)
+      if (lane == 0 && ok && a.obs_c && !hbm)
+        atomicAdd(&c.ctrl->host_bytes,
+                  (unsigned long long)a.F8 * 8ull + (a.tok_out ? a.L16 * 16ull : 0ull));
       if (a.tok_out) {
         const uint4 *ts = reinterpret_cast<const uint4 *>(
             (hbm ? a.tok_h : a.tok_c) + ps * a.L16 * 4ull);

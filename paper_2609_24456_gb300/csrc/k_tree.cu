@@ -553,6 +553,7 @@ extern "C" edp_status edp_update_priorities_td_static(
   if (ctx->cfg.device < 0 || ctx->cfg.device >= kMaxDevices)
     return fail(ctx, EDP_ERR_INVALID, "%s: device ordinal out of range", who);
   DeviceGuard dg(ctx->cfg.device);
+  EDP_TRACE(who);
   uint32_t *qbuf = nullptr;
   cudaError_t e = static_qbuf(ctx->cfg.device, &qbuf);
   if (e != cudaSuccess) {

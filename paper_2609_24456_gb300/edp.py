@@ -124,6 +124,8 @@ SIGNATURES = {
     "edp_gae_stats": (C.c_int, [_VP, _VP, _VP, _VP, _U32, _U32, _D, _D, _VP, _VP, _VP,
                                 _VP]),
     "edp_gae_normalize": (C.c_int, [_VP, _VP, _U64, _VP, _VP, _VP]),
+    "edp_get_counters": (C.c_int, [_VP, _VP]),
+    "edp_reset_counters": (C.c_int, [_VP]),
     "edp_sync": (C.c_int, [_VP, _VP]),
     "edp_last_error": (C.c_char_p, [_VP]),
     "edp_get_info": (C.c_int, [_VP, C.POINTER(edp_info)]),
@@ -317,6 +319,22 @@ def edp_gae_stats(ctx, r, v, d, T, E, gamma, lam, adv, stats, ret=None, stream=N
 def edp_gae_normalize(ctx, adv, n, stats, adv_norm, stream=None):
     return _check(ctx, lib().edp_gae_normalize(ctx, ptr(adv), n, ptr(stats), ptr(adv_norm),
                                                stream_handle(stream)), "edp_gae_normalize")
+
+
+class edp_counters(C.Structure):
+    _fields_ = [("calls", _U64), ("ingested", _U64), ("sampled", _U64), ("delivered", _U64),
+                ("hbm_read", _U64), ("hbm_write", _U64), ("link_read", _U64),
+                ("link_write", _U64)]
+
+
+def edp_get_counters(ctx) -> dict:
+    out = edp_counters()
+    _check(ctx, lib().edp_get_counters(ctx, C.byref(out)), "edp_get_counters")
+    return {name: getattr(out, name) for name, _ in edp_counters._fields_}
+
+
+def edp_reset_counters(ctx):
+    return _check(ctx, lib().edp_reset_counters(ctx), "edp_reset_counters")
 
 
 def edp_sync(ctx, stream=None):

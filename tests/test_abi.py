@@ -47,7 +47,7 @@ def test_struct_layouts_match_binding(tmp_path):
                "edp_info": edp.edp_info, "edp_sched_costs": edp.edp_sched_costs,
                "edp_sched_choice": edp.edp_sched_choice,
                "edp_place_option": edp.edp_place_option,
-               "edp_place_bw": edp.edp_place_bw}
+               "edp_place_bw": edp.edp_place_bw, "edp_counters": edp.edp_counters}
     lines = ['#include <stdio.h>', '#include <stddef.h>', '#include "edp.h"',
              "int main(void) {"]
     for sname, cls in structs.items():
