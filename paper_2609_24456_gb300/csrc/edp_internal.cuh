@@ -335,7 +335,9 @@ __device__ __forceinline__ bool mbar_wait(unsigned long long *bar, uint32_t pari
   if (mbar_test(bar, parity)) return true;
   const uint64_t t0 = global_ns();
   for (;;) {
-    for (int i = 0; i < 8; ++i)  // a try_wait may itself suspend the thread
+    // the timer is read once per 64 tests: reading it more often slows the
+    // waiting warps measurably (a stage's consumers poll the barrier)
+    for (int i = 0; i < 64; ++i)
       if (mbar_test(bar, parity)) return true;
     if (global_ns() - t0 > limit_ns) return false;
   }
