@@ -1775,7 +1775,9 @@ def run_reference(args):
             "impl": "reference", "n_gpus": args.gpus, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": dt * 1e3 / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-            "dtype": wl.dtype, "data": "synthetic", "config": wl.config(),
+            "dtype": wl.dtype, "data": "synthetic",
+            "config": dict(wl.config(), parallelism="replicas%d" % int(
+                os.environ.get("WORLD_SIZE", "1"))),
             "cpu_baseline": {"value": gbs, "unit": "GB/s", "cores": cores,
                              "kind": "oracle", "sample": wl.cpu_sample},
             "e2e": {"value": gbs, "unit": "GB/s", "h2d_bytes_per_step": 0,
@@ -1957,11 +1959,12 @@ def run_edp(args):
                 "unit": "GB/s", "n_gpus": world, "steps": K, "warmup": W,
                 "ms_per_step": ms_step, "higher_is_better": True,
                 "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype,
-                "data": "synthetic", "config": dict(wl.config(),
-                                                    parallelism=("sharded%d" if sharded
-                                                                 else "replicas%d") % world,
-                                                    graph=use_graph,
-                                                    schedule="%s: %s" % scheds[0][::2]),
+                "data": "synthetic",
+                # the workload alone, as the reference arm prints it; how it
+                # ran goes beside it
+                "config": dict(wl.config(), parallelism=("sharded%d" if sharded
+                                                         else "replicas%d") % world),
+                "schedule": "%s: %s" % scheds[0][::2], "graph": use_graph,
                 "pct_hbm_peak": 100.0 * value / peak,
                 "batches_per_s": K * world / (ms / 1e3),
                 "p50_sample_to_batch_us": p50,
