@@ -10,6 +10,8 @@
    targets never decrease, so grouping them by owner keeps stratum order.
    Checked with the oracle's sampler, target rule and Philox on random
    shards, including empty shards and zero priorities.
+3. A rank that leaves between rounds: the survivor's next exchange ends in
+   an error within the process group's timeout, not in an endless wait.
 """
 import os
 import socket
@@ -126,3 +128,43 @@ def test_routing_by_shard_prefix_is_the_global_inverse_cdf(orc, case):
         assert offsets[owner] + local == g_idx[k]
         assert shards[owner][local] == g_q[k]
     assert owners == sorted(owners)  # grouped by owner, stratum order kept
+
+
+def _dying_rank(rank, world, port, out):
+    import datetime
+    import torch
+    import torch.distributed as dist
+    sys.path.insert(0, ROOT)
+    from paper_2609_24456_gb300.shard import ShardComm
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world,
+                            timeout=datetime.timedelta(seconds=5))
+    c = ShardComm()
+    c.all_gather(torch.tensor([rank]))  # one exchange that both ranks make
+    if rank == 1:
+        os._exit(0)  # leaves between exchanges, without a word
+    try:
+        c.all_gather(torch.tensor([rank]))  # the next round's first exchange
+        out.put("no error")
+    except Exception as e:  # the peer's departure surfaces here
+        out.put("error: %s" % type(e).__name__)
+
+
+@pytest.mark.timeout(120)
+def test_a_rank_that_leaves_between_rounds_is_detected():
+    """A rank that exits between two rounds (no kernel or collective of
+    its own in flight) makes the other rank's next exchange fail with an
+    error instead of waiting forever: the process group's timeout bounds
+    it.  Host-side failure detection for the sharded buffer."""
+    world = 2
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_dying_rank, args=(r, world, port, q)) for r in range(world)]
+    for p in procs:
+        p.start()
+    res = q.get(timeout=100)
+    for p in procs:
+        p.join(timeout=30)
+    assert res.startswith("error"), res
