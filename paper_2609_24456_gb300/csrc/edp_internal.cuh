@@ -225,6 +225,58 @@ __device__ __forceinline__ double pow_pos(double x, double a) {
   return q * __longlong_as_double((ni + 1023) << 52);
 }
 
+// Double-float arithmetic: a value is an unevaluated sum hi + lo of two
+// fp32 numbers (about 48 significant bits), with Knuth's TwoSum, Dekker's
+// product via FMA and the renormalisations of Hida, Li and Bailey.  Every
+// operation is one IEEE rounding: the intrinsics are never contracted or
+// reassociated by the compiler.
+struct df {
+  float hi, lo;
+};
+__device__ __forceinline__ df two_sum(float a, float b) {
+  const float s = __fadd_rn(a, b);
+  const float bb = __fsub_rn(s, a);
+  const float e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
+  return {s, e};
+}
+__device__ __forceinline__ df quick_two_sum(float a, float b) {  // |a| >= |b|
+  const float s = __fadd_rn(a, b);
+  return {s, __fsub_rn(b, __fsub_rn(s, a))};
+}
+__device__ __forceinline__ df df_add(df a, df b) {
+  df s = two_sum(a.hi, b.hi);
+  const df t = two_sum(a.lo, b.lo);
+  s.lo = __fadd_rn(s.lo, t.hi);
+  s = quick_two_sum(s.hi, s.lo);
+  s.lo = __fadd_rn(s.lo, t.lo);
+  return quick_two_sum(s.hi, s.lo);
+}
+__device__ __forceinline__ df df_add_f(df a, float b) {
+  df s = two_sum(a.hi, b);
+  s.lo = __fadd_rn(s.lo, a.lo);
+  return quick_two_sum(s.hi, s.lo);
+}
+__device__ __forceinline__ df df_mul(df a, df b) {
+  const float p = __fmul_rn(a.hi, b.hi);
+  float e = __fmaf_rn(a.hi, b.hi, -p);
+  e = __fmaf_rn(a.hi, b.lo, e);
+  e = __fmaf_rn(a.lo, b.hi, e);
+  return quick_two_sum(p, e);
+}
+__device__ __forceinline__ df df_mul_f(df a, float b) {
+  const float p = __fmul_rn(a.hi, b);
+  float e = __fmaf_rn(a.hi, b, -p);
+  e = __fmaf_rn(a.lo, b, e);
+  return quick_two_sum(p, e);
+}
+__device__ __forceinline__ df df_split(double x) {
+  const float hi = (float)x;
+  return {hi, (float)(x - (double)hi)};
+}
+__device__ __forceinline__ double df_to_d(df a) {
+  return (double)a.hi + (double)a.lo;
+}
+
 // Importance weight (q_min / q_k)^beta in fp64, one rounding to fp32 (PER:
 // (N P(i))^-beta over its batch maximum, in which N and the total cancel).
 __device__ __forceinline__ float is_weight(uint32_t m, uint32_t qk, double beta) {
@@ -364,7 +416,12 @@ __device__ __forceinline__ void flag(Ctrl *c, uint32_t bits,
 // writes are visible, so every such kernel calls it before touching memory
 // the predecessor may write.  pdl_launch() lets the next kernel in the
 // stream start launching.  Both are no-ops for a kernel launched without
-// the attribute.
+// the attribute.  The samplers, small grids that a one-wave delivery grid
+// follows, call pdl_launch() at their end: triggered at their start, the
+// delivery's CTAs are placed while the sampler's CTAs still hold their SMs,
+// and the block scheduler packs them onto the other SMs up to the occupancy
+// limit (304 CTAs on 88 of the 152 SMs), leaving the rest idle for the
+// whole delivery.
 __device__ __forceinline__ void pdl_wait() {
   asm volatile("griddepcontrol.wait;" ::: "memory");
 }

@@ -41,58 +41,9 @@ constexpr int kGaeWarps = 4;   // environments per CTA
 constexpr int kGaeThreads = kGaeWarps * 32;
 constexpr int kNormThreads = 256;
 
-// ---- double-float arithmetic (every operation one IEEE rounding: the
-// intrinsics are never contracted or reassociated by the compiler)
-struct df {
-  float hi, lo;
-};
-__device__ __forceinline__ df two_sum(float a, float b) {
-  const float s = __fadd_rn(a, b);
-  const float bb = __fsub_rn(s, a);
-  const float e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
-  return {s, e};
-}
-__device__ __forceinline__ df quick_two_sum(float a, float b) {  // |a| >= |b|
-  const float s = __fadd_rn(a, b);
-  return {s, __fsub_rn(b, __fsub_rn(s, a))};
-}
-__device__ __forceinline__ df df_add(df a, df b) {
-  df s = two_sum(a.hi, b.hi);
-  const df t = two_sum(a.lo, b.lo);
-  s.lo = __fadd_rn(s.lo, t.hi);
-  s = quick_two_sum(s.hi, s.lo);
-  s.lo = __fadd_rn(s.lo, t.lo);
-  return quick_two_sum(s.hi, s.lo);
-}
-__device__ __forceinline__ df df_add_f(df a, float b) {
-  df s = two_sum(a.hi, b);
-  s.lo = __fadd_rn(s.lo, a.lo);
-  return quick_two_sum(s.hi, s.lo);
-}
-__device__ __forceinline__ df df_mul(df a, df b) {
-  const float p = __fmul_rn(a.hi, b.hi);
-  float e = __fmaf_rn(a.hi, b.hi, -p);
-  e = __fmaf_rn(a.hi, b.lo, e);
-  e = __fmaf_rn(a.lo, b.hi, e);
-  return quick_two_sum(p, e);
-}
-__device__ __forceinline__ df df_mul_f(df a, float b) {
-  const float p = __fmul_rn(a.hi, b);
-  float e = __fmaf_rn(a.hi, b, -p);
-  e = __fmaf_rn(a.lo, b, e);
-  return quick_two_sum(p, e);
-}
 __device__ __forceinline__ df df_shfl_down(df a, int o) {
   return {__shfl_down_sync(kFull, a.hi, o), __shfl_down_sync(kFull, a.lo, o)};
 }
-__device__ __forceinline__ df df_split(double x) {
-  const float hi = (float)x;
-  return {hi, (float)(x - (double)hi)};
-}
-__device__ __forceinline__ double df_to_d(df a) {
-  return (double)a.hi + (double)a.lo;
-}
-
 // One environment's scan (one warp): writes its advantages and returns and
 // adds this lane's A and A^2 to s1, s2.
 __device__ __forceinline__ void gae_env(const float *__restrict__ r,

@@ -24,12 +24,12 @@ __global__ void k_sample_uniform(uint32_t B, uint64_t seed, uint64_t round,
                                  uint64_t n_valid, uint64_t oldest,
                                  uint64_t cap, int64_t *__restrict__ idx) {
   pdl_wait();
-  pdl_launch();
   for (uint32_t k = blockIdx.x * blockDim.x + threadIdx.x; k < B;
        k += gridDim.x * blockDim.x) {
     const uint64_t off = mulhi64(philox_u64(seed, k, round, 0), n_valid);
     idx[k] = (int64_t)((oldest + off) % cap);
   }
+  pdl_launch();  // at the end: see pdl_launch()
 }
 
 constexpr int kPermThreads = 256;

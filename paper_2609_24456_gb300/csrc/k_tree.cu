@@ -131,7 +131,6 @@ k_sample_prio(TreeView t, uint32_t B, uint64_t seed, uint64_t round,
   const int lane = threadIdx.x & 31;
   const uint64_t keep = policy_keep();
   pdl_wait();
-  pdl_launch();
   const uint64_t S = t.nodes[0];  // issued beside the loads of the top levels
   const uint32_t cached = cache_top(t, top, keep);
   __syncthreads();
@@ -155,6 +154,7 @@ k_sample_prio(TreeView t, uint32_t B, uint64_t seed, uint64_t round,
       if (qout) qout[k] = t.leaves[node];
     }
   }
+  pdl_launch();  // at the end: see pdl_launch()
 }
 
 // Descent of given targets (the shard side of a sharded buffer: targets
@@ -168,7 +168,6 @@ k_sample_targets(TreeView t, const uint64_t *__restrict__ targets, uint32_t n,
   const int lane = threadIdx.x & 31;
   const uint64_t keep = policy_keep();
   pdl_wait();
-  pdl_launch();
   const uint64_t S = t.nodes[0];  // issued beside the loads of the top levels
   const uint32_t cached = cache_top(t, top, keep);
   __syncthreads();
@@ -191,26 +190,138 @@ k_sample_targets(TreeView t, const uint64_t *__restrict__ targets, uint32_t n,
       if (qout) qout[k] = t.leaves[node];
     }
   }
+  pdl_launch();  // at the end: see pdl_launch()
 }
 
 // PER priority from a TD error: clamp(rn((|td| + eps)^alpha * 2^20), 1,
-// 2^32 - 1), fp64.
-__device__ __forceinline__ uint32_t prio_td(float td, double alpha, double eps) {
-  const double x = fabs((double)td) + eps;
-  double p = (x > 1e-300 && x < 1e300) ? pow_pos<true>(x, alpha) * 1048576.0
-                                       : pow(x, alpha) * 1048576.0;
+// 2^32 - 1) (the rule is defined in fp64).  The exponent, eps and the
+// constants of the fast path travel as double-float splits made on the host.
+struct PrioRule {
+  double alpha, eps;
+  float a_hi, a_lo, e_hi, e_lo;
+  int fast;  // alpha in (0, 1], eps in [0, 2^90]: the double-float path applies
+};
+
+PrioRule prio_rule(double alpha, double eps) {
+  PrioRule r{};
+  r.alpha = alpha;
+  r.eps = eps;
+  r.a_hi = (float)alpha;
+  r.a_lo = (float)(alpha - (double)r.a_hi);
+  r.e_hi = (float)eps;
+  r.e_lo = (float)(eps - (double)r.e_hi);
+  r.fast = alpha > 0.0 && alpha <= 1.0 && eps >= 0.0 && eps <= 0x1p90;
+  return r;
+}
+
+// x^a * 2^20 for x in [2^-100, 2^100] and a in (0, 1], rounded to the nearest
+// integer and clamped, in double-float arithmetic.  An fp64 instruction
+// occupies this GPU's fp64 pipe for about 64 cycles whatever the number of
+// active lanes, so the fp64 evaluation of the rule costs ~4,000 cycles per
+// warp; this one issues fp32 and integer work only.
+//   log: x = 2^e m with m in [sqrt(1/2), sqrt(2)); ln m = 2 atanh(s),
+//   s = (m - 1)/(m + 1), |s| <= 0.1716, by its series through s^17 (the
+//   terms beyond s^7 in fp32: they are below 2^-17 relative to the sum);
+//   exp: Cody and Waite's reduction t = n ln 2 + r, |r| <= ln(2)/2, with
+//   ln 2 split into three floats (the first with 15 significant bits, so
+//   that n times it is exact), and Taylor's series of e^r through r^12
+//   (terms from r^7 on in fp32).
+// Relative error below 2^-40: against the fp64 rule evaluated with the C
+// library's pow, the integer differs in about one case per million, by one.
+constexpr double kLn2 = 0.69314718055994530942;
+constexpr float kLn2A = 0.693145751953125f;  // 0x3f317200
+constexpr float kLn2B = (float)(kLn2 - (double)kLn2A);
+constexpr float kLn2C = (float)(kLn2 - (double)kLn2A - (double)kLn2B);
+#define EDP_DF_CONST(v) df{(float)(v), (float)((v) - (double)(float)(v))}
+
+__device__ __forceinline__ df df_div(df a, df b) {
+  const float q1 = __fdiv_rn(a.hi, b.hi);
+  df r = df_add(a, df_mul_f(b, -q1));
+  const float q2 = __fdiv_rn(r.hi, b.hi);
+  r = df_add(r, df_mul_f(b, -q2));
+  const float q3 = __fdiv_rn(r.hi, b.hi);
+  return df_add_f(quick_two_sum(q1, q2), q3);
+}
+
+__device__ __forceinline__ df df_two_prod(float a, float b) {
+  const float p = __fmul_rn(a, b);
+  return {p, __fmaf_rn(a, b, -p)};
+}
+
+__device__ __forceinline__ uint32_t prio_df(df x, df a) {
+  const int bits = __float_as_int(x.hi);
+  int e = ((bits >> 23) & 0xff) - 127;
+  if ((bits & 0x7fffff) > 0x3504f3) e += 1;  // mantissa above sqrt(2)
+  const float sc = __int_as_float((127 - e) << 23);
+  const df m{__fmul_rn(x.hi, sc), __fmul_rn(x.lo, sc)};
+  const df s = df_div(df_add_f(m, -1.0f), df_add_f(m, 1.0f));
+  const df s2 = df_mul(s, s);
+  float tail = 1.0f / 17;
+  tail = __fmaf_rn(tail, s2.hi, 1.0f / 15);
+  tail = __fmaf_rn(tail, s2.hi, 1.0f / 13);
+  tail = __fmaf_rn(tail, s2.hi, 1.0f / 11);
+  tail = __fmaf_rn(tail, s2.hi, 1.0f / 9);
+  df p = df_add(EDP_DF_CONST(1.0 / 7), df_mul_f(s2, tail));
+  p = df_add(EDP_DF_CONST(1.0 / 5), df_mul(s2, p));
+  p = df_add(EDP_DF_CONST(1.0 / 3), df_mul(s2, p));
+  p = df_add_f(df_mul(s2, p), 1.0f);
+  df lnm = df_mul(s, p);
+  lnm.hi = __fmul_rn(lnm.hi, 2.0f);
+  lnm.lo = __fmul_rn(lnm.lo, 2.0f);
+  const float ef = (float)e;
+  df el{__fmul_rn(ef, kLn2A), 0.0f};
+  el = df_add(el, df_two_prod(ef, kLn2B));
+  el = df_add_f(el, __fmul_rn(ef, kLn2C));
+  const df t = df_mul(a, df_add(el, lnm));
+  const float nf = rintf(__fmul_rn(t.hi, 1.44269504f));
+  df r = df_add_f(t, -__fmul_rn(nf, kLn2A));
+  r = df_add(r, df_two_prod(-nf, kLn2B));
+  r = df_add_f(r, -__fmul_rn(nf, kLn2C));
+  float qt = 1.0f / 479001600;
+  qt = __fmaf_rn(qt, r.hi, 1.0f / 39916800);
+  qt = __fmaf_rn(qt, r.hi, 1.0f / 3628800);
+  qt = __fmaf_rn(qt, r.hi, 1.0f / 362880);
+  qt = __fmaf_rn(qt, r.hi, 1.0f / 40320);
+  qt = __fmaf_rn(qt, r.hi, 1.0f / 5040);
+  df q = df_add(EDP_DF_CONST(1.0 / 720), df_mul_f(r, qt));
+  q = df_add(EDP_DF_CONST(1.0 / 120), df_mul(r, q));
+  q = df_add(EDP_DF_CONST(1.0 / 24), df_mul(r, q));
+  q = df_add(EDP_DF_CONST(1.0 / 6), df_mul(r, q));
+  q = df_add_f(df_mul(r, q), 0.5f);
+  q = df_add_f(df_mul(r, q), 1.0f);
+  q = df_add_f(df_mul(r, q), 1.0f);
+  const float sc2 = __int_as_float((127 + (int)nf + 20) << 23);  // 2^(n + 20)
+  const float vh = __fmul_rn(q.hi, sc2), vl = __fmul_rn(q.lo, sc2);
+  if (vh >= 4294967296.0f) return 0xffffffffu;
+  const float rh = rintf(vh);
+  const float d = __fadd_rn(__fsub_rn(vh, rh), vl);
+  long long res = (long long)rh + (long long)rintf(d);
+  if (res < 1) res = 1;
+  if (res > 4294967295ll) res = 4294967295ll;
+  return (uint32_t)res;
+}
+#undef EDP_DF_CONST
+
+__device__ __forceinline__ uint32_t prio_td(float td, const PrioRule &rule) {
+  if (rule.fast) {
+    const df x = df_add_f(df{rule.e_hi, rule.e_lo}, fabsf(td));
+    if (x.hi >= 0x1p-100f && x.hi <= 0x1p100f) return prio_df(x, df{rule.a_hi, rule.a_lo});
+  }
+  // the fp64 evaluation: exponents outside (0, 1], and arguments far from 1
+  const double x = fabs((double)td) + rule.eps;
+  double p = (x > 1e-300 && x < 1e300) ? pow_pos<true>(x, rule.alpha) * 1048576.0
+                                       : pow(x, rule.alpha) * 1048576.0;
   double r = rint(p);
   if (!(r >= 1.0)) r = 1.0;
   if (r > 4294967295.0) r = 4294967295.0;
   return (uint32_t)r;
 }
 
-__global__ void k_prio_from_td(const float *__restrict__ td, uint32_t n,
-                               double alpha, double eps,
+__global__ void k_prio_from_td(const float *__restrict__ td, uint32_t n, PrioRule rule,
                                uint32_t *__restrict__ q) {
   for (uint32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < n;
        i += gridDim.x * blockDim.x)
-    q[i] = prio_td(td[i], alpha, eps);
+    q[i] = prio_td(td[i], rule);
 }
 
 constexpr int kUpdThreads = 512;
@@ -226,7 +337,8 @@ __device__ __forceinline__ uint32_t tab_hash(uint32_t x, uint32_t mask) {
   return x & mask;
 }
 
-// Priority update.  Phase 1 (all CTAs): the priority of every pair -- the
+// Priority update of a large batch (more than kUpdSmallMax pairs; smaller
+// ones take k_update_small below).  Phase 1 (all CTAs): the priority of every pair -- the
 // given u32, or PER's rule from the TD error, whose fp64 pow is spread over
 // the CTAs -- goes to qbuf.  The last CTA to finish (ticket counter, no
 // waiting) then applies the pairs in batch order, in chunks of 1024 (two
@@ -239,7 +351,7 @@ __device__ __forceinline__ uint32_t tab_hash(uint32_t x, uint32_t mask) {
 __global__ void __launch_bounds__(kUpdThreads, 1)
 k_update(TreeView t, const int64_t *__restrict__ idx,
          const uint32_t *__restrict__ q, const float *__restrict__ td,
-         uint32_t *__restrict__ qbuf, double alpha, double eps, uint32_t n,
+         uint32_t *__restrict__ qbuf, PrioRule rule, uint32_t n,
          uint64_t cap, uint64_t oldest, uint64_t size, int defer, Ctrl *ctrl) {
   __shared__ uint32_t hkey[kUpdTable];
   __shared__ uint32_t hpos[kUpdTable];
@@ -257,7 +369,7 @@ k_update(TreeView t, const int64_t *__restrict__ idx,
     // spreads over SMs
     if (threadIdx.x < 32)
       for (uint32_t p = blockIdx.x * 32 + threadIdx.x; p < n; p += gridDim.x * 32)
-        qbuf[p] = prio_td(td[p], alpha, eps);
+        qbuf[p] = prio_td(td[p], rule);
     __threadfence();
     __syncthreads();
     if (threadIdx.x == 0) ticket = atomicAdd(&ctrl->upd_count, 1u);
@@ -393,6 +505,119 @@ k_update(TreeView t, const int64_t *__restrict__ idx,
   }
 }
 
+// Priority update of a small batch (n <= kUpdSmallMax pairs): one CTA per 32
+// pairs and a single pass, with no ticket and no second phase.  Each CTA
+// stages the slots of the whole batch in shared memory and checks, for each
+// of its own 32 pairs, whether a later pair of the batch sets the same slot
+// (the table warps split the batch between them; every comparison reads one
+// broadcast word).  The pairs that are the last occurrence of their slot
+// write their leaves and add their exact deltas to the ancestors with
+// atomics: each slot has exactly one writer in the batch, and integer sums
+// do not depend on the order of the additions, so the tree equals the one
+// the sequential application gives.  Warp 0 holds the CTA's pairs and
+// evaluates their priorities meanwhile.
+constexpr int kUpdSmallMax = 2048;
+constexpr int kUpdSmallThreads = 256;
+constexpr int kUpdScan = kUpdSmallThreads - 32;                        // scanning threads
+constexpr int kUpdScanPer = (kUpdSmallMax + kUpdScan - 1) / kUpdScan;  // slots each loads
+
+__global__ void __launch_bounds__(kUpdSmallThreads)
+k_update_small(TreeView t, const int64_t *__restrict__ idx,
+               const uint32_t *__restrict__ q, const float *__restrict__ td,
+               PrioRule rule, uint32_t n, uint64_t cap, uint64_t oldest,
+               uint64_t size, int defer, Ctrl *ctrl) {
+  __shared__ uint32_t bkey[kUpdSmallMax];  // slot of each pair, kEmpty if it sets none
+  __shared__ uint32_t later;               // bit l: a later pair sets pair l's slot
+  __shared__ unsigned long long acc1[32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const uint32_t p0 = blockIdx.x * 32, p = p0 + lane;  // warp 0's pair
+  pdl_wait();
+  pdl_launch();
+  int64_t sl = -1;
+  uint64_t k = 0;
+  bool holds = false;
+  uint32_t qv = 0, old = 0;
+  if (warp == 0) {
+    float tdv = 0.f;
+    if (p < n) {
+      sl = idx[p];
+      if (td) tdv = td[p];
+      else qv = q[p];
+      const bool valid = sl >= 0 && (uint64_t)sl < cap;
+      if (!valid) flag(ctrl, DEVERR_INDEX, (unsigned long long)sl);
+      k = !valid ? 0
+          : (uint64_t)sl >= oldest ? (uint64_t)sl - oldest : (uint64_t)sl + cap - oldest;
+      holds = valid && k < size;  // the slot holds a transition
+      if (holds) old = t.leaves[sl];
+    }
+    if (holds && td) qv = prio_td(tdv, rule);
+    if (!holds) qv = 0;
+  } else {
+    // the slots of the whole batch, every load in flight at once
+    const uint32_t f = threadIdx.x - 32;
+#pragma unroll
+    for (int j = 0; j < kUpdScanPer; ++j) {
+      const uint32_t i = f + j * kUpdScan;
+      if (i < n) {
+        const int64_t s2 = idx[i];
+        uint32_t key = kEmpty;
+        if (s2 >= 0 && (uint64_t)s2 < cap) {
+          const uint64_t k2 = (uint64_t)s2 >= oldest ? (uint64_t)s2 - oldest
+                                                     : (uint64_t)s2 + cap - oldest;
+          if (k2 < size) key = (uint32_t)s2;
+        }
+        bkey[i] = key;
+      }
+    }
+    if (f == 0) later = 0;
+    asm volatile("bar.sync 1, %0;" :: "r"(kUpdScan) : "memory");
+    // warp w - 1 of the scanning warps compares the CTA's pairs (one per
+    // lane) with pairs [j0, j1) of the batch after them
+    const uint32_t mine = p < n ? bkey[p] : kEmpty;
+    const uint32_t per = (n + (kUpdScan / 32) - 1) / (kUpdScan / 32);
+    uint32_t j = (warp - 1) * per;
+    const uint32_t j1 = min(n, j + per);
+    if (j <= p) j = p + 1;
+    bool dup = false;
+    for (; j + 4 <= j1; j += 4)
+      dup |= (bkey[j] == mine) | (bkey[j + 1] == mine) | (bkey[j + 2] == mine) |
+             (bkey[j + 3] == mine);
+    for (; j < j1; ++j) dup |= bkey[j] == mine;
+    const unsigned m = __ballot_sync(kFull, dup && mine != kEmpty);
+    if (lane == 0 && m) atomicOr(&later, m);
+  }
+  __syncthreads();
+  if (warp != 0) return;
+  bool win = holds && !((later >> lane) & 1u);  // no later pair sets this slot
+  if (win && defer && k == size - 1) {
+    ctrl->pending_q = qv;
+    win = false;
+  }
+  unsigned long long delta = 0;
+  if (win) {
+    t.leaves[sl] = qv;
+    delta = (unsigned long long)((long long)qv - (long long)old);
+  }
+  if (delta)
+    for (uint32_t d = 2; d < t.depth; ++d)
+      atomicAdd((unsigned long long *)&t.lvl(d)[(uint64_t)sl >> (5 * (t.depth - d))], delta);
+  if (t.depth >= 2) {  // level 1 (32 nodes): the warp's deltas per node first
+    acc1[lane] = 0;
+    __syncwarp();
+    if (delta) atomicAdd(&acc1[(uint64_t)sl >> (5 * (t.depth - 1))], delta);
+    __syncwarp();
+    if (acc1[lane]) atomicAdd((unsigned long long *)&t.lvl(1)[lane], acc1[lane]);
+  }
+  const unsigned long long root = warp_sum_u64(delta);
+  uint32_t qmax = qv;  // 0 for a pair that sets no leaf
+#pragma unroll
+  for (int o = 16; o; o >>= 1) qmax = max(qmax, __shfl_xor_sync(kFull, qmax, o));
+  if (lane == 0) {
+    if (root) atomicAdd((unsigned long long *)&t.nodes[0], root);
+    if (qmax) atomicMax(&ctrl->max_q, qmax);
+  }
+}
+
 }  // namespace
 
 void tree_ranges(const edp_ctx *c, uint64_t first, uint64_t count, TreeRanges *out) {
@@ -471,6 +696,10 @@ cudaError_t launch_update(edp_ctx *c, const int64_t *idx, const uint32_t *q,
                           cudaStream_t s) {
   const uint64_t size = c->total < c->cap ? c->total : c->cap;
   const uint64_t oldest = (c->total - size) % c->cap;
+  if (n <= (uint32_t)kUpdSmallMax)
+    return launch_pdl(k_update_small, dim3((n + 31) / 32), dim3(kUpdSmallThreads), s,
+                      view(c), idx, q, td, prio_rule(alpha, eps), n, c->cap, oldest,
+                      size, c->defer, c->ctrl);
   uint32_t *qbuf = nullptr;
   unsigned grid = 1;
   if (td) {
@@ -481,24 +710,25 @@ cudaError_t launch_update(edp_ctx *c, const int64_t *idx, const uint32_t *q,
     if (grid > 2u * (unsigned)c->coop_sms) grid = 2u * (unsigned)c->coop_sms;
   }
   return launch_pdl(k_update, dim3(grid), dim3(kUpdThreads), s, view(c), idx, q,
-                    td, qbuf, alpha, eps, n, c->cap, oldest, size, c->defer,
+                    td, qbuf, prio_rule(alpha, eps), n, c->cap, oldest, size, c->defer,
                     c->ctrl);
 }
 
 cudaError_t launch_prio_from_td(const float *td, uint32_t n, double alpha,
                                 double eps, uint32_t *q, cudaStream_t s) {
   const unsigned blocks = (n + 255) / 256 < 1024 ? (n + 255) / 256 : 1024;
-  k_prio_from_td<<<blocks, 256, 0, s>>>(td, n, alpha, eps, q);
+  k_prio_from_td<<<blocks, 256, 0, s>>>(td, n, prio_rule(alpha, eps), q);
   return cudaGetLastError();
 }
 
 }  // namespace edp
 
 // ---------------------------------------------------------------------------
-// Allocation-free priority update.  Same kernel as edp_update_priorities_td,
-// but the per-pair priorities computed from the TD errors go to the fixed
-// array below instead of context-owned scratch that is allocated on first
-// use.  Callers that must not allocate device memory use it: code being
+// Allocation-free priority update.  Same kernels as edp_update_priorities_td:
+// up to 2,048 pairs the single-pass kernel, which needs no memory beyond
+// its arguments; above that the two-phase kernel, whose per-pair priorities
+// computed from the TD errors go to the fixed array below instead of
+// context-owned scratch that is allocated on first use.  Callers that must not allocate device memory use it: code being
 // captured into a CUDA graph (cudaMalloc may not be called during stream
 // capture), and runtimes that hand out all device memory up front and forbid
 // allocation later, or that cannot afford the device-wide synchronisation a
@@ -554,20 +784,31 @@ extern "C" edp_status edp_update_priorities_td_static(
     return fail(ctx, EDP_ERR_INVALID, "%s: device ordinal out of range", who);
   DeviceGuard dg(ctx->cfg.device);
   EDP_TRACE(who);
+  const uint64_t size = ctx->total < ctx->cap ? ctx->total : ctx->cap;
+  const uint64_t oldest = (ctx->total - size) % ctx->cap;
+  cudaError_t e;
+  if (n <= (uint32_t)kUpdSmallMax) {  // needs no priority array
+    e = launch_pdl(k_update_small, dim3((n + 31) / 32), dim3(kUpdSmallThreads),
+                   (cudaStream_t)stream, view(ctx), idx, (const uint32_t *)nullptr, td,
+                   prio_rule(alpha, eps), n, ctx->cap, oldest, size, ctx->defer, ctx->ctrl);
+    if (e != cudaSuccess) {
+      cudaGetLastError();
+      return fail(ctx, EDP_ERR_CUDA, "%s: %s", who, cudaGetErrorString(e));
+    }
+    return EDP_OK;
+  }
   uint32_t *qbuf = nullptr;
-  cudaError_t e = static_qbuf(ctx->cfg.device, &qbuf);
+  e = static_qbuf(ctx->cfg.device, &qbuf);
   if (e != cudaSuccess) {
     cudaGetLastError();
     return fail(ctx, EDP_ERR_CUDA, "%s: cudaGetSymbolAddress: %s", who,
                 cudaGetErrorString(e));
   }
-  const uint64_t size = ctx->total < ctx->cap ? ctx->total : ctx->cap;
-  const uint64_t oldest = (ctx->total - size) % ctx->cap;
   unsigned grid = (n + 31) / 32;
   if (grid > 2u * (unsigned)ctx->coop_sms) grid = 2u * (unsigned)ctx->coop_sms;
   e = launch_pdl(k_update, dim3(grid), dim3(kUpdThreads), (cudaStream_t)stream,
-                 view(ctx), idx, (const uint32_t *)nullptr, td, qbuf, alpha, eps, n,
-                 ctx->cap, oldest, size, ctx->defer, ctx->ctrl);
+                 view(ctx), idx, (const uint32_t *)nullptr, td, qbuf, prio_rule(alpha, eps),
+                 n, ctx->cap, oldest, size, ctx->defer, ctx->ctrl);
   if (e != cudaSuccess) {
     cudaGetLastError();
     return fail(ctx, EDP_ERR_CUDA, "%s: %s", who, cudaGetErrorString(e));

@@ -173,6 +173,29 @@ def test_priorities_from_td_within_one(edp_lib, orc):
     assert u32(qe).tolist() == [1, 2**32 - 1, 2**32 - 1, 1]
 
 
+@pytest.mark.parametrize("alpha,eps", [(1.0, 0.0), (0.05, 1e-6), (0.4, 1e-2),
+                                       (1.5, 1e-6), (0.0, 1e-6)])
+def test_priorities_from_td_other_exponents(edp_lib, orc, alpha, eps):
+    """The rule at other exponents and offsets: (0, 1] takes the
+    double-float evaluation, 0 and exponents above 1 the fp64 one; errors
+    from 1e-30 to 3e38 (beyond 2^100 the fp64 one again).  Within one of
+    the oracle, and rarely off by one (an exponent of 1 with no offset
+    makes exact ties, which a rounding step may resolve either way)."""
+    edp = edp_lib
+    m = MirroredDqn(64, prioritized=True)
+    rng = np.random.default_rng(int(alpha * 100) + int(eps * 1e6))
+    td = np.exp(rng.uniform(np.log(1e-30), np.log(3e38), 1 << 18)).astype(np.float32)
+    td[: 1 << 17] = fx.td_errors(6, 1 << 17)
+    td *= np.where(rng.random(len(td)) < 0.5, -1, 1).astype(np.float32)
+    q = torch.zeros(len(td), dtype=torch.int32, device="cuda")
+    edp.edp_priorities_from_td(m.ring.ctx, cuda(td), len(td), alpha, eps, q)
+    edp.edp_sync(m.ring.ctx)
+    ref = orc.priorities_from_td(td, alpha, eps).astype(np.int64)
+    diff = np.abs(u32(q).astype(np.int64) - ref)
+    assert diff.max() <= 1
+    assert (diff > 0).mean() < 1e-3
+
+
 def test_all_zero_priorities_report_empty(edp_lib, orc):
     edp = edp_lib
     m = MirroredDqn(40, prioritized=True)
