@@ -571,18 +571,20 @@ k_update_small(TreeView t, const int64_t *__restrict__ idx,
     }
     if (f == 0) later = 0;
     asm volatile("bar.sync 1, %0;" :: "r"(kUpdScan) : "memory");
-    // warp w - 1 of the scanning warps compares the CTA's pairs (one per
-    // lane) with pairs [j0, j1) of the batch after them
+    // scanning warp w - 1 compares the CTA's pairs (one per lane) with the
+    // later pairs among [j0, j1); every lane reads the same word (a
+    // broadcast), and the loop is the same for all lanes
     const uint32_t mine = p < n ? bkey[p] : kEmpty;
     const uint32_t per = (n + (kUpdScan / 32) - 1) / (kUpdScan / 32);
-    uint32_t j = (warp - 1) * per;
-    const uint32_t j1 = min(n, j + per);
-    if (j <= p) j = p + 1;
+    const uint32_t j0 = (warp - 1) * per;
+    const uint32_t j1 = min(n, j0 + per);
+    uint32_t j = max(j0, p0 + 1);
     bool dup = false;
-    for (; j + 4 <= j1; j += 4)
-      dup |= (bkey[j] == mine) | (bkey[j + 1] == mine) | (bkey[j + 2] == mine) |
-             (bkey[j + 3] == mine);
-    for (; j < j1; ++j) dup |= bkey[j] == mine;
+    for (; j + 8 <= j1; j += 8) {
+#pragma unroll
+      for (int u = 0; u < 8; ++u) dup |= (bkey[j + u] == mine) & (j + u > p);
+    }
+    for (; j < j1; ++j) dup |= (bkey[j] == mine) & (j > p);
     const unsigned m = __ballot_sync(kFull, dup && mine != kEmpty);
     if (lane == 0 && m) atomicOr(&later, m);
   }
@@ -598,15 +600,18 @@ k_update_small(TreeView t, const int64_t *__restrict__ idx,
     t.leaves[sl] = qv;
     delta = (unsigned long long)((long long)qv - (long long)old);
   }
-  if (delta)
-    for (uint32_t d = 2; d < t.depth; ++d)
-      atomicAdd((unsigned long long *)&t.lvl(d)[(uint64_t)sl >> (5 * (t.depth - d))], delta);
+  if (delta) {
+    uint64_t first = 33;  // level d starts at node (32^d - 1) / 31
+    for (uint32_t d = 2; d < t.depth; ++d, first = first * 32 + 1)
+      atomicAdd((unsigned long long *)&t.nodes[first + ((uint64_t)sl >> (5 * (t.depth - d)))],
+                delta);
+  }
   if (t.depth >= 2) {  // level 1 (32 nodes): the warp's deltas per node first
     acc1[lane] = 0;
     __syncwarp();
     if (delta) atomicAdd(&acc1[(uint64_t)sl >> (5 * (t.depth - 1))], delta);
     __syncwarp();
-    if (acc1[lane]) atomicAdd((unsigned long long *)&t.lvl(1)[lane], acc1[lane]);
+    if (acc1[lane]) atomicAdd((unsigned long long *)&t.nodes[1 + lane], acc1[lane]);
   }
   const unsigned long long root = warp_sum_u64(delta);
   uint32_t qmax = qv;  // 0 for a pair that sets no leaf
