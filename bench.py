@@ -406,6 +406,17 @@ class PerReplay(Workload):
         self.td = torch.stack([dev(fx.td_errors(self.seed, B, r), device)
                                for r in range(self.td_rounds)])
         self._init_overlap(device, self.R)
+        # index sets for the kernel's back-to-back timing: a fresh sample for
+        # each launch (64 sets, ~18 MB of distinct frames each), so that no
+        # launch finds an earlier launch's frames in L2
+        self.fresh = []
+        for k in range(64):
+            idx = torch.empty(B, dtype=torch.int64, device=device)
+            q = torch.empty(B, dtype=torch.int32, device=device)
+            edp.edp_sample(ctx, edp.EDP_SAMPLE_PRIORITIZED, B, self.seed + 1, k, idx, q)
+            o = self.outs[k % self.R]
+            self.fresh.append((idx, q, edp.make_batch(o["obs"], o["nxt"], o["act"], o["rew"],
+                                                      o["done"], q=q, isw=o["isw"], beta=BETA)))
 
     def _sample(self, r, o):
         self.edp.edp_sample(self.ring.ctx, self.edp.EDP_SAMPLE_PRIORITIZED, self.B,
@@ -445,8 +456,8 @@ class PerReplay(Workload):
                 ("serial", self.round, "sample -> deliver -> update, one stream")]
 
     def deliver_once(self, r):
-        o = self.outs[r % self.R]
-        self.edp.edp_deliver(self.ring.ctx, o["idx"], self.B, o["batch"])
+        idx, _, batch = self.fresh[r % len(self.fresh)]
+        self.edp.edp_deliver(self.ring.ctx, idx, self.B, batch)
 
     def extra(self, device, mk, stream, deliver_us):
         """Ingestion (row a1) on this ring, timed after everything else: 4,096
