@@ -188,30 +188,52 @@ struct MetaArgs {
   int defer;
 };
 
-// Transitions j = j0, j0 + stride, ... of the insertion.
+// Transitions j = j0, j0 + stride, ... of the insertion, kMetaBatch at a
+// time: the batch's source loads are all issued before its stores (a store
+// to the ring could alias a source as far as the compiler knows, so loads
+// interleaved with stores would each wait a round trip).
+constexpr int kMetaBatch = 4;
 __device__ __forceinline__ void ingest_meta_range(const MetaArgs &a, uint64_t j0,
                                                   uint64_t stride) {
   uint32_t qdefault = 0;
   if (a.leaves && !a.q) qdefault = a.ctrl->max_q;
   uint32_t qmax_local = 0;  // one atomic per warp, not per transition
-  for (uint64_t j = j0; j < a.n; j += stride) {
-    const uint64_t m = (a.total + j) % a.cap;
-    if (a.action) a.action[m] = a.s_action ? a.s_action[j] : 0;
-    if (a.reward) a.reward[m] = a.s_reward ? a.s_reward[j] : 0.f;
-    if (a.done) a.done[m] = a.s_done ? a.s_done[j] : (uint8_t)0;
-    if (a.leaves) {
-      const uint32_t qj = a.q ? a.q[j] : qdefault;
-      if (a.q) qmax_local = max(qmax_local, qj);
-      if (a.defer) {
-        a.leaves[m] = (j == a.n - 1) ? 0u : qj;
-        if (j == 0) {
-          // only this thread touches pending_q and the previous newest leaf
-          if (a.total >= 1 && a.n < a.cap)
-            a.leaves[(a.total - 1) % a.cap] = a.ctrl->pending_q;
-          a.ctrl->pending_q = a.q ? a.q[a.n - 1] : qdefault;
+  for (uint64_t jb = j0; jb < a.n; jb += kMetaBatch * stride) {
+    int32_t act[kMetaBatch];
+    float rew[kMetaBatch];
+    uint8_t dn[kMetaBatch];
+    uint32_t qs[kMetaBatch];
+#pragma unroll
+    for (int b = 0; b < kMetaBatch; ++b) {
+      const uint64_t j = jb + b * stride;
+      const bool in = j < a.n;
+      act[b] = in && a.s_action ? a.s_action[j] : 0;
+      rew[b] = in && a.s_reward ? a.s_reward[j] : 0.f;
+      dn[b] = in && a.s_done ? a.s_done[j] : (uint8_t)0;
+      qs[b] = in && a.q ? a.q[j] : qdefault;
+    }
+#pragma unroll
+    for (int b = 0; b < kMetaBatch; ++b) {
+      const uint64_t j = jb + b * stride;
+      if (j >= a.n) break;
+      const uint64_t m = (a.total + j) % a.cap;
+      if (a.action) a.action[m] = act[b];
+      if (a.reward) a.reward[m] = rew[b];
+      if (a.done) a.done[m] = dn[b];
+      if (a.leaves) {
+        const uint32_t qj = qs[b];
+        if (a.q) qmax_local = max(qmax_local, qj);
+        if (a.defer) {
+          a.leaves[m] = (j == a.n - 1) ? 0u : qj;
+          if (j == 0) {
+            // only this thread touches pending_q and the previous newest leaf
+            if (a.total >= 1 && a.n < a.cap)
+              a.leaves[(a.total - 1) % a.cap] = a.ctrl->pending_q;
+            a.ctrl->pending_q = a.q ? a.q[a.n - 1] : qdefault;
+          }
+        } else {
+          a.leaves[m] = qj;
         }
-      } else {
-        a.leaves[m] = qj;
       }
     }
   }
