@@ -304,17 +304,23 @@ class Workload:
         return e0.elapsed_time(e1) * 1e3 / n
 
     def time_latency(self, n, mk, stream):
-        """Sample -> batch latency (us) of n steps, events around each."""
+        """Sample -> batch latency (us) of n steps: the time on the device
+        from an event before the step's first call to one after its batch
+        is complete.  Each step is queued behind a short spin kernel, so the
+        host has submitted all of the step before the device reaches it:
+        the events time the step's kernels and their launches, not the
+        host's submission of the calls (nor the event nodes of a graph,
+        which split it)."""
         import torch
-        evs = [(mk(), mk()) for _ in range(n)]
-        g = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g, capture_error_mode="thread_local"):
-            for r in range(n):
-                evs[r][0].record()
-                self.latency_step(100000 + r, evs[r][1])
-        g.replay()
-        torch.cuda.synchronize()
-        return [a.elapsed_time(b) * 1e3 for a, b in evs]
+        out = []
+        for r in range(n):
+            e0, e1 = mk(), mk()
+            torch.cuda._sleep(200000)  # ~0.1 ms at 2 GHz: the host queues the step meanwhile
+            e0.record(stream)
+            self.latency_step(100000 + r, e1)
+            torch.cuda.synchronize()
+            out.append(e0.elapsed_time(e1) * 1e3)
+        return out
 
 
 def _stack_bytes(B, K, F, next_obs=True):
