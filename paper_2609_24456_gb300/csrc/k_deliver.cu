@@ -732,11 +732,23 @@ k_deliver_norm(Common c, NormArgs a) {
         atomicAdd(&c.ctrl->host_bytes,
                   (unsigned long long)a.F8 * 8ull + (a.tok_out ? a.L16 * 16ull : 0ull));
       if (a.tok_out) {
+        // the row's tokens, kTokBatch 16-byte loads per lane in flight
+        // before their stores
+        constexpr int kTokBatch = 4;
         const uint4 *ts = reinterpret_cast<const uint4 *>(
             (hbm ? a.tok_h : a.tok_c) + ps * a.L16 * 4ull);
         uint4 *td = reinterpret_cast<uint4 *>(a.tok_out + (uint64_t)k * a.L16 * 4ull);
-        for (uint32_t i = lane; i < a.L16; i += 32)
-          td[i] = ok ? ts[i] : make_uint4(0u, 0u, 0u, 0u);
+        for (uint32_t i0 = lane; i0 < a.L16; i0 += 32 * kTokBatch) {
+          uint4 t4[kTokBatch];
+#pragma unroll
+          for (int u = 0; u < kTokBatch; ++u) {
+            const uint32_t i = i0 + u * 32;
+            t4[u] = (ok && i < a.L16) ? ts[i] : make_uint4(0u, 0u, 0u, 0u);
+          }
+#pragma unroll
+          for (int u = 0; u < kTokBatch; ++u)
+            if (i0 + u * 32 < a.L16) td[i0 + u * 32] = t4[u];
+        }
       }
     }
     f = seg_end;
