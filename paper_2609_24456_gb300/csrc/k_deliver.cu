@@ -33,15 +33,15 @@ namespace {
 constexpr unsigned kFull = 0xffffffffu;
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
-// loads in flight per lane (8 x 8 bytes) in the normalising delivery
-constexpr int kNormUnroll = 8;
+// loads in flight per lane (6 x 8 bytes) in the normalising delivery
+constexpr int kNormUnroll = 6;
 
 // unrolled rows per warp iteration and iterations per warp (chunk span) of
 // each kernel
 constexpr int kStackUnroll = 4;
 constexpr int kStackMinBlocks = 6;  // __launch_bounds__: at most 40 registers
 constexpr int kHwcUnroll = 2, kHwcIters = 2;
-constexpr int kNormIters = 3;
+constexpr int kNormIters = 2;
 
 struct Common {
   const int64_t *idx;
