@@ -151,6 +151,44 @@ def test_update_batch_sizes(edp_lib, orc, n, path):
         check_tree(orc, m.ring, m.st)
 
 
+def test_small_updates_queued_back_to_back(edp_lib, orc):
+    """Single-pass updates (up to 2,048 pairs) queued straight after each
+    other on one stream, with nothing between them: each waits for the one
+    before, so the later batch wins on the slots both touch.  Four calls
+    (TD errors and u32 priorities, 2,048 / 513 / 32 / 1 pairs, many shared
+    slots and the deferred newest one), then the whole tree bit-exact."""
+    edp = edp_lib
+    cap = 3000
+    frames, action, reward, done = fx.dqn_transitions(17, 2600, 84 * 4)
+    q0 = orc.priorities_from_td(fx.td_errors(17, 2600), ALPHA, EPS)
+    m = MirroredDqn(cap, prioritized=True, F=84 * 4)
+    m.ingest(orc, frames, action, reward, done, q=q0)
+    rng = np.random.default_rng(18)
+    calls = []
+    for k, n in enumerate((2048, 513, 32, 1)):
+        idx = rng.integers(0, 300, size=n).astype(np.int64)  # shared slots
+        idx[n // 2] = m.total - 1  # the newest (deferred) transition
+        if k % 2 == 0:
+            td = (rng.standard_normal(n) * 2).astype(np.float32)
+            d_td = cuda(td)
+            qd = torch.zeros(n, dtype=torch.int32, device="cuda")
+            edp.edp_priorities_from_td(m.ring.ctx, d_td, n, ALPHA, EPS, qd)
+            calls.append((cuda(idx), d_td, None, n, idx, qd))
+        else:
+            qu = rng.integers(1, 1 << 31, size=n).astype(np.uint32)
+            calls.append((cuda(idx), None, cuda(qu.view(np.int32)), n, idx, qu))
+    torch.cuda.synchronize()
+    for d_idx, d_td, d_q, n, _, _ in calls:
+        if d_td is not None:
+            edp.edp_update_priorities_td(m.ring.ctx, d_idx, d_td, n, ALPHA, EPS)
+        else:
+            edp.edp_update_priorities(m.ring.ctx, d_idx, d_q, n)
+    edp.edp_sync(m.ring.ctx)
+    for _, _, _, _, idx, q in calls:
+        orc.update_leaves(m.st, m.total, idx, u32(q) if torch.is_tensor(q) else q)
+    check_tree(orc, m.ring, m.st)
+
+
 def test_priorities_from_td_within_one(edp_lib, orc):
     edp = edp_lib
     m = MirroredDqn(64, prioritized=True)
