@@ -151,6 +151,38 @@ def test_update_batch_sizes(edp_lib, orc, n, path):
         check_tree(orc, m.ring, m.st)
 
 
+@pytest.mark.parametrize("cap", [20, 33, 500])
+@pytest.mark.parametrize("path", ["u32", "td"])
+def test_update_shallow_trees(edp_lib, orc, cap, path):
+    """Trees of depth 1 (20 leaves under the root), 2 (33 and 500 leaves):
+    the single-pass update's level-1 and root sums on their own, batches of
+    1 to 300 pairs with repeats, slots that hold nothing and the deferred
+    newest transition; the whole tree bit-exact after each."""
+    edp = edp_lib
+    n_in = cap - 3
+    frames, action, reward, done = fx.dqn_transitions(23, n_in, 84 * 4)
+    q0 = orc.priorities_from_td(fx.td_errors(23, n_in), ALPHA, EPS)
+    m = MirroredDqn(cap, prioritized=True, F=84 * 4)
+    m.ingest(orc, frames, action, reward, done, q=q0)
+    rng = np.random.default_rng(cap * 7 + (path == "td"))
+    for n in (1, 7, 40, 300):
+        idx = rng.integers(0, cap, size=n).astype(np.int64)  # cap - 3 .. hold nothing
+        idx[n // 2] = m.total - 1
+        if path == "u32":
+            qu = rng.integers(0, 1 << 31, size=n).astype(np.uint32)
+            edp.edp_update_priorities(m.ring.ctx, cuda(idx), cuda(qu), n)
+        else:
+            d_td = cuda((rng.standard_normal(n) * 3).astype(np.float32))
+            qd = torch.zeros(n, dtype=torch.int32, device="cuda")
+            edp.edp_priorities_from_td(m.ring.ctx, d_td, n, ALPHA, EPS, qd)
+            edp.edp_update_priorities_td(m.ring.ctx, cuda(idx), d_td, n, ALPHA, EPS)
+            edp.edp_sync(m.ring.ctx)
+            qu = u32(qd)
+        orc.update_leaves(m.st, m.total, idx, qu)
+        edp.edp_sync(m.ring.ctx)
+        check_tree(orc, m.ring, m.st)
+
+
 def test_small_updates_queued_back_to_back(edp_lib, orc):
     """Single-pass updates (up to 2,048 pairs) queued straight after each
     other on one stream, with nothing between them: each waits for the one
