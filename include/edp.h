@@ -309,8 +309,11 @@ EDP_API edp_status edp_update_priorities(edp_ctx *ctx, const int64_t *idx,
                                  edp_stream stream);
 
 /* Same, from TD errors: q = clamp(rn((|td| + eps)^alpha * 2^20), 1,
- * 2^32-1) computed in fp64 on the device.  pow is not correctly rounded, so
- * q may differ by 1 from a host evaluation. */
+ * 2^32-1), the rule defined in fp64.  For alpha in (0, 1] and |td| + eps in
+ * [2^-100, 2^100] the device evaluates it in double-float arithmetic
+ * (relative error below 2^-40), otherwise in fp64; neither is correctly
+ * rounded, so q may differ by 1 from a host evaluation (about one case in
+ * a million).  Batches of up to 2048 pairs need no scratch. */
 EDP_API edp_status edp_update_priorities_td(edp_ctx *ctx, const int64_t *idx,
                                     const float *td, uint32_t n, double alpha,
                                     double eps, edp_stream stream);
@@ -321,10 +324,10 @@ EDP_API edp_status edp_update_priorities_td(edp_ctx *ctx, const int64_t *idx,
  * CUDA graph, where cudaMalloc may not be called, and runtimes that hand out
  * all device memory at start-up and forbid later allocation, or cannot
  * afford the device-wide synchronisation an allocation may bring.
- * edp_update_priorities_td allocates its scratch (one uint32 per pair) on
- * first use; this variant keeps that scratch in a fixed per-device array of
- * 16384 pairs (64 KiB), held by every GPU that loads libedp until the process
- * exits.  n > 16384 returns EDP_ERR_INVALID.  The first call on a device
+ * Above 2048 pairs edp_update_priorities_td allocates its scratch (one
+ * uint32 per pair) on first use; this variant keeps that scratch in a fixed
+ * per-device array of 16384 pairs (64 KiB), held by every GPU that loads
+ * libedp until the process exits.  n > 16384 returns EDP_ERR_INVALID.  The first call on a device
  * looks up the array's device address (make it before any stream capture).
  * All calls on a device share the array.  Calls queued on one stream are
  * ordered (a call touches the array only after the previous kernel on its
