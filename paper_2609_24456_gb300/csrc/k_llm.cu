@@ -24,7 +24,7 @@ constexpr unsigned kFull = 0xffffffffu;
 constexpr int kGrpoThreads = 64;
 constexpr int kGrpoWarps = kGrpoThreads / 32;
 constexpr int kPackThreads = 256;
-constexpr int kPackUnroll = 8;
+constexpr uint64_t kPackWaitNs = 1000000000ull;  // bound of the gather's wait for its copy
 constexpr uint32_t kDirectChunks = 256;  // chunk sums a gather CTA adds itself
 static_assert(kDirectChunks <= kPackThreads, "a gather CTA adds one chunk sum per thread");
 
@@ -205,15 +205,30 @@ __device__ __forceinline__ void st_stream32(void *p, uint32_t v, uint64_t pol) {
 
 // One CTA per sequence: its output offset is the prefix of its 256-entry
 // chunk (from `pre`, or the chunk sums before it) plus the lengths before it
-// in the chunk (one round trip and a block sum), then a thread keeps
-// kPackUnroll loads in flight (2,048 tokens per CTA pass).  The CTA of the
-// last entry writes out_off[batch] = the total and flags an overflow.
-__global__ void __launch_bounds__(kPackThreads, 8)  // 32 registers: 8 CTAs per SM
+// in the chunk (one round trip and a block sum).  The tokens then move in
+// chunks of up to kPackChunk: the source's 16-byte-aligned interior by one
+// bulk copy into shared memory (completion on an mbarrier, waited for with a
+// bound), its up to three unaligned tokens at either end by plain loads;
+// the destination's aligned interior by 16-byte stores read from shared
+// memory at the offset between the two alignments, its ends by 4-byte
+// stores.  The per-token value is a fill with the same split, written while
+// the copy is in flight.  The CTA of the last entry writes out_off[batch] =
+// the total and flags an overflow.
+constexpr uint32_t kPackChunk = 4096;  // tokens per bulk copy (16 KB of shared memory)
+__global__ void __launch_bounds__(kPackThreads, 6)  // 36 registers, 16.5 KB: 6 CTAs per SM
 k_pack_gather(const int32_t *__restrict__ tokens, const PackEntry *__restrict__ ent,
               const uint64_t *__restrict__ part, const uint64_t *__restrict__ pre, uint32_t B,
               const float *__restrict__ sv, int32_t *__restrict__ otok,
               uint64_t *__restrict__ ooff, float *__restrict__ osv, uint64_t cap, Ctrl *ctrl) {
   __shared__ uint64_t red[kPackThreads / 32];
+  __shared__ alignas(16) uint32_t tbuf[kPackChunk + 8];
+  __shared__ unsigned long long bar;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    mbar_init_fence();
+  }
+  __syncthreads();
+  uint32_t uses = 0;  // completed phases of bar
   const uint64_t pol = policy_stream();
   pdl_wait();
   pdl_launch();
@@ -240,22 +255,62 @@ k_pack_gather(const int32_t *__restrict__ tokens, const PackEntry *__restrict__ 
     const uint64_t n = min((uint64_t)e.len, cap - dst);
     const int32_t *src = tokens + e.src;
     int32_t *out = otok + dst;
-    for (uint64_t t0 = threadIdx.x; t0 < n; t0 += kPackThreads * kPackUnroll) {
-      int32_t w[kPackUnroll];
-#pragma unroll
-      for (int u = 0; u < kPackUnroll; ++u) {
-        const uint64_t t = t0 + u * kPackThreads;
-        w[u] = t < n ? (int32_t)ld_stream(reinterpret_cast<const uint32_t *>(src + t), pol)
-                     : 0;
+    float *vout = osv ? osv + dst : nullptr;
+    const uint32_t vbits = __float_as_uint(value);
+    for (uint64_t c0 = 0; c0 < n; c0 += kPackChunk) {
+      const uint32_t m = (uint32_t)min((uint64_t)kPackChunk, n - c0);
+      const int32_t *sc = src + c0;
+      // source: tokens [0, head) and [head + body, m) by plain loads, the
+      // 16-byte-aligned [head, head + body) by one bulk copy; token t sits at
+      // tbuf[t + shift], which puts token `head` on a 16-byte boundary
+      const uint32_t hs = (uint32_t)(((16u - ((uint32_t)(uintptr_t)sc & 15u)) & 15u) >> 2);
+      const uint32_t head = min(hs, m);
+      const uint32_t body = (m - head) & ~3u;
+      const uint32_t shift = (4u - head) & 3u;
+      if (threadIdx.x == 0 && body) {
+        // the previous chunk's reads of tbuf (generic proxy) come before
+        // this copy's writes (async proxy)
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        mbar_arrive_tx(&bar, body * 4);
+        bulk_load(&tbuf[head + shift], sc + head, body * 4, &bar, pol);
       }
-#pragma unroll
-      for (int u = 0; u < kPackUnroll; ++u) {
-        const uint64_t t = t0 + u * kPackThreads;
-        if (t < n) {
-          st_stream32(out + t, (uint32_t)w[u], pol);
-          if (osv) st_stream32(osv + dst + t, __float_as_uint(value), pol);
+      const uint32_t tail0 = head + body;
+      if (threadIdx.x < head) tbuf[threadIdx.x + shift] = (uint32_t)sc[threadIdx.x];
+      if (threadIdx.x < m - tail0)
+        tbuf[tail0 + threadIdx.x + shift] = (uint32_t)sc[tail0 + threadIdx.x];
+      // values: the same split on the destination
+      if (vout) {
+        float *vo = vout + c0;
+        const uint32_t hv = min((uint32_t)(((16u - ((uint32_t)(uintptr_t)vo & 15u)) & 15u) >> 2), m);
+        const uint32_t qv = (m - hv) >> 2;
+        if (threadIdx.x < hv) st_stream32(vo + threadIdx.x, vbits, pol);
+        const uint4 v4 = make_uint4(vbits, vbits, vbits, vbits);
+        for (uint32_t i = threadIdx.x; i < qv; i += kPackThreads)
+          st_stream(reinterpret_cast<uint4 *>(vo + hv) + i, v4, pol);
+        const uint32_t tv = hv + 4 * qv;
+        if (threadIdx.x < m - tv) st_stream32(vo + tv + threadIdx.x, vbits, pol);
+      }
+      if (body) {
+        if (!mbar_wait(&bar, uses & 1u, kPackWaitNs)) {
+          if (threadIdx.x == 0) flag(ctrl, DEVERR_TIMEOUT, k);
+          mbar_wait(&bar, uses & 1u, kPackWaitNs);  // bounded: the copy lands first
         }
+        ++uses;
       }
+      __syncthreads();
+      // destination: 16-byte stores of its aligned interior
+      int32_t *oc = out + c0;
+      const uint32_t ho = min((uint32_t)(((16u - ((uint32_t)(uintptr_t)oc & 15u)) & 15u) >> 2), m);
+      const uint32_t q = (m - ho) >> 2;
+      if (threadIdx.x < ho) st_stream32(oc + threadIdx.x, tbuf[threadIdx.x + shift], pol);
+      for (uint32_t i = threadIdx.x; i < q; i += kPackThreads) {
+        const uint32_t t = ho + 4 * i + shift;
+        st_stream(reinterpret_cast<uint4 *>(oc + ho) + i,
+                  make_uint4(tbuf[t], tbuf[t + 1], tbuf[t + 2], tbuf[t + 3]), pol);
+      }
+      const uint32_t to = ho + 4 * q;
+      if (threadIdx.x < m - to) st_stream32(oc + to + threadIdx.x, tbuf[to + threadIdx.x + shift], pol);
+      __syncthreads();  // tbuf is refilled by the next chunk
     }
   }
 }
