@@ -134,6 +134,45 @@ def test_pack_unaligned_outputs(edp_lib, tok_shift, val_shift):
     assert np.isnan(to_np(base_v[:val_shift])).all() and np.isnan(to_np(base_v[val_shift + n:])).all()
 
 
+@pytest.mark.parametrize("shift", [0, 1, 3])
+def test_pack_long_sequences(edp_lib, shift):
+    """Sequences longer than one 4,096-token bulk copy (4,095 .. 10,000
+    tokens, several chunks each) among short ones, from sources at every
+    alignment, into an output starting 0, 4 or 12 bytes past a 16-byte
+    boundary; then the same batch cut by out_cap inside the second chunk of
+    a long sequence."""
+    edp = edp_lib
+    ring = _ctx(edp)
+    from oracle import llm
+    lens = np.array([4095, 1, 4096, 3, 4097, 5, 8191, 2, 8192, 10000, 0, 7], np.uint64)
+    seq_off = np.concatenate([[0], np.cumsum(lens)]).astype(np.uint64)
+    rng = np.random.default_rng(40 + shift)
+    tokens = rng.integers(0, 152064, size=int(seq_off[-1]), dtype=np.int32)
+    value = rng.standard_normal(len(lens)).astype(np.float32)
+    idx = np.concatenate([rng.permutation(len(lens)), [9, 6]]).astype(np.int64)
+    ref, ref_off, ref_v = llm.pack(tokens, seq_off, idx, value)
+    n = len(ref)
+    for cap in (n, int(ref_off[list(idx).index(9)]) + 4096 + 1001):
+        base_t = torch.full((n + 8,), -7, dtype=torch.int32, device="cuda")
+        base_v = torch.full((n + 8,), float("nan"), device="cuda")
+        out, ov = base_t[shift:shift + cap], base_v[shift:shift + cap]
+        ooff = torch.full((len(idx) + 1,), -1, dtype=torch.int64, device="cuda")
+        edp.edp_pack_deliver(ring.ctx, cuda(tokens), cuda(seq_off), len(lens), cuda(idx),
+                             len(idx), out, ooff, cap, seq_value=cuda(value), out_value=ov)
+        if cap < n:
+            with pytest.raises(edp.EdpError) as e:
+                edp.edp_sync(ring.ctx)
+            assert str(n) in str(e.value)
+        else:
+            edp.edp_sync(ring.ctx)
+        assert np.array_equal(to_np(ooff).view(np.uint64), ref_off)
+        assert np.array_equal(to_np(out), ref[:cap])
+        assert np.array_equal(bits(ov), ref_v[:cap].view(np.uint32))
+        # nothing written past the output or before it
+        assert (to_np(base_t[:shift]) == -7).all() and (to_np(base_t[shift + cap:]) == -7).all()
+        assert np.isnan(to_np(base_v[:shift])).all() and np.isnan(to_np(base_v[shift + cap:])).all()
+
+
 def test_pack_invalid_index_and_overflow(edp_lib):
     edp = edp_lib
     ring = _ctx(edp)
